@@ -1,0 +1,219 @@
+/*
+ * gc.h — C ABI of libgc: prefix-reuse prefill on one GB300 GPU (sm_103a).
+ *
+ * The operation is the data-plane step of context caching described in
+ * arXiv 2505.23970, Sec. 2.2 ("Caching for LLM Serving", Fig. 2a): when a
+ * request's context is found in the cache, its KV cache is loaded back into
+ * GPU memory, the KV of the new tokens is stitched after it, and the new
+ * tokens are prefilled against [cached context ++ new tokens] instead of
+ * recomputing the whole context.  Sec. 2.1 defines the KV cache as the keys
+ * and values of processed tokens kept for reuse.  The three calls below are
+ * that step:
+ *
+ *   gc_kv_restore           cached pages (pinned host or device staging)
+ *                           -> paged HBM KV pool                  (load)
+ *   gc_kv_append            new tokens' K,V -> pool slots after each
+ *                           request's cached prefix                (stitch)
+ *   gc_prefix_prefill_attn  causal GQA attention of the new tokens over
+ *                           the pool through a block table         (prefill)
+ *
+ * Conventions for every call
+ *  - All device work is ordered on the caller's stream; no call synchronises
+ *    the device except gc_kv_pool_check().
+ *  - Every array argument is borrowed: no call keeps a pointer after it
+ *    returns, but asynchronous work reads it later in stream order, so the
+ *    caller keeps it alive and unchanged until the stream has passed it (the
+ *    same rule as cudaMemcpyAsync).
+ *  - Host-side argument checks (null pointers, negative sizes, unsupported
+ *    shapes) fail with a status before anything is launched; the message is
+ *    available from gc_last_error() on the same thread.
+ *  - Indices that live in device memory (block ids, block tables, lengths)
+ *    are checked by the kernels: a bad one is skipped (never dereferenced)
+ *    and its error code is recorded in the pool's device status word, read
+ *    and cleared by gc_kv_pool_check().
+ *  - Zero sizes (n_blocks = 0, batch = 0, a request with no new tokens) are
+ *    valid no-ops.
+ *  - A pool handle is not thread-safe; distinct pools are independent.
+ *  - bf16 is the only element type.  All tensors are dense and row-major.
+ *
+ * Layouts (element = bf16 unless stated)
+ *   pool       [L][2][num_pages][Hkv][ps][d]    plane 0 = K, plane 1 = V
+ *   host_src   [n_blocks][L][2][Hkv][ps][d]     one cached page per block
+ *   q, out     [T_new][Hq][d]                   new tokens of all requests,
+ *                                               packed request after request
+ *   k_new, v_new [T_new][Hkv][d]
+ *   block_table  int32 [batch][max_blocks_per_seq]: page of each block of
+ *                each request's sequence (prefix pages first)
+ *   prefix_lens  int32 [batch]   cached prefix length P_b of each request
+ *   new_lens     int32 [batch]   new-token count n_b of each request
+ *   cu_new_lens  int32 [batch+1] exclusive prefix sum of new_lens
+ *                (cu_new_lens[0] = 0, cu_new_lens[batch] = T_new)
+ */
+#ifndef GC_H_
+#define GC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h> /* cudaStream_t */
+
+#if defined(__GNUC__)
+#define GC_API __attribute__((visibility("default")))
+#else
+#define GC_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum gc_status {
+  GC_OK = 0,
+  GC_ERR_INVALID_ARG = 1,  /* null pointer, negative size, inconsistent shape */
+  GC_ERR_OUT_OF_RANGE = 2, /* a block id / page / layer outside the pool    */
+  GC_ERR_OOM = 3,          /* device allocation failed                       */
+  GC_ERR_CUDA = 4,         /* a CUDA runtime call or launch failed           */
+  GC_ERR_UNSUPPORTED = 5,  /* valid request this build has no kernel for     */
+  GC_ERR_TIMEOUT = 6       /* a device-side wait gave up (kernel returned)   */
+} gc_status;
+
+/* Opaque pool handle, owned by the library. */
+typedef struct gc_kv_pool gc_kv_pool;
+
+typedef struct gc_pool_config {
+  int32_t num_layers;   /* L >= 1                                   */
+  int32_t num_kv_heads; /* Hkv >= 1                                 */
+  int32_t head_dim;     /* d: 64 or 128                             */
+  int32_t page_size;    /* ps tokens per page: 16, 32, 64 or 128    */
+  int32_t num_pages;    /* pages per (layer, K/V) plane, >= 1       */
+} gc_pool_config;
+
+/* Device bytes a pool of this shape needs: the KV planes
+ * (L*2*num_pages*Hkv*ps*d*2 bytes) plus a 256-byte status trailer.
+ * Returns 0 for an invalid configuration. */
+GC_API size_t gc_kv_pool_bytes(const gc_pool_config* cfg);
+
+/* Create a paged KV pool on the current CUDA device.
+ *   dev_mem == NULL: the library allocates gc_kv_pool_bytes(cfg) bytes with
+ *                    cudaMalloc and frees them in gc_kv_pool_destroy.
+ *   dev_mem != NULL: caller-owned device memory of dev_bytes >=
+ *                    gc_kv_pool_bytes(cfg) bytes, 256-byte aligned; the
+ *                    library never frees it.
+ * The KV planes are not initialised; the status word is cleared.
+ * Errors: GC_ERR_INVALID_ARG, GC_ERR_UNSUPPORTED (d or ps), GC_ERR_OOM,
+ * GC_ERR_CUDA. */
+GC_API gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, size_t dev_bytes,
+                            gc_kv_pool** out);
+
+/* Destroy a pool (NULL is a no-op).  Frees library-owned memory only.  The
+ * caller must make sure no stream still uses the pool. */
+GC_API gc_status gc_kv_pool_destroy(gc_kv_pool* pool);
+
+/* Device address and byte size of the KV planes (status trailer excluded). */
+GC_API gc_status gc_kv_pool_data(const gc_kv_pool* pool, void** dev_ptr, size_t* bytes);
+
+/* Synchronise `stream`, then read and clear the pool's device status word:
+ * *device_status receives GC_OK or the first error a kernel recorded since
+ * the last check (GC_ERR_OUT_OF_RANGE for a bad device-side index,
+ * GC_ERR_TIMEOUT for a device wait that gave up).  The return value reports
+ * failures of the check itself (GC_ERR_CUDA). */
+GC_API gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t* device_status);
+
+/* gc_kv_restore flags */
+#define GC_RESTORE_SRC_DEVICE 1u /* host_src is device memory (already staged) */
+#define GC_RESTORE_VECTOR 2u     /* 16-byte vector-copy kernel instead of bulk copies */
+
+/* Restore cached prefix pages into the pool (Sec. 2.2, Fig. 2a: on a hit
+ * the cached KV of the context is loaded instead of recomputed).
+ * For i < n_blocks and every layer l and plane kv:
+ *     pool[l][kv][block_ids[i]] <- host_src[i][l][kv]
+ * a byte-exact copy of Hkv*ps*d*2 bytes; no other page changes.
+ *   host_src   [n_blocks][L][2][Hkv][ps][d] bf16.  Pinned host memory
+ *              (cudaHostAlloc / cudaHostRegister), or device memory when
+ *              flags has GC_RESTORE_SRC_DEVICE.
+ *   block_ids  int32 [n_blocks], DEVICE memory.  Ids outside
+ *              [0, num_pages) are skipped and recorded as
+ *              GC_ERR_OUT_OF_RANGE in the status word.  Duplicate ids give
+ *              an unspecified choice between the duplicates' contents.
+ *   dev_staging  NULL: the kernel reads host_src directly over the
+ *              host-device link (zero copy).  Otherwise device memory of at
+ *              least n_blocks*L*2*Hkv*ps*d*2 bytes: host_src is first copied
+ *              there with one cudaMemcpyAsync, then scattered.  Ignored with
+ *              GC_RESTORE_SRC_DEVICE.
+ * Errors: GC_ERR_INVALID_ARG (null/negative, or host_src not pinned on the
+ * zero-copy path), GC_ERR_CUDA. */
+GC_API gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
+                        int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags);
+
+/* Append the new tokens' K and V after each request's cached prefix
+ * (Sec. 2.2: the KV of the cached tokens and of the new tokens is stitched
+ * into one sequence).  For request b, new token t < n_b and kv head g:
+ *     pos = seq_lens[b] + t
+ *     pool[layer][0][block_table[b][pos/ps]][g][pos%ps] <- k_new[cu_new_lens[b]+t][g]
+ *     pool[layer][1][...same slot...]                   <- v_new[cu_new_lens[b]+t][g]
+ *   k_new, v_new  [T_new][Hkv][d] bf16, device.
+ *   block_table   int32 [batch][max_blocks_per_seq], device.
+ *   seq_lens      int32 [batch], device: the write offset of each request,
+ *                 i.e. its cached prefix length P_b.
+ *   cu_new_lens   int32 [batch+1], device.
+ * A token whose block index is >= max_blocks_per_seq or whose page is
+ * outside the pool is skipped and recorded as GC_ERR_OUT_OF_RANGE.
+ *   total_new_tokens  T_new = cu_new_lens[batch], passed from the host; it
+ *                 sizes the grid and bounds every k_new / v_new row read.
+ *                 A request whose rows would pass it is skipped and
+ *                 recorded as GC_ERR_OUT_OF_RANGE.
+ * Errors: GC_ERR_INVALID_ARG, GC_ERR_OUT_OF_RANGE (layer), GC_ERR_CUDA. */
+GC_API gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v_new,
+                       const int32_t* block_table, const int32_t* seq_lens, cudaStream_t stream,
+                       int32_t layer, const int32_t* cu_new_lens, int32_t batch,
+                       int32_t max_blocks_per_seq, int32_t total_new_tokens);
+
+/* Prefill of the new tokens over [cached prefix ++ new tokens] (Sec. 2.2:
+ * the cached and new tokens' KV are processed together; Sec. 2.1: prefill).
+ * For request b, q head h and new row i < n_b, with g = h / (Hq/Hkv),
+ * P = prefix_lens[b] and keys j read through block_table[b]:
+ *     out[cu_new_lens[b]+i][h] = sum_{j <= P+i} softmax_j(softmax_scale *
+ *                                   q[cu_new_lens[b]+i][h] . k_j) v_j
+ * i.e. causal attention bottom-right aligned: new row i sits at absolute
+ * position P+i.  The result equals the corresponding rows of a full causal
+ * prefill of the concatenated sequence.  Keys at positions >= P_b + n_b are
+ * never used, whatever their contents (NaN included).
+ *   q, out      [T_new][Hq][d] bf16, device (out is written for valid rows
+ *               only).  Accumulation is fp32, P is rounded to bf16 before
+ *               the PV product, out is rounded to nearest even.
+ *   prefix_lens, new_lens  int32 [batch], device.  cu_new_lens int32
+ *               [batch+1], device, consistent with new_lens.
+ *   num_q_heads Hq, a multiple of the pool's Hkv with Hq/Hkv in
+ *               {1,2,4,8,16}.
+ *   total_new_tokens  T_new = cu_new_lens[batch], passed from the host; it
+ *               bounds every q / out row access.  A request whose rows would
+ *               pass it is skipped and recorded as GC_ERR_OUT_OF_RANGE.
+ * Errors: GC_ERR_INVALID_ARG, GC_ERR_OUT_OF_RANGE (layer),
+ * GC_ERR_UNSUPPORTED (head grouping), GC_ERR_CUDA. */
+GC_API gc_status gc_prefix_prefill_attn(const void* q, const gc_kv_pool* pool, const int32_t* block_table,
+                                 const int32_t* prefix_lens, const int32_t* new_lens, void* out,
+                                 cudaStream_t stream, int32_t layer, const int32_t* cu_new_lens,
+                                 int32_t batch, int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                 float softmax_scale, int32_t total_new_tokens);
+
+/* Same operation and arguments as gc_prefix_prefill_attn, computed by a
+ * plain CUDA-core kernel (one warp per row, fp32 throughout, no tensor
+ * cores).  Slow; kept as an independent GPU cross-check of the indexing. */
+GC_API gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* pool,
+                                      const int32_t* block_table, const int32_t* prefix_lens,
+                                      const int32_t* new_lens, void* out, cudaStream_t stream,
+                                      int32_t layer, const int32_t* cu_new_lens, int32_t batch,
+                                      int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                      float softmax_scale, int32_t total_new_tokens);
+
+/* Message of the last failing call on this thread ("" if none). */
+GC_API const char* gc_last_error(void);
+
+/* Static name of a status code. */
+GC_API const char* gc_status_string(gc_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GC_H_ */

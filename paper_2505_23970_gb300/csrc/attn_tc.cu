@@ -1,0 +1,608 @@
+// Prefix-reuse causal GQA attention on the sm_103a tensor cores.
+//
+// Operation (Sec. 2.2: the cached context KV and the new tokens' KV are
+// processed together; Sec. 2.1: prefill): for request b, q head h, new row
+// i < n_b and kv head g = h / G,
+//     O[b,i,h] = sum_{j <= P_b + i} softmax_j(scale * q . k_j) v_j
+// with keys read from the paged pool through block_table[b].
+//
+// Design
+//  * Work item = (request b, kv head g, pair of 128-row Q tiles).  A Q tile
+//    packs 128/G new tokens x the G q heads of one kv group (row = token*G +
+//    head), so every K/V tile fetched from the pool feeds all G heads, and
+//    the two Q tiles of a CTA share each K/V tile as well.
+//  * One persistent CTA per SM, 12 warps:
+//      warp 0        TMA producer: Q tiles (3-D map over [T_new][Hq][d]) and
+//                    K/V tiles page by page (2-D map over the pool rows);
+//                    zeroes V rows past the end of the sequence.
+//      warp 1        TMEM owner; lane 0 issues every tcgen05.mma:
+//                      S_i = Q_i K^T   (SS, both operands K-major, fp32 in TMEM)
+//                      O_i += P_i V    (TS: P_i read from TMEM, V MN-major)
+//      warps 4-7     softmax of Q tile 0; warps 8-11 softmax of Q tile 1.
+//                    One thread per row: S row from TMEM, causal mask, online
+//                    softmax in the log2 domain with lazy rescaling (the
+//                    reference max moves only when a row max grows by more
+//                    than 2^8), P as bf16 written back over S in TMEM, final
+//                    1/l normalisation and the bf16 store of O.
+//  * TMEM (512 columns): S0 [0,128) S1 [128,256) O0 [256,256+d) O1 [.., +d).
+//    P_i overwrites the first 64 columns of S_i.  Because P_i aliases S_i,
+//    S_i(j+1) is issued only after PV_i(j) has completed; the MMA order
+//    S0 S1 PV0 PV1 keeps the tensor pipe fed while it waits.
+//  * Every mbarrier wait is bounded; a timeout raises the CTA's abort flag,
+//    all roles leave their loops, in-flight copies and MMAs are drained, TMEM
+//    is freed and GC_ERR_TIMEOUT is recorded in the pool status word.
+#include <cmath>
+
+#include "gc_internal.cuh"
+#include "sm103_ptx.cuh"
+
+namespace gc {
+namespace {
+
+using namespace ptx;
+
+constexpr int kThreads = 384;
+constexpr int kTileM = 128;     // rows per Q tile
+constexpr int kTileN = 128;     // keys per K/V tile
+constexpr float kRescaleLog2 = 8.0f;
+
+template <int D>
+struct Cfg {
+  static constexpr int kHalves = D / 64;               // 128-byte column blocks
+  static constexpr int kHalfBytes = kTileM * 128;      // one 64-column block of a tile
+  static constexpr int kTileBytes = kHalves * kHalfBytes;
+  static constexpr int kStages = D == 128 ? 4 : 8;
+  static constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO0 = 256, kColO1 = 256 + D;
+  static constexpr uint32_t kIdescQK = idesc_bf16_f32(kTileM, kTileN, false, false);
+  static constexpr uint32_t kIdescPV = idesc_bf16_f32(kTileM, D, false, true);
+};
+
+struct Geom {
+  int32_t batch, Hq, Hkv, G, ps, ps_shift, num_pages, max_blocks, layer, total_new;
+  float scale_log2;
+};
+
+struct Barriers {
+  uint64_t q_full, q_empty, vfix, drain;
+  uint64_t kv_full[8], kv_empty[8];
+  uint64_t s_full[2], p_full[2], pv_done[2];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+// A work item and the quantities every role derives from it.
+struct Item {
+  int b, g, P, n, cu, T;
+  int tok0[2], nt_i[2], nt;
+  bool valid[2];
+};
+
+__device__ __forceinline__ bool decode_item(int it, const int* item_start, const Geom& geo,
+                                            const int32_t* __restrict__ prefix_lens,
+                                            const int32_t* __restrict__ new_lens,
+                                            const int32_t* __restrict__ cu_new_lens, Item& w) {
+  int lo = 0, hi = geo.batch;  // last b with item_start[b] <= it
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (item_start[mid] <= it) lo = mid; else hi = mid;
+  }
+  w.b = lo;
+  const int local = it - item_start[lo];
+  const int pairs = (item_start[lo + 1] - item_start[lo]) / geo.Hkv;
+  const int pair = pairs - 1 - local / geo.Hkv;  // later rows (more keys) first
+  w.g = local % geo.Hkv;
+  w.P = __ldg(prefix_lens + lo);
+  w.n = __ldg(new_lens + lo);
+  w.cu = __ldg(cu_new_lens + lo);
+  w.T = w.P + w.n;
+  const int rows = w.n * geo.G;
+  w.nt = 0;
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const int r0 = pair * 2 * kTileM + i * kTileM;
+    w.valid[i] = r0 < rows;
+    w.tok0[i] = r0 / geo.G;
+    const int r1 = min(r0 + kTileM - 1, rows - 1);
+    const int kend = w.P + r1 / geo.G + 1;  // keys [0, kend) reach some row
+    w.nt_i[i] = w.valid[i] ? (kend + kTileN - 1) / kTileN : 0;
+    w.nt = max(w.nt, w.nt_i[i]);
+  }
+  return true;
+}
+
+// ------------------------------------------------------------------ roles
+template <int D>
+__device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const int* item_start,
+                         int total_items, const Geom& geo, const CUtensorMap* map_q,
+                         const CUtensorMap* map_kv, const int32_t* __restrict__ block_table,
+                         const int32_t* __restrict__ prefix_lens,
+                         const int32_t* __restrict__ new_lens,
+                         const int32_t* __restrict__ cu_new_lens, int32_t* status) {
+  using C = Cfg<D>;
+  const int lane = threadIdx.x & 31;
+  volatile int* abortp = &bar.abort_flag;
+  uint32_t q_count = 0, kv_count = 0, vfix_count = 0;
+  int armed_slot_parity[C::kStages];
+  int armed_q = -1, armed_vfix = -1;
+#pragma unroll
+  for (int s = 0; s < C::kStages; ++s) armed_slot_parity[s] = -1;
+  bool ok = true;
+  const uint32_t box_bytes = static_cast<uint32_t>(geo.ps) * 128;  // one page, one column block
+
+  for (int it = blockIdx.x; ok && it < total_items; it += gridDim.x) {
+    Item w;
+    decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
+    // ---- Q tiles
+    ok = mbar_wait(&bar.q_empty, (q_count & 1) ^ 1, abortp);
+    if (!ok) break;
+    if (lane == 0) {
+      uint32_t bytes = 0;
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+        if (w.valid[i]) bytes += C::kTileBytes;
+      mbar_arrive_expect_tx(&bar.q_full, bytes);
+#pragma unroll
+      for (int i = 0; i < 2; ++i)
+        if (w.valid[i])
+#pragma unroll
+          for (int h = 0; h < C::kHalves; ++h)
+            tma_load_3d(smem_q + i * C::kTileBytes + h * C::kHalfBytes, map_q, &bar.q_full, h * 64,
+                        w.g * geo.G, w.cu + w.tok0[i]);
+    }
+    armed_q = q_count & 1;
+    ++q_count;
+    // ---- K/V tiles, page by page
+    const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
+    for (int j = 0; ok && j < w.nt; ++j) {
+      const int key0 = j * kTileN;
+      const int nkeys = min(kTileN, w.T - key0);
+      const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
+#pragma unroll 1
+      for (int kv = 0; kv < 2; ++kv) {
+        const int slot = kv_count % C::kStages;
+        ok = mbar_wait(&bar.kv_empty[slot], ((kv_count / C::kStages) & 1) ^ 1, abortp);
+        if (!ok) break;
+        uint8_t* dst = smem_kv + slot * C::kTileBytes;
+        const bool fix = kv == 1 && nkeys < kTileN;
+        uint64_t* full = fix ? &bar.vfix : &bar.kv_full[slot];
+        if (lane == 0) {
+          int good = 0;
+          for (int pg = 0; pg < npages; ++pg) {
+            const int blk = (key0 >> geo.ps_shift) + pg;
+            const int page = blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
+            good += (page >= 0 && page < geo.num_pages);
+          }
+          mbar_arrive_expect_tx(full, static_cast<uint32_t>(good) * box_bytes * C::kHalves);
+          for (int pg = 0; pg < npages; ++pg) {
+            const int blk = (key0 >> geo.ps_shift) + pg;
+            const int page = blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
+            if (page < 0 || page >= geo.num_pages) {
+              record_error(status, GC_ERR_OUT_OF_RANGE);
+              continue;
+            }
+            const int row = (((geo.layer * 2 + kv) * geo.num_pages + page) * geo.Hkv + w.g)
+                            << geo.ps_shift;
+#pragma unroll
+            for (int h = 0; h < C::kHalves; ++h)
+              tma_load_2d(dst + h * C::kHalfBytes + pg * box_bytes, map_kv, full, h * 64, row);
+          }
+        }
+        if (fix) {
+          // V rows past the end of the sequence must be zero, not stale or NaN:
+          // their P is zero but 0 * NaN would poison the PV product.
+          ok = mbar_wait(&bar.vfix, vfix_count & 1, abortp);
+          if (!ok) {
+            armed_slot_parity[slot] = -1;
+            armed_vfix = vfix_count & 1;
+            break;
+          }
+          ++vfix_count;
+          const int zrows = kTileN - nkeys;
+          for (int h = 0; h < C::kHalves; ++h) {
+            uint4* z = reinterpret_cast<uint4*>(dst + h * C::kHalfBytes + nkeys * 128);
+            for (int k = lane; k < zrows * 8; k += 32) z[k] = make_uint4(0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar.kv_full[slot]);
+        } else {
+          armed_slot_parity[slot] = (kv_count / C::kStages) & 1;
+        }
+        ++kv_count;
+      }
+    }
+  }
+  if (!ok && lane == 0) {
+    // drain copies still in flight before the CTA exits (bounded, ignores abort)
+    int no_abort = 0;
+    if (armed_q >= 0) mbar_wait(&bar.q_full, armed_q, &no_abort);
+    if (armed_vfix >= 0) mbar_wait(&bar.vfix, armed_vfix, &no_abort);
+    for (int s = 0; s < C::kStages; ++s)
+      if (armed_slot_parity[s] >= 0) mbar_wait(&bar.kv_full[s], armed_slot_parity[s], &no_abort);
+  }
+}
+
+template <int D>
+__device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uint32_t tmem,
+                           const int* item_start, int total_items, const Geom& geo,
+                           const int32_t* __restrict__ prefix_lens,
+                           const int32_t* __restrict__ new_lens,
+                           const int32_t* __restrict__ cu_new_lens) {
+  using C = Cfg<D>;
+  volatile int* abortp = &bar.abort_flag;
+  uint32_t q_count = 0, kv_count = 0;
+  uint32_t pv_issued[2] = {0, 0}, pv_waited[2] = {0, 0}, p_count[2] = {0, 0};
+  bool ok = true;
+  const uint32_t q_base = smem_addr(smem_q), kv_base = smem_addr(smem_kv);
+  const uint32_t col_s[2] = {C::kColS0, C::kColS1};
+  const uint32_t col_o[2] = {C::kColO0, C::kColO1};
+
+  for (int it = blockIdx.x; ok && it < total_items; it += gridDim.x) {
+    Item w;
+    decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
+    ok = mbar_wait(&bar.q_full, q_count & 1, abortp);
+    ++q_count;
+    if (!ok) break;
+    tc_fence_after();
+    for (int j = 0; ok && j < w.nt; ++j) {
+      // ---- S_i = Q_i K_j^T
+      const int ks = kv_count % C::kStages;
+      ok = mbar_wait(&bar.kv_full[ks], (kv_count / C::kStages) & 1, abortp);
+      ++kv_count;
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t k_addr = kv_base + ks * C::kTileBytes;
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        if (j >= w.nt_i[i]) continue;
+        if (pv_issued[i] > pv_waited[i]) {  // P_i aliases S_i: PV_i must be done
+          ok = mbar_wait(&bar.pv_done[i], (pv_issued[i] - 1) & 1, abortp);
+          if (!ok) break;
+          pv_waited[i] = pv_issued[i];
+          tc_fence_after();
+        }
+        const uint32_t q_addr = q_base + i * C::kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * C::kHalfBytes + (kk & 3) * 32;
+          mma_ss(tmem + col_s[i], sdesc_sw128(q_addr + off, 16, 1024),
+                 sdesc_sw128(k_addr + off, 16, 1024), C::kIdescQK, kk > 0);
+        }
+        mma_commit(&bar.s_full[i]);
+      }
+      if (!ok) break;
+      mma_commit(&bar.kv_empty[ks]);
+      if (j == w.nt - 1) mma_commit(&bar.q_empty);
+      // ---- O_i += P_i V_j
+      const int vs = kv_count % C::kStages;
+      ok = mbar_wait(&bar.kv_full[vs], (kv_count / C::kStages) & 1, abortp);
+      ++kv_count;
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t v_addr = kv_base + vs * C::kTileBytes;
+#pragma unroll
+      for (int i = 0; i < 2; ++i) {
+        if (j >= w.nt_i[i]) continue;
+        ok = mbar_wait(&bar.p_full[i], p_count[i] & 1, abortp);
+        ++p_count[i];
+        if (!ok) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < kTileN / 16; ++kk)
+          mma_ts(tmem + col_o[i], tmem + col_s[i] + kk * 8,
+                 sdesc_sw128(v_addr + kk * 16 * 128, C::kHalfBytes, 1024), C::kIdescPV,
+                 (j > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&bar.pv_done[i]);
+        ++pv_issued[i];
+      }
+      if (!ok) break;
+      mma_commit(&bar.kv_empty[vs]);
+    }
+  }
+  // wait for every MMA this thread issued before TMEM is released
+  mma_commit(&bar.drain);
+  int no_abort = 0;
+  mbar_wait(&bar.drain, 0, &no_abort);
+}
+
+template <int D>
+__device__ void softmax_wg(int i, Barriers& bar, uint32_t tmem, const int* item_start,
+                           int total_items, const Geom& geo,
+                           const int32_t* __restrict__ prefix_lens,
+                           const int32_t* __restrict__ new_lens,
+                           const int32_t* __restrict__ cu_new_lens,
+                           __nv_bfloat16* __restrict__ out) {
+  using C = Cfg<D>;
+  volatile int* abortp = &bar.abort_flag;
+  const int warp = threadIdx.x >> 5;
+  const int r = threadIdx.x - kTileM * (1 + i);               // row of the Q tile (= TMEM lane)
+  const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+  const uint32_t tS = lane_addr + (i ? C::kColS1 : C::kColS0);
+  const uint32_t tO = lane_addr + (i ? C::kColO1 : C::kColO0);
+  uint32_t s_count = 0, pv_total = 0;
+  bool ok = true;
+
+  for (int it = blockIdx.x; ok && it < total_items; it += gridDim.x) {
+    Item w;
+    decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
+    if (!w.valid[i]) continue;
+    const int tok = w.tok0[i] + r / geo.G;
+    const bool row_valid = tok < w.n;
+    const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
+    float m_run = -INFINITY, l = 0.f;
+    for (int j = 0; j < w.nt_i[i]; ++j) {
+      ok = mbar_wait(&bar.s_full[i], s_count & 1, abortp);
+      ++s_count;
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t sr[4][32];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+      tmem_wait_ld();
+      const int key0 = j * kTileN;
+      float mt = -INFINITY;
+      if (key0 + kTileN - 1 > kmax) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const float v = key0 + c * 32 + e > kmax ? -INFINITY : __uint_as_float(sr[c][e]);
+            sr[c][e] = __float_as_uint(v);
+            mt = fmaxf(mt, v);
+          }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e) mt = fmaxf(mt, __uint_as_float(sr[c][e]));
+      }
+      const float mt2 = mt * geo.scale_log2;
+      if (__any_sync(0xffffffffu, mt2 > m_run + kRescaleLog2)) {
+        const float m_new = fmaxf(m_run, mt2);
+        const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;  // 0 if m_run = -inf
+        if (j > 0) {
+          // O_i is complete up to tile j-1: S_i(j) was issued after PV_i(j-1)
+#pragma unroll 1
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(tO + c * 32, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+            tmem_st32(tO + c * 32, o);
+          }
+        }
+        l *= alpha;
+        m_run = m_new;
+      }
+      const float neg_m = -m_run;
+      float lsum0 = 0.f, lsum1 = 0.f;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c][2 * e]), geo.scale_log2, neg_m));
+          const float p1 =
+              ex2_approx(fmaf(__uint_as_float(sr[c][2 * e + 1]), geo.scale_log2, neg_m));
+          lsum0 += p0;
+          lsum1 += p1;
+          pk[e] = pack_bf16x2(p0, p1);
+        }
+        tmem_st16(tS + c * 16, pk);
+      }
+      l += lsum0 + lsum1;
+      tmem_wait_st();
+      tc_fence_before();
+      mbar_arrive(&bar.p_full[i]);
+    }
+    if (!ok) break;
+    // ---- epilogue: O / l -> bf16
+    pv_total += w.nt_i[i];
+    ok = mbar_wait(&bar.pv_done[i], (pv_total - 1) & 1, abortp);
+    if (!ok) break;
+    tc_fence_after();
+    const float inv_l = 1.f / l;
+    const int h = w.g * geo.G + r % geo.G;
+    uint4* orow = reinterpret_cast<uint4*>(
+        out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * D);
+#pragma unroll 1
+    for (int c = 0; c < D / 32; ++c) {
+      uint32_t o[32];
+      tmem_ld32(tO + c * 32, o);
+      tmem_wait_ld();
+      if (row_valid) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 pk;
+          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+          orow[c * 4 + v] = pk;
+        }
+      }
+    }
+    tc_fence_before();
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
+                   const __grid_constant__ CUtensorMap map_kv,
+                   const int32_t* __restrict__ block_table, const int32_t* __restrict__ prefix_lens,
+                   const int32_t* __restrict__ new_lens, const int32_t* __restrict__ cu_new_lens,
+                   __nv_bfloat16* __restrict__ out, Geom geo, int32_t* status) {
+  using C = Cfg<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* smem_q = base;
+  uint8_t* smem_kv = base + 2 * C::kTileBytes;
+  Barriers& bar = *reinterpret_cast<Barriers*>(smem_kv + C::kStages * C::kTileBytes);
+  int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bar.q_full, 1);
+    mbar_init(&bar.q_empty, 1);
+    mbar_init(&bar.vfix, 1);
+    mbar_init(&bar.drain, 1);
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&bar.kv_full[s], 1);
+      mbar_init(&bar.kv_empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bar.s_full[i], 1);
+      mbar_init(&bar.p_full[i], kTileM);
+      mbar_init(&bar.pv_done[i], 1);
+    }
+    bar.abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&map_q);
+    prefetch_tensormap(&map_kv);
+  }
+  if (warp == 1) {
+    tmem_alloc(&bar.tmem_base, 512);
+    tmem_relinquish();
+  }
+  if (warp == 2) {
+    // work items per request: Hkv * ceil(n_b * G / 256); exclusive scan
+    int running = 0;
+    for (int b0 = 0; b0 < geo.batch; b0 += 32) {
+      const int b = b0 + lane;
+      int cnt = 0;
+      if (b < geo.batch) {
+        const int n = __ldg(new_lens + b), P = __ldg(prefix_lens + b);
+        const int cu = __ldg(cu_new_lens + b);
+        const bool sane = n >= 0 && P >= 0 && cu >= 0 && cu + n <= geo.total_new;
+        if (!sane && n != 0) record_error(status, GC_ERR_OUT_OF_RANGE);
+        if (sane && n > 0) cnt = geo.Hkv * ((n * geo.G + 2 * kTileM - 1) / (2 * kTileM));
+      }
+      int incl = cnt;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (b < geo.batch) item_start[b] = running + incl - cnt;
+      running += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) item_start[geo.batch] = running;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = bar.tmem_base;
+  const int total_items = item_start[geo.batch];
+
+  if (warp == 0) {
+    producer<D>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv, block_table,
+                prefix_lens, new_lens, cu_new_lens, status);
+  } else if (warp == 1) {
+    if (lane == 0)
+      mma_issuer<D>(smem_q, smem_kv, bar, tmem, item_start, total_items, geo, prefix_lens,
+                    new_lens, cu_new_lens);
+    __syncwarp();
+  } else if (warp >= 4) {
+    softmax_wg<D>((warp - 4) >> 2, bar, tmem, item_start, total_items, geo, prefix_lens, new_lens,
+                  cu_new_lens, out);
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+  if (threadIdx.x == 0 && bar.abort_flag) record_error(status, GC_ERR_TIMEOUT);
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+template <int D>
+gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
+  using C = Cfg<D>;
+  auto enc = encode_fn();
+  if (!enc) return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: cuTensorMapEncodeTiled unavailable");
+  const auto& cfg = pool->cfg;
+  Geom geo;
+  geo.batch = a.batch;
+  geo.Hq = a.num_q_heads;
+  geo.Hkv = cfg.num_kv_heads;
+  geo.G = geo.Hq / geo.Hkv;
+  geo.ps = cfg.page_size;
+  int s = 0;
+  while ((1 << s) < geo.ps) ++s;
+  geo.ps_shift = s;
+  geo.num_pages = cfg.num_pages;
+  geo.max_blocks = a.max_blocks;
+  geo.layer = a.layer;
+  geo.total_new = a.total_new_tokens;
+  geo.scale_log2 = a.softmax_scale * 1.4426950408889634f;
+
+  const uint64_t pool_rows = static_cast<uint64_t>(cfg.num_layers) * 2 * cfg.num_pages *
+                             cfg.num_kv_heads * cfg.page_size;
+  if (pool_rows >= (1ull << 31))
+    return fail(GC_ERR_UNSUPPORTED, "gc_prefix_prefill_attn: pool has %llu rows (limit 2^31)",
+                static_cast<unsigned long long>(pool_rows));
+  CUtensorMap map_q, map_kv;
+  {
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(geo.Hq),
+                          static_cast<cuuint64_t>(geo.total_new)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2,
+                             static_cast<cuuint64_t>(geo.Hq) * D * 2};
+    cuuint32_t box[3] = {64, static_cast<cuuint32_t>(geo.G), static_cast<cuuint32_t>(kTileM / geo.G)};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = enc(&map_q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.q), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: q tensor map (CUresult %d)", (int)r);
+  }
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(D), pool_rows};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(D) * 2};
+    cuuint32_t box[2] = {64, static_cast<cuuint32_t>(geo.ps)};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = enc(&map_kv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool->data, dims, strides, box,
+                     es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: pool tensor map (CUresult %d)", (int)r);
+  }
+  const size_t smem = 1024 + 2 * C::kTileBytes + C::kStages * C::kTileBytes + sizeof(Barriers) +
+                      (static_cast<size_t>(a.batch) + 1) * sizeof(int);
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: smem attribute");
+  attn_tc_kernel<D><<<pool->num_sms, kThreads, smem, stream>>>(
+      map_q, map_kv, a.block_table, a.prefix_lens, a.new_lens, a.cu_new_lens,
+      static_cast<__nv_bfloat16*>(a.out), geo, pool->status);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: launch");
+  return GC_OK;
+}
+
+}  // namespace
+
+gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
+  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream);
+  return launch<64>(pool, a, stream);
+}
+
+}  // namespace gc

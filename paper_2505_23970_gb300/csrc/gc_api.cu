@@ -1,0 +1,296 @@
+// C ABI of libgc: pool management, host-side argument checks and dispatch to
+// the CUDA kernels.  Nothing here computes on the host: every byte of the
+// restore, append and attention results is produced by a kernel.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "gc_internal.cuh"
+
+namespace {
+thread_local char g_msg[512] = "";
+constexpr size_t kTrailer = 256;  // status word + padding after the KV planes
+}  // namespace
+
+namespace gc {
+
+gc_status fail(gc_status s, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_msg, sizeof g_msg, fmt, ap);
+  va_end(ap);
+  return s;
+}
+
+gc_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(e == cudaErrorMemoryAllocation ? GC_ERR_OOM : GC_ERR_CUDA, "%s: %s (%s)", what,
+              cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+}  // namespace gc
+
+using gc::fail;
+
+static bool pool_config_ok(const gc_pool_config* c) {
+  return c && c->num_layers >= 1 && c->num_kv_heads >= 1 && c->head_dim >= 1 &&
+         c->page_size >= 1 && c->num_pages >= 1;
+}
+
+static bool pool_config_supported(const gc_pool_config* c) {
+  const bool d_ok = c->head_dim == 64 || c->head_dim == 128;
+  const bool ps_ok = c->page_size == 16 || c->page_size == 32 || c->page_size == 64 ||
+                     c->page_size == 128;
+  return d_ok && ps_ok;
+}
+
+extern "C" {
+
+const char* gc_last_error(void) { return g_msg; }
+
+const char* gc_status_string(gc_status s) {
+  switch (s) {
+    case GC_OK: return "GC_OK";
+    case GC_ERR_INVALID_ARG: return "GC_ERR_INVALID_ARG";
+    case GC_ERR_OUT_OF_RANGE: return "GC_ERR_OUT_OF_RANGE";
+    case GC_ERR_OOM: return "GC_ERR_OOM";
+    case GC_ERR_CUDA: return "GC_ERR_CUDA";
+    case GC_ERR_UNSUPPORTED: return "GC_ERR_UNSUPPORTED";
+    case GC_ERR_TIMEOUT: return "GC_ERR_TIMEOUT";
+  }
+  return "GC_ERR_UNKNOWN";
+}
+
+size_t gc_kv_pool_bytes(const gc_pool_config* cfg) {
+  if (!pool_config_ok(cfg)) return 0;
+  const size_t planes = static_cast<size_t>(cfg->num_layers) * 2 * cfg->num_pages *
+                        gc::page_bytes(*cfg);
+  return ((planes + 255) / 256) * 256 + kTrailer;
+}
+
+gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, size_t dev_bytes,
+                            gc_kv_pool** out) {
+  g_msg[0] = 0;
+  if (!out) return fail(GC_ERR_INVALID_ARG, "gc_kv_pool_create: out is NULL");
+  *out = nullptr;
+  if (!pool_config_ok(cfg))
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_pool_create: invalid configuration");
+  if (!pool_config_supported(cfg))
+    return fail(GC_ERR_UNSUPPORTED,
+                "gc_kv_pool_create: head_dim %d / page_size %d not supported "
+                "(head_dim 64 or 128; page_size 16, 32, 64 or 128)",
+                cfg->head_dim, cfg->page_size);
+  const size_t need = gc_kv_pool_bytes(cfg);
+  if (dev_mem) {
+    if (dev_bytes < need)
+      return fail(GC_ERR_INVALID_ARG, "gc_kv_pool_create: dev_bytes %zu < required %zu",
+                  dev_bytes, need);
+    if (reinterpret_cast<uintptr_t>(dev_mem) % 256)
+      return fail(GC_ERR_INVALID_ARG, "gc_kv_pool_create: dev_mem not 256-byte aligned");
+  }
+  int dev = 0, sms = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_pool_create: device query");
+  void* mem = dev_mem;
+  void* owned = nullptr;
+  if (!mem) {
+    e = cudaMalloc(&mem, need);
+    if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_pool_create: cudaMalloc");
+    owned = mem;
+  }
+  auto* p = new (std::nothrow) gc_kv_pool;
+  if (!p) {
+    if (owned) cudaFree(owned);
+    return fail(GC_ERR_OOM, "gc_kv_pool_create: host allocation");
+  }
+  p->cfg = *cfg;
+  p->data = static_cast<uint8_t*>(mem);
+  p->data_bytes = need - kTrailer;
+  p->status = reinterpret_cast<int32_t*>(p->data + p->data_bytes);
+  p->owned = owned;
+  p->device = dev;
+  p->num_sms = sms;
+  e = cudaMemset(p->status, 0, kTrailer);
+  if (e != cudaSuccess) {
+    if (owned) cudaFree(owned);
+    delete p;
+    return gc::cuda_fail(e, "gc_kv_pool_create: clearing the status word");
+  }
+  // data_bytes reported to the caller excludes the alignment padding
+  p->data_bytes = static_cast<size_t>(cfg->num_layers) * 2 * cfg->num_pages *
+                  gc::page_bytes(*cfg);
+  *out = p;
+  return GC_OK;
+}
+
+gc_status gc_kv_pool_destroy(gc_kv_pool* pool) {
+  g_msg[0] = 0;
+  if (!pool) return GC_OK;
+  if (pool->owned) {
+    cudaError_t e = cudaFree(pool->owned);
+    delete pool;
+    if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_pool_destroy: cudaFree");
+    return GC_OK;
+  }
+  delete pool;
+  return GC_OK;
+}
+
+gc_status gc_kv_pool_data(const gc_kv_pool* pool, void** dev_ptr, size_t* bytes) {
+  g_msg[0] = 0;
+  if (!pool || !dev_ptr || !bytes) return fail(GC_ERR_INVALID_ARG, "gc_kv_pool_data: NULL argument");
+  *dev_ptr = pool->data;
+  *bytes = pool->data_bytes;
+  return GC_OK;
+}
+
+gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t* device_status) {
+  g_msg[0] = 0;
+  if (!pool || !device_status) return fail(GC_ERR_INVALID_ARG, "gc_kv_pool_check: NULL argument");
+  int32_t host = 0;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e == cudaSuccess) e = cudaMemcpy(&host, pool->status, sizeof host, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemset(pool->status, 0, sizeof host);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_pool_check");
+  *device_status = host;
+  return GC_OK;
+}
+
+gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
+                        int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  g_msg[0] = 0;
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: pool is NULL");
+  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: n_blocks < 0");
+  if (flags & ~(GC_RESTORE_SRC_DEVICE | GC_RESTORE_VECTOR))
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: unknown flags 0x%x", flags);
+  if (n_blocks == 0) return GC_OK;
+  if (!host_src || !block_ids)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: host_src / block_ids is NULL");
+  const size_t bytes = static_cast<size_t>(n_blocks) * pool->cfg.num_layers * 2 *
+                       gc::page_bytes(pool->cfg);
+  const uint8_t* src = static_cast<const uint8_t*>(host_src);
+  bool vector = (flags & GC_RESTORE_VECTOR) != 0;
+  if (!(flags & GC_RESTORE_SRC_DEVICE)) {
+    cudaPointerAttributes attr;
+    cudaError_t e = cudaPointerGetAttributes(&attr, host_src);
+    if (e != cudaSuccess || attr.type != cudaMemoryTypeHost) {
+      cudaGetLastError();
+      return fail(GC_ERR_INVALID_ARG,
+                  "gc_kv_restore: host_src must be pinned host memory "
+                  "(cudaHostAlloc / cudaHostRegister) unless GC_RESTORE_SRC_DEVICE is set");
+    }
+    if (dev_staging) {
+      if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
+        return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: dev_staging not 16-byte aligned");
+      e = cudaMemcpyAsync(dev_staging, host_src, bytes, cudaMemcpyHostToDevice, stream);
+      if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_restore: staging copy");
+      src = static_cast<const uint8_t*>(dev_staging);
+    } else {
+      // zero copy: the kernel reads the pinned buffer through its device alias
+      void* dptr = attr.devicePointer;
+      if (!dptr) return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: host_src has no device mapping");
+      src = static_cast<const uint8_t*>(dptr);
+      vector = true;
+    }
+  }
+  if (reinterpret_cast<uintptr_t>(src) % 16)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: source not 16-byte aligned");
+  return vector ? gc::launch_restore_vector(pool, src, block_ids, n_blocks, stream)
+                : gc::launch_restore_bulk(pool, src, block_ids, n_blocks, stream);
+}
+
+gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v_new,
+                       const int32_t* block_table, const int32_t* seq_lens, cudaStream_t stream,
+                       int32_t layer, const int32_t* cu_new_lens, int32_t batch,
+                       int32_t max_blocks_per_seq, int32_t total_new_tokens) {
+  g_msg[0] = 0;
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_kv_append: pool is NULL");
+  if (batch < 0 || total_new_tokens < 0 || max_blocks_per_seq < 0)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_append: negative size");
+  if (layer < 0 || layer >= pool->cfg.num_layers)
+    return fail(GC_ERR_OUT_OF_RANGE, "gc_kv_append: layer %d outside [0, %d)", layer,
+                pool->cfg.num_layers);
+  if (batch == 0 || total_new_tokens == 0) return GC_OK;
+  if (!k_new || !v_new || !block_table || !seq_lens || !cu_new_lens)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_append: NULL array argument");
+  if (max_blocks_per_seq == 0)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_append: max_blocks_per_seq is 0");
+  if ((reinterpret_cast<uintptr_t>(k_new) | reinterpret_cast<uintptr_t>(v_new)) % 16)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_append: k_new / v_new not 16-byte aligned");
+  return gc::launch_append(pool, k_new, v_new, block_table, seq_lens, cu_new_lens, batch,
+                           max_blocks_per_seq, layer, total_new_tokens, stream);
+}
+
+static gc_status attn_common(const char* who, const void* q, const gc_kv_pool* pool,
+                             const int32_t* block_table, const int32_t* prefix_lens,
+                             const int32_t* new_lens, void* out, int32_t layer,
+                             const int32_t* cu_new_lens, int32_t batch,
+                             int32_t max_blocks_per_seq, int32_t num_q_heads,
+                             float softmax_scale, int32_t total_new_tokens, gc::AttnArgs* a,
+                             bool* noop) {
+  *noop = false;
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (batch < 0 || total_new_tokens < 0 || max_blocks_per_seq < 0)
+    return fail(GC_ERR_INVALID_ARG, "%s: negative size", who);
+  if (layer < 0 || layer >= pool->cfg.num_layers)
+    return fail(GC_ERR_OUT_OF_RANGE, "%s: layer %d outside [0, %d)", who, layer,
+                pool->cfg.num_layers);
+  const int hkv = pool->cfg.num_kv_heads;
+  if (num_q_heads <= 0 || num_q_heads % hkv)
+    return fail(GC_ERR_INVALID_ARG, "%s: num_q_heads %d not a multiple of num_kv_heads %d", who,
+                num_q_heads, hkv);
+  const int G = num_q_heads / hkv;
+  if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16)
+    return fail(GC_ERR_UNSUPPORTED, "%s: q heads per kv head %d not in {1,2,4,8,16}", who, G);
+  if (!(softmax_scale > 0.0f) || softmax_scale == __builtin_inff())
+    return fail(GC_ERR_INVALID_ARG, "%s: softmax_scale must be positive and finite", who);
+  if (batch > 8192) return fail(GC_ERR_UNSUPPORTED, "%s: batch %d > 8192", who, batch);
+  if (batch == 0 || total_new_tokens == 0) {
+    *noop = true;
+    return GC_OK;
+  }
+  if (!q || !out || !block_table || !prefix_lens || !new_lens || !cu_new_lens)
+    return fail(GC_ERR_INVALID_ARG, "%s: NULL array argument", who);
+  if (max_blocks_per_seq == 0)
+    return fail(GC_ERR_INVALID_ARG, "%s: max_blocks_per_seq is 0", who);
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out)) % 16)
+    return fail(GC_ERR_INVALID_ARG, "%s: q / out not 16-byte aligned", who);
+  *a = gc::AttnArgs{q, out, block_table, prefix_lens, new_lens, cu_new_lens, batch,
+                    max_blocks_per_seq, layer, num_q_heads, total_new_tokens, softmax_scale};
+  return GC_OK;
+}
+
+gc_status gc_prefix_prefill_attn(const void* q, const gc_kv_pool* pool, const int32_t* block_table,
+                                 const int32_t* prefix_lens, const int32_t* new_lens, void* out,
+                                 cudaStream_t stream, int32_t layer, const int32_t* cu_new_lens,
+                                 int32_t batch, int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                 float softmax_scale, int32_t total_new_tokens) {
+  g_msg[0] = 0;
+  gc::AttnArgs a;
+  bool noop;
+  gc_status s = attn_common("gc_prefix_prefill_attn", q, pool, block_table, prefix_lens, new_lens,
+                            out, layer, cu_new_lens, batch, max_blocks_per_seq, num_q_heads,
+                            softmax_scale, total_new_tokens, &a, &noop);
+  if (s != GC_OK || noop) return s;
+  return gc::launch_attn_tc(pool, a, stream);
+}
+
+gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* pool,
+                                      const int32_t* block_table, const int32_t* prefix_lens,
+                                      const int32_t* new_lens, void* out, cudaStream_t stream,
+                                      int32_t layer, const int32_t* cu_new_lens, int32_t batch,
+                                      int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                      float softmax_scale, int32_t total_new_tokens) {
+  g_msg[0] = 0;
+  gc::AttnArgs a;
+  bool noop;
+  gc_status s = attn_common("gc_prefix_prefill_attn_simt", q, pool, block_table, prefix_lens,
+                            new_lens, out, layer, cu_new_lens, batch, max_blocks_per_seq,
+                            num_q_heads, softmax_scale, total_new_tokens, &a, &noop);
+  if (s != GC_OK || noop) return s;
+  return gc::launch_attn_simt(pool, a, stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,62 @@
+// Internal declarations shared by the libgc translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "gc.h"
+
+struct gc_kv_pool {
+  gc_pool_config cfg;
+  uint8_t* data;          // KV planes [L][2][num_pages][Hkv][ps][d] bf16
+  size_t data_bytes;
+  int32_t* status;        // device status word (first error recorded by a kernel)
+  void* owned;            // cudaMalloc'd block, or nullptr if caller-owned
+  int device;
+  int num_sms;
+};
+
+namespace gc {
+
+// Thread-local error message; returns `s` for convenient `return fail(...)`.
+gc_status fail(gc_status s, const char* fmt, ...);
+gc_status cuda_fail(cudaError_t e, const char* what);
+
+inline size_t page_bytes(const gc_pool_config& c) {
+  return static_cast<size_t>(c.num_kv_heads) * c.page_size * c.head_dim * 2;
+}
+
+// Record the first device-side error in the pool's status word.
+__device__ __forceinline__ void record_error(int32_t* status, int32_t code) {
+  atomicCAS(status, 0, code);
+}
+
+// ---------------------------------------------------------------- launchers
+// Each returns GC_OK or a status with the message already set.
+gc_status launch_restore_bulk(const gc_kv_pool* pool, const uint8_t* src,
+                              const int32_t* block_ids, int32_t n_blocks, cudaStream_t stream);
+gc_status launch_restore_vector(const gc_kv_pool* pool, const uint8_t* src,
+                                const int32_t* block_ids, int32_t n_blocks, cudaStream_t stream);
+gc_status launch_append(const gc_kv_pool* pool, const void* k_new, const void* v_new,
+                        const int32_t* block_table, const int32_t* prefix_lens,
+                        const int32_t* cu_new_lens, int32_t batch, int32_t max_blocks,
+                        int32_t layer, int32_t total_new_tokens, cudaStream_t stream);
+
+struct AttnArgs {
+  const void* q;
+  void* out;
+  const int32_t* block_table;
+  const int32_t* prefix_lens;
+  const int32_t* new_lens;
+  const int32_t* cu_new_lens;
+  int32_t batch, max_blocks, layer, num_q_heads, total_new_tokens;
+  float softmax_scale;
+};
+
+gc_status launch_attn_simt(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
+gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
+
+}  // namespace gc

@@ -1,0 +1,117 @@
+"""Device-side plumbing around the C ABI for one batch of requests.
+
+``DeviceBatch`` places a :class:`workloads.Workload`'s inputs in device (and
+pinned host) memory with torch, then runs the three steps of the path —
+restore, append, attention — through :mod:`binding`.  It moves inputs and
+allocates buffers only; every result is computed by libgc's kernels.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+from . import binding as gcb
+from .workloads import BF16_NAN, Workload
+
+
+def _i32(a, device):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).to(device)
+
+
+def bf16_tensor(bits: np.ndarray, device="cuda", pin: bool = False):
+    """uint16 bit patterns -> torch.bfloat16 tensor (device, or pinned host)."""
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16)
+    if pin:
+        return t.pin_memory()
+    return t.to(device)
+
+
+def bf16_bits(t) -> np.ndarray:
+    """torch.bfloat16 tensor -> numpy uint16 bit patterns (host copy)."""
+    import torch
+    return t.detach().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+class DeviceBatch:
+    def __init__(self, w: Workload, device: str = "cuda", fill=BF16_NAN, with_restore=True,
+                 staging: bool = True):
+        import torch
+        self.w = w
+        self.device = device
+        self.pool = gcb.KVPool.create(w.L, w.Hkv, w.d, w.ps, w.num_pages, device=device)
+        self.pool.planes().view(torch.int16).fill_(int(np.int16(np.uint16(fill).view(np.int16))))
+        self.block_table = _i32(w.block_table, device)
+        self.prefix_lens = _i32(w.prefix_lens, device)
+        self.new_lens = _i32(w.new_lens, device)
+        self.cu_new_lens = _i32(w.cu_new_lens, device)
+        self.n_blocks = 0
+        if with_restore:
+            ids = w.prefix_blocks()
+            self.n_blocks = int(ids.size)
+            self.block_ids = _i32(ids, device)
+            self.host_src = bf16_tensor(w.host_src(), pin=True) if self.n_blocks else None
+            self.staging = (torch.empty_like(self.host_src, device=device)
+                            if staging and self.n_blocks else None)
+        k, v = w.kv_new()
+        self.k_new = bf16_tensor(k, device)
+        self.v_new = bf16_tensor(v, device)
+        self.q = bf16_tensor(w.q(), device)
+        self.out = torch.full((w.T_new, w.Hq, w.d), float("nan"), dtype=torch.bfloat16,
+                              device=device)
+
+    # ---------------------------------------------------------------- steps
+    def restore(self, stream=None, mode: str = "staged", vector: bool = False):
+        """mode: 'staged' (pinned host -> staging -> pool), 'device' (staging
+        already holds the image: scatter only) or 'zerocopy' (kernel reads
+        pinned host memory)."""
+        if self.n_blocks == 0:
+            return
+        flags = gcb.GC_RESTORE_VECTOR if vector else 0
+        if mode == "staged":
+            gcb.gc_kv_restore(self.pool.handle, self.host_src, self.block_ids, self.n_blocks,
+                              stream, self.staging, flags)
+        elif mode == "device":
+            gcb.gc_kv_restore(self.pool.handle, self.staging, self.block_ids, self.n_blocks,
+                              stream, None, flags | gcb.GC_RESTORE_SRC_DEVICE)
+        elif mode == "zerocopy":
+            gcb.gc_kv_restore(self.pool.handle, self.host_src, self.block_ids, self.n_blocks,
+                              stream, None, flags)
+        else:
+            raise ValueError(mode)
+
+    def stage(self, stream=None):
+        """Copy the pinned image into the device staging buffer (torch copy)."""
+        if self.n_blocks:
+            self.staging.copy_(self.host_src, non_blocking=True)
+
+    def append(self, stream=None, layer: int = 0):
+        w = self.w
+        gcb.gc_kv_append(self.pool.handle, self.k_new, self.v_new, self.block_table,
+                         self.prefix_lens, stream, layer, self.cu_new_lens, w.B, w.max_blocks,
+                         w.T_new)
+
+    def attn(self, stream=None, impl: str = "tc", layer: int = 0, out=None):
+        w = self.w
+        fn = gcb.gc_prefix_prefill_attn if impl == "tc" else gcb.gc_prefix_prefill_attn_simt
+        fn(self.q, self.pool.handle, self.block_table, self.prefix_lens, self.new_lens,
+           self.out if out is None else out, stream, layer, self.cu_new_lens, w.B, w.max_blocks,
+           w.Hq, w.scale, w.T_new)
+
+    def run(self, stream=None, restore_mode: str = "staged", impl: str = "tc"):
+        self.restore(stream, restore_mode)
+        self.append(stream)
+        self.attn(stream, impl)
+
+    def check(self, stream=None) -> int:
+        return self.pool.check(stream)
+
+    def pool_bits(self) -> np.ndarray:
+        return bf16_bits(self.pool.planes())
+
+    def out_f64(self) -> np.ndarray:
+        import torch
+        return self.out.to(torch.float64).cpu().numpy()
+
+    def close(self):
+        self.pool.close()

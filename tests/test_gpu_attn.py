@@ -1,0 +1,211 @@
+"""GPU parity of prefix-reuse attention against the float64 oracle, through
+the C ABI, plus metamorphic checks that need no oracle (bit-exact)."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2505_23970_gb300 import binding as gcb
+from paper_2505_23970_gb300 import workloads as wl
+from paper_2505_23970_gb300.harness import DeviceBatch, _i32, bf16_tensor
+
+from ._util import assert_attn_close, gather_rows, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2505_23970_gb300 import build
+    build.build()
+
+
+def oracle_pool(w):
+    pool = w.empty_pool()
+    if w.prefix_blocks().size:
+        oracle.kv_restore(pool, w.host_src(), w.prefix_blocks())
+    k, v = w.kv_new()
+    oracle.kv_append(pool, 0, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
+    return pool
+
+
+def full_parity(w, impl="tc"):
+    db = DeviceBatch(w)
+    db.run(impl=impl)
+    assert db.check() == gcb.GC_OK
+    got = db.out_f64()
+    db.close()
+    ref = oracle.prefix_attn(w.q(), oracle_pool(w), 0, w.block_table, w.prefix_lens,
+                             w.cu_new_lens, w.scale)
+    return assert_attn_close(got, ref, f"{w.name} [{impl}]")
+
+
+def sampled_parity(w, n_random=512, impl="tc"):
+    db = DeviceBatch(w)
+    db.run(impl=impl)
+    assert db.check() == gcb.GC_OK
+    got = db.out_f64()
+    db.close()
+    rows = sample_rows(w, n_random)
+    ref = oracle.prefix_attn_rows(w.q(), oracle_pool(w), 0, w.block_table, w.prefix_lens,
+                                  w.cu_new_lens, w.scale, rows)
+    return assert_attn_close(gather_rows(got, w, rows), ref, f"{w.name} sampled [{impl}]")
+
+
+# ------------------------------------------------------------ the five configs
+@pytest.mark.parametrize("impl", ["tc", "simt"])
+def test_tiny_config(impl):
+    full_parity(wl.tiny(), impl)
+
+
+@pytest.mark.parametrize("impl", ["tc", "simt"])
+def test_llama3_8b_layer(impl):
+    full_parity(wl.llama3_8b_layer(seed=0), impl)
+
+
+def test_llama3_70b_layer_sampled():
+    sampled_parity(wl.llama3_70b_layer(seed=0), n_random=768)
+
+
+@pytest.mark.parametrize("hit_p", [0.0, 0.5, 1.0])
+def test_conversation_mix_sampled(hit_p):
+    sampled_parity(wl.conversation_mix(seed=1, hit_p=hit_p), n_random=512)
+
+
+def test_long_document_sampled():
+    sampled_parity(wl.long_document(seed=0), n_random=256)
+
+
+def test_long_document_recompute_sampled():
+    sampled_parity(wl.long_document(seed=0, recompute=True), n_random=128)
+
+
+# --------------------------------------------------------------- edge cases
+@pytest.mark.parametrize("G,d,ps", [(1, 128, 16), (2, 64, 32), (4, 64, 16), (8, 128, 64),
+                                    (16, 128, 128), (8, 64, 128), (4, 128, 32)])
+def test_head_grouping_dims_and_page_sizes(G, d, ps):
+    Hkv = 2
+    w = wl.custom(f"g{G}d{d}p{ps}", 4, Hkv * G, Hkv, d, ps, [0, 77, 300, 129], [200, 1, 45, 130],
+                  seed=G * 7 + d + ps)
+    full_parity(w)
+
+
+def test_ragged_lengths_and_empty_requests():
+    """Requests with no new tokens, prefixes ending mid-page, new rows that
+    do not fill a Q tile, a prefix of 0 and one-token requests."""
+    w = wl.custom("ragged", 7, 16, 2, 128, 16, [0, 5, 17, 128, 255, 0, 1000],
+                  [3, 0, 1, 129, 17, 1, 0], seed=3)
+    full_parity(w)
+
+
+def test_batch_with_no_new_tokens_is_noop():
+    import torch
+    w = wl.custom("none", 2, 8, 1, 64, 16, [10, 20], [0, 0], seed=4)
+    db = DeviceBatch(w)
+    db.restore()
+    gcb.gc_prefix_prefill_attn(db.q, db.pool.handle, db.block_table, db.prefix_lens, db.new_lens,
+                               db.out, None, 0, db.cu_new_lens, w.B, w.max_blocks, w.Hq, w.scale,
+                               0)
+    assert db.check() == gcb.GC_OK
+    db.close()
+
+
+def test_single_key_row_returns_v_bit_exact():
+    """prefix 0, row 0: one visible key, so the output is v_0 exactly."""
+    import torch
+    w = wl.custom("single", 3, 8, 2, 128, 16, [0, 0, 0], [1, 5, 130], seed=6)
+    db = DeviceBatch(w)
+    db.run()
+    assert db.check() == gcb.GC_OK
+    cu = w.cu_new_lens
+    _, v = w.kv_new()
+    for b in range(w.B):
+        row = db.out[cu[b]].view(torch.int16).cpu().numpy().view(np.uint16)
+        for h in range(w.Hq):
+            assert np.array_equal(row[h], v[cu[b], h // w.G])
+    db.close()
+
+
+def test_tc_matches_simt_kernel():
+    w = wl.custom("xcheck", 3, 32, 4, 128, 16, [700, 33, 0], [300, 70, 260], seed=8)
+    a = DeviceBatch(w)
+    a.run(impl="tc")
+    b = DeviceBatch(w)
+    b.run(impl="simt")
+    assert a.check() == gcb.GC_OK and b.check() == gcb.GC_OK
+    assert_attn_close(a.out_f64(), b.out_f64(), "tc vs simt")
+    a.close()
+    b.close()
+
+
+# -------------------------------------------------------------- metamorphic
+def test_deterministic_run_to_run():
+    import torch
+    w = wl.llama3_8b_layer(seed=5, B=6)
+    db = DeviceBatch(w)
+    db.run()
+    first = db.out.clone()
+    for _ in range(2):
+        db.out.fill_(0)
+        db.attn()
+        assert torch.equal(db.out.view(torch.int16), first.view(torch.int16))
+    db.close()
+
+
+def test_page_permutation_invariance():
+    """Moving every page elsewhere in the pool (and the block table with it)
+    leaves the output bit-identical."""
+    import torch
+    w = wl.custom("perm", 3, 16, 2, 128, 16, [100, 0, 260], [90, 33, 64], seed=9)
+    a = DeviceBatch(w)
+    a.run()
+    w2 = wl.custom("perm", 3, 16, 2, 128, 16, [100, 0, 260], [90, 33, 64], seed=9)
+    perm = np.random.default_rng(0).permutation(w2.num_pages).astype(np.int32)
+    bt = np.where(w2.block_table >= 0, perm[np.maximum(w2.block_table, 0)], -1).astype(np.int32)
+    w2.block_table = bt
+    w2._cache = dict(w._cache)  # same tensors, new placement
+    b = DeviceBatch(w2)
+    b.run()
+    assert a.check() == gcb.GC_OK and b.check() == gcb.GC_OK
+    assert torch.equal(a.out.view(torch.int16), b.out.view(torch.int16))
+    a.close()
+    b.close()
+
+
+def test_batch_composition_invariance():
+    """A request's output does not depend on the other requests in the batch."""
+    import torch
+    P, n = [300, 17, 1000, 0], [40, 129, 7, 250]
+    w = wl.custom("batch", 4, 32, 4, 128, 16, P, n, seed=10)
+    full = DeviceBatch(w)
+    full.run()
+    assert full.check() == gcb.GC_OK
+    cu = w.cu_new_lens
+    for b in range(4):
+        wb = wl.custom("one", 1, 32, 4, 128, 16, [P[b]], [n[b]], seed=10)
+        # same tensors as request b of the batch
+        pool_src = w.host_src()
+        blocks = [-(-p // 16) for p in P]
+        start = sum(blocks[:b])
+        wb._cache["src"] = pool_src[start:start + blocks[b]]
+        k, v = w.kv_new()
+        wb._cache["kvn"] = (k[cu[b]:cu[b + 1]], v[cu[b]:cu[b + 1]])
+        wb._cache["q"] = w.q()[cu[b]:cu[b + 1]]
+        one = DeviceBatch(wb)
+        one.run()
+        assert one.check() == gcb.GC_OK
+        assert torch.equal(one.out.view(torch.int16), full.out[cu[b]:cu[b + 1]].view(torch.int16))
+        one.close()
+    full.close()
+
+
+def test_bad_block_table_entry_is_reported_not_faulted():
+    w = wl.custom("badbt", 2, 8, 1, 64, 16, [40, 8], [30, 9], seed=11)
+    db = DeviceBatch(w)
+    db.run()
+    assert db.check() == gcb.GC_OK
+    bt = w.block_table.copy()
+    bt[1, 0] = -5
+    db.block_table = _i32(bt, "cuda")
+    db.attn()
+    assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
+    db.close()

@@ -1,0 +1,146 @@
+"""GPU parity of the paged KV restore and append (bit-exact against the
+float64 oracle's index maps), through the C ABI."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2505_23970_gb300 import binding as gcb
+from paper_2505_23970_gb300 import workloads as wl
+from paper_2505_23970_gb300.harness import DeviceBatch, _i32
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2505_23970_gb300 import build
+    build.build()
+
+
+def oracle_pool(w, restore=True, append=True):
+    pool = w.empty_pool()
+    if restore and w.prefix_blocks().size:
+        oracle.kv_restore(pool, w.host_src(), w.prefix_blocks())
+    if append:
+        k, v = w.kv_new()
+        oracle.kv_append(pool, 0, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
+    return pool
+
+
+@pytest.mark.parametrize("mode,vector", [("staged", False), ("staged", True), ("device", False),
+                                         ("zerocopy", False)])
+@pytest.mark.parametrize("make", [wl.tiny, lambda: wl.llama3_8b_layer(seed=1, B=6)])
+def test_restore_bit_exact(make, mode, vector):
+    w = make()
+    db = DeviceBatch(w)
+    if mode == "device":
+        db.stage()
+    db.restore(mode=mode, vector=vector)
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(db.pool_bits(), oracle_pool(w, append=False))
+    db.close()
+
+
+def test_restore_full_80_layer_prefix():
+    """Full 80-layer KV of one 8192-token prefix (80 x 2 x 8 x 128 x 8192
+    bf16 = 2,684,354,560 bytes) from pinned host into a 640-page pool."""
+    w = wl.llama3_70b_restore_80layer()
+    assert w.host_src().nbytes == 2_684_354_560
+    db = DeviceBatch(w)
+    db.restore(mode="staged")
+    assert db.check() == gcb.GC_OK
+    got = db.pool_bits()
+    db.close()
+    assert np.array_equal(got, oracle_pool(w, append=False))
+
+
+def test_restore_skips_out_of_range_block_and_reports_it():
+    w = wl.tiny()
+    db = DeviceBatch(w)
+    ids = w.prefix_blocks().copy()
+    ids[3] = w.num_pages          # one bad id; the others must still land
+    db.block_ids = _i32(ids, "cuda")
+    db.restore(mode="staged")
+    assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
+    ref = w.empty_pool()
+    keep = np.ones(ids.size, bool)
+    keep[3] = False
+    oracle.kv_restore(ref, w.host_src()[keep], ids[keep])
+    assert np.array_equal(db.pool_bits(), ref)
+    assert db.check() == gcb.GC_OK  # the status word was cleared
+    db.close()
+
+
+def test_restore_rejects_pageable_host_memory():
+    w = wl.tiny()
+    db = DeviceBatch(w)
+    pageable = np.zeros(w.host_src().size, dtype=np.uint16)
+    with pytest.raises(gcb.GcError) as e:
+        gcb.gc_kv_restore(db.pool.handle, pageable.ctypes.data, db.block_ids, db.n_blocks, None,
+                          db.staging, 0)
+    assert e.value.status == gcb.GC_ERR_INVALID_ARG
+    db.close()
+
+
+@pytest.mark.parametrize("make", [
+    wl.tiny,
+    lambda: wl.llama3_8b_layer(seed=2),
+    lambda: wl.conversation_mix(seed=3, hit_p=0.5, B=16),
+    lambda: wl.custom("ragged", 5, 8, 2, 64, 32, [0, 31, 32, 33, 100], [1, 0, 64, 5, 31], seed=4),
+])
+def test_append_bit_exact(make):
+    w = make()
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(db.pool_bits(), oracle_pool(w))
+    db.close()
+
+
+def test_append_reports_bad_page():
+    w = wl.custom("badpage", 2, 4, 1, 64, 16, [16, 3], [20, 4], seed=5)
+    bt = w.block_table.copy()
+    bt[0, 2] = w.num_pages + 7    # tokens 32..35 of request 0 have no valid page
+    db = DeviceBatch(w)
+    db.block_table = _i32(bt, "cuda")
+    db.restore()
+    db.append()
+    assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
+    db.close()
+
+
+def test_zero_sizes_are_noops():
+    w = wl.tiny()
+    db = DeviceBatch(w)
+    before = db.pool_bits()
+    gcb.gc_kv_restore(db.pool.handle, db.host_src, db.block_ids, 0, None, db.staging, 0)
+    gcb.gc_kv_append(db.pool.handle, db.k_new, db.v_new, db.block_table, db.prefix_lens, None, 0,
+                     db.cu_new_lens, 0, w.max_blocks, 0)
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(db.pool_bits(), before)
+    db.close()
+
+
+def test_library_owned_pool_matches_caller_owned():
+    """A pool whose memory the library allocates itself gives the same
+    attention output, bit for bit, as one in caller-owned memory."""
+    import torch
+    w = wl.tiny()
+    db = DeviceBatch(w)
+    db.run()
+    ref = db.out.clone()
+    cfg = gcb.make_config(w.L, w.Hkv, w.d, w.ps, w.num_pages)
+    h = gcb.gc_kv_pool_create(cfg)
+    ptr, nbytes = gcb.gc_kv_pool_data(h)
+    assert ptr and nbytes == int(np.prod(w.pool_shape)) * 2
+    gcb.gc_kv_restore(h, db.host_src, db.block_ids, db.n_blocks, None, db.staging, 0)
+    gcb.gc_kv_append(h, db.k_new, db.v_new, db.block_table, db.prefix_lens, None, 0,
+                     db.cu_new_lens, w.B, w.max_blocks, w.T_new)
+    out = torch.full_like(ref, float("nan"))
+    gcb.gc_prefix_prefill_attn(db.q, h, db.block_table, db.prefix_lens, db.new_lens, out, None,
+                               0, db.cu_new_lens, w.B, w.max_blocks, w.Hq, w.scale, w.T_new)
+    assert gcb.gc_kv_pool_check(h) == gcb.GC_OK
+    gcb.gc_kv_pool_destroy(h)
+    assert torch.equal(out.view(torch.int16), ref.view(torch.int16))
+    db.close()
