@@ -1,0 +1,491 @@
+#!/usr/bin/env python3
+"""Benchmark of prefix-reuse prefill on GB300: one step = restore of the
+cached prefix KV into the paged pool + append of the new tokens' KV +
+causal GQA attention of the new tokens over [prefix ++ new], for one layer
+of the Llama-3-70B-shaped workload (8 requests x 8192 cached + 1024 new
+tokens, 64 q heads / 8 kv heads, d 128, page size 16).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  `value` is new-token prefill throughput of
+the whole step with inputs already in HBM (restore reads a device staging
+buffer); `e2e` is the same metric through the C ABI with the step's inputs
+copied from pinned host memory (prefix pages, q, new K/V) and the output
+copied back inside the timed region.  Under torchrun each rank runs an
+independent replica on its own batch (the path has no exchange step).
+`--impl reference` times the float64 CPU oracle on the host cores instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "new-token prefill tok/s & attn TFLOP/s vs bf16 peak; KV restore GB/s vs HBM"
+WORKLOAD = "llama3-70b-layer"
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def make_workload(name: str, seed: int):
+    from paper_2505_23970_gb300 import workloads as wl
+    if name == "70b":
+        return wl.llama3_70b_layer(seed=seed)
+    if name == "8b":
+        return wl.llama3_8b_layer(seed=seed)
+    if name == "tiny":
+        return wl.tiny(seed=seed)
+    if name.startswith("mix"):
+        return wl.conversation_mix(seed=seed, hit_p=float(name[3:] or 1.0))
+    if name == "long":
+        return wl.long_document(seed=seed)
+    if name == "long-recompute":
+        return wl.long_document(seed=seed, recompute=True)
+    raise ValueError(name)
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while running."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.gpu)],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                rows.append((float(f[1]), float(f[2]), float(f[3]), f[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        # samples under load: power above the idle floor
+        pmax = max(r[2] for r in rows)
+        load = [r for r in rows if r[2] >= 0.5 * pmax] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in load for k, v in enumerate(r[3]) if v == "Active"})
+        return {"sm_mhz": statistics.median(r[0] for r in load), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(load), "power_w_max": pmax}
+
+
+# ------------------------------------------------------------- distributed
+def dist_setup(n_gpus: int):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl"
+        import torch
+        if not torch.cuda.is_available():
+            backend = "gloo"
+        else:
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ------------------------------------------------------------ CPU oracle
+def oracle_sample(w, seconds: float, rng, pool=None, threads=None):
+    """Time the float64 oracle on a bounded sample of one step and
+    extrapolate the full step: restore of a block subset, the full append,
+    attention of random (b, h, i) rows until `seconds` have passed."""
+    import oracle
+    threads = threads or os.cpu_count() or 1
+    if pool is None:
+        pool = w.empty_pool()
+    ids = w.prefix_blocks()
+    nb = min(ids.size, 256)
+    t0 = time.perf_counter()
+    if nb:
+        oracle.kv_restore(pool, w.host_src()[:nb], ids[:nb])
+    t_restore = (time.perf_counter() - t0) * (ids.size / max(nb, 1))
+    if nb < ids.size:  # the rest of the image, untimed, so attention reads real keys
+        oracle.kv_restore(pool, w.host_src()[nb:], ids[nb:])
+    k, v = w.kv_new()
+    t0 = time.perf_counter()
+    oracle.kv_append(pool, 0, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
+    t_append = time.perf_counter() - t0
+    nonempty = np.flatnonzero(w.new_lens > 0)
+    rows_done, t_attn = 0, 0.0
+    q = w.q()
+    batch = max(threads * 4, 16)
+    while t_attn < seconds:
+        bsel = rng.choice(nonempty, batch)
+        rows = np.stack([bsel, rng.integers(0, w.Hq, batch),
+                         (rng.random(batch) * w.new_lens[bsel]).astype(np.int64)], 1).astype(np.int32)
+        t0 = time.perf_counter()
+        oracle.prefix_attn_rows(q, pool, 0, w.block_table, w.prefix_lens, w.cu_new_lens, w.scale,
+                                rows, nthreads=threads)
+        t_attn += time.perf_counter() - t0
+        rows_done += batch
+    total_rows = w.T_new * w.Hq
+    t_step = t_restore + t_append + t_attn * total_rows / rows_done
+    return {"t_step_s": t_step, "rows": rows_done, "restore_blocks": int(nb),
+            "threads": threads, "t_attn_s": t_attn, "pool": pool}
+
+
+def cpu_baseline_entry(w, seconds=12.0, seed=0):
+    s = oracle_sample(w, seconds, np.random.default_rng(seed))
+    return {"value": w.T_new / s["t_step_s"], "unit": "tok/s", "cores": s["threads"],
+            "kind": "oracle",
+            "sample": (f"float64 C oracle on {s['threads']} host threads: restore of "
+                       f"{s['restore_blocks']} of {w.prefix_blocks().size} blocks, full append, "
+                       f"attention of {s['rows']} random (request, head, row) rows of "
+                       f"{w.T_new * w.Hq}; step time extrapolated per block / per row")}
+
+
+def run_reference(args):
+    world, rank, _ = dist_setup(args.gpus)
+    if rank != 0:
+        return
+    w = make_workload(args.config, args.seed)
+    rng = np.random.default_rng(args.seed)
+    pool = None
+    per_step = max(1.0, min(6.0, 150.0 / max(args.steps + args.warmup, 1)))
+    for _ in range(args.warmup):
+        s = oracle_sample(w, per_step / 2, rng, pool)
+        pool = s["pool"]
+    times = []
+    last = None
+    for _ in range(args.steps):
+        last = oracle_sample(w, per_step, rng, pool)
+        pool = last["pool"]
+        times.append(last["t_step_s"])
+    t = statistics.mean(times)
+    value = w.T_new / t
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tok/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": t * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "batch": w.B, "prefix_len": int(w.prefix_lens[0]),
+                       "new_len": int(w.new_lens[0]), "q_heads": w.Hq, "kv_heads": w.Hkv,
+                       "head_dim": w.d, "page_size": w.ps, "parallelism": "replicas",
+                       "l2": "n/a (host)"},
+            "cpu_baseline": {"value": value, "unit": "tok/s", "cores": last["threads"],
+                             "kind": "oracle",
+                             "sample": f"each step: {last['rows']} random attention rows, "
+                                       f"{last['restore_blocks']} restored blocks, full append; "
+                                       "extrapolated to the full step"},
+            "e2e": {"value": value, "unit": "tok/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------- GPU arm
+def traffic_record(kernel: str, workload: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel source."""
+    import hashlib
+    p = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.json")
+    src = os.path.join(ROOT, "paper_2505_23970_gb300", "csrc", "attn_tc.cu" if kernel.startswith(
+        "attn") else "kv_copy.cu")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p))
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    return d.get("dram_bytes_per_launch") if d.get("src_sha") == sha else None
+
+
+def run_ours(args):
+    import torch
+
+    from paper_2505_23970_gb300 import binding as gcb
+    from paper_2505_23970_gb300.harness import DeviceBatch, bf16_tensor
+
+    world, rank, local = dist_setup(args.gpus)
+    torch.cuda.set_device(local)
+    pk = peaks()
+    w = make_workload(args.config, args.seed + rank)
+    db = DeviceBatch(w, device=f"cuda:{local}")
+    db.stage()
+    stream = torch.cuda.current_stream()
+    flops = w.attn_flops()
+    restore_payload = db.n_blocks * w.page_bytes
+    T_new = w.T_new
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        gcb.gc_kv_restore(db.pool.handle, db.staging, db.block_ids, db.n_blocks, stream, None,
+                          gcb.GC_RESTORE_SRC_DEVICE)
+        if ev:
+            ev[1].record(stream)
+        db.append(stream)
+        if ev:
+            ev[2].record(stream)
+        db.attn(stream)
+        if ev:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    status = db.check(stream)
+    if status != gcb.GC_OK:
+        raise RuntimeError(f"device status {gcb.status_name(status)} after warm-up")
+
+    sampler = ClockSampler(local) if not args.profile else None
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
+    barrier(world)
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for k in range(args.steps):
+        step(evs[k])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clocks = sampler.stop() if sampler else None
+    ms = t_start.elapsed_time(t_end) / args.steps
+    status = db.check(stream)
+    if status != gcb.GC_OK:
+        raise RuntimeError(f"device status {gcb.status_name(status)} in the timed region")
+    restore_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    append_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in evs)
+    attn_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in evs)
+    ms_max = max_over_ranks(ms, world)
+    value = world * T_new / (ms_max / 1e3)
+
+    if args.profile:
+        if rank == 0:
+            print(json.dumps({"profile_run": True, "ms_per_step": ms, "attn_ms": attn_ms}))
+        return
+
+    # ---- end to end through the C ABI with host buffers
+    e2e = None
+    if not args.no_e2e:
+        q_h = bf16_tensor(w.q(), pin=True)
+        k, v = w.kv_new()
+        k_h, v_h = bf16_tensor(k, pin=True), bf16_tensor(v, pin=True)
+        out_h = torch.empty(db.out.shape, dtype=torch.bfloat16).pin_memory()
+        h2d = q_h.numel() * 2 + k_h.numel() * 2 + v_h.numel() * 2 + restore_payload
+        d2h = out_h.numel() * 2
+
+        def e2e_step():
+            db.q.copy_(q_h, non_blocking=True)
+            db.k_new.copy_(k_h, non_blocking=True)
+            db.v_new.copy_(v_h, non_blocking=True)
+            gcb.gc_kv_restore(db.pool.handle, db.host_src, db.block_ids, db.n_blocks, stream,
+                              db.staging, 0)
+            db.append(stream)
+            db.attn(stream)
+            out_h.copy_(db.out, non_blocking=True)
+
+        for _ in range(args.warmup):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        e2e_ms = max_over_ranks(a.elapsed_time(b) / args.steps, world)
+        e2e = {"value": world * T_new / (e2e_ms / 1e3), "unit": "tok/s",
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "ms_per_step": e2e_ms, "gpu_launches_per_step": 3}
+        if db.check(stream) != gcb.GC_OK:
+            raise RuntimeError("device status after the end-to-end loop")
+
+    # ---- restore of the full 80-layer KV of one 8192-token prefix
+    restore80 = None
+    if not args.no_restore80 and rank == 0:
+        restore80 = bench_restore80(args, pk)
+
+    attn_tflops = flops / (attn_ms / 1e3) / 1e12
+    restore_gbs = 2 * restore_payload / (restore_ms / 1e3) / 1e9
+    peak_t = pk["bf16_tflops"]
+    line = {
+        "metric": METRIC, "value": value, "unit": "tok/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "batch": w.B, "prefix_len": int(w.prefix_lens[0]),
+                   "new_len": int(w.new_lens[0]), "q_heads": w.Hq, "kv_heads": w.Hkv,
+                   "head_dim": w.d, "page_size": w.ps, "pool_pages": w.num_pages,
+                   "parallelism": "replicas" if world > 1 else "single",
+                   "l2": "inputs larger than L2 (q 134 MB, paged K/V 302 MB, staging 268 MB)",
+                   "step": "restore scatter (device staging -> pool) + append + attention"},
+        "roofline": {"bound": "tensor", "achieved": attn_tflops, "peak": peak_t,
+                     "unit": "TFLOP/s", "frac": attn_tflops / peak_t,
+                     "traffic": traffic_record("attn_tc", WORKLOAD),
+                     "kernel": "attn_tc_kernel<128>", "peak_source": pk["source"] + " burst",
+                     "frac_of_sustained": (attn_tflops / pk["bf16_tflops_sustained"]
+                                           if pk.get("bf16_tflops_sustained") else None),
+                     "flops_per_launch": flops, "ms_per_launch": attn_ms},
+        "roofline_restore": {"bound": "hbm", "achieved": restore_gbs, "peak": pk["hbm_gbs"],
+                             "unit": "GB/s", "frac": restore_gbs / pk["hbm_gbs"],
+                             "traffic": traffic_record("restore_bulk", WORKLOAD),
+                             "kernel": "restore_bulk_kernel",
+                             "bytes_per_launch": 2 * restore_payload, "ms_per_launch": restore_ms},
+        "breakdown_ms": {"restore": restore_ms, "append": append_ms, "attention": attn_ms},
+        "attn_tflops": attn_tflops, "restore_gbs": restore_gbs,
+        "e2e": e2e, "restore_80layer": restore80, "clocks": clocks,
+        "gpu_launches": 3 * args.steps,
+    }
+    if world == 1 and rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_entry(w, seconds=args.cpu_seconds, seed=args.seed)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def bench_restore80(args, pk):
+    """Restore of the 80-layer KV of one 8192-token prefix (2.68 GB): the
+    scatter from a device staging buffer (read + write bytes vs HBM) and the
+    whole pinned host -> pool path (payload bytes), next to a plain pinned
+    host -> device cudaMemcpyAsync of the same bytes."""
+    import torch
+
+    from paper_2505_23970_gb300 import binding as gcb
+    from paper_2505_23970_gb300 import workloads as wl
+    from paper_2505_23970_gb300.harness import DeviceBatch
+
+    w = wl.llama3_70b_restore_80layer(seed=args.seed)
+    db = DeviceBatch(w)
+    payload = db.n_blocks * w.page_bytes
+    stream = torch.cuda.current_stream()
+    reps = 10
+
+    def timed(fn):
+        for _ in range(2):
+            fn()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    db.stage()
+    scatter_ms = timed(lambda: gcb.gc_kv_restore(db.pool.handle, db.staging, db.block_ids,
+                                                 db.n_blocks, stream, None,
+                                                 gcb.GC_RESTORE_SRC_DEVICE))
+    vec_ms = timed(lambda: gcb.gc_kv_restore(db.pool.handle, db.staging, db.block_ids,
+                                             db.n_blocks, stream, None,
+                                             gcb.GC_RESTORE_SRC_DEVICE | gcb.GC_RESTORE_VECTOR))
+    staged_ms = timed(lambda: gcb.gc_kv_restore(db.pool.handle, db.host_src, db.block_ids,
+                                                db.n_blocks, stream, db.staging, 0))
+    zc_ms = timed(lambda: gcb.gc_kv_restore(db.pool.handle, db.host_src, db.block_ids,
+                                            db.n_blocks, stream, None, 0))
+    h2d_ms = timed(lambda: db.staging.copy_(db.host_src, non_blocking=True))
+    ok = db.check(stream) == gcb.GC_OK
+    db.close()
+    gbs = lambda nbytes, ms: nbytes / (ms / 1e3) / 1e9  # noqa: E731
+    return {
+        "payload_bytes": payload, "device_status_ok": ok,
+        "scatter_bulk_gbs": gbs(2 * payload, scatter_ms),
+        "scatter_bulk_frac_hbm": gbs(2 * payload, scatter_ms) / pk["hbm_gbs"],
+        "scatter_vector_gbs": gbs(2 * payload, vec_ms),
+        "host_to_pool_staged_gbs": gbs(payload, staged_ms),
+        "host_to_pool_zero_copy_gbs": gbs(payload, zc_ms),
+        "pinned_h2d_memcpy_gbs": gbs(payload, h2d_ms),
+        "ms": {"scatter_bulk": scatter_ms, "scatter_vector": vec_ms, "staged": staged_ms,
+               "zero_copy": zc_ms, "h2d_memcpy": h2d_ms},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="70b",
+                    help="70b (default), 8b, tiny, mix<p>, long, long-recompute")
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-restore80", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--profile", action="store_true",
+                    help="timed loop only (for ncu launch lists): no e2e, clocks or baselines")
+    args = ap.parse_args()
+    if args.warmup < 3 and not args.profile:
+        ap.error("--warmup must be >= 3")
+    global WORKLOAD
+    WORKLOAD = {"70b": "llama3-70b-layer", "8b": "llama3-8b-layer", "tiny": "tiny",
+                "long": "long-document", "long-recompute": "long-document-recompute"}.get(
+                    args.config, f"conversation-{args.config}")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()
