@@ -15,10 +15,16 @@
 //      warp 0        TMA producer: Q tiles (3-D map over [T_new][Hq][d]) and
 //                    K/V tiles page by page (2-D map over the pool rows);
 //                    zeroes V rows past the end of the sequence.
-//      warp 1        TMEM owner; lane 0 issues every tcgen05.mma:
+//      warp 1        TMEM owner; lane 0 is the MMA issuer:
 //                      S_i = Q_i K^T   (SS, both operands K-major, fp32 in TMEM)
 //                      O_i += P_i V    (TS: P_i read from TMEM, V MN-major)
+//                    It polls the readiness of every pending MMA of both Q
+//                    tiles and issues each whole MMA as soon as its inputs
+//                    are ready, so the tensor pipe serialises the two tiles'
+//                    S -> softmax -> PV chains into a staggered schedule in
+//                    which one tile's softmax overlaps the other's MMAs.
 //      warps 4-7     softmax of Q tile 0; warps 8-11 softmax of Q tile 1.
+//    Warps 0-3 give registers to the softmax warpgroups (setmaxnreg).
 //                    One thread per row: S row from TMEM, causal mask, online
 //                    softmax in the log2 domain with lazy rescaling (the
 //                    reference max moves only when a row max grows by more
@@ -26,8 +32,8 @@
 //                    1/l normalisation and the bf16 store of O.
 //  * TMEM (512 columns): S0 [0,128) S1 [128,256) O0 [256,256+d) O1 [.., +d).
 //    P_i overwrites the first 64 columns of S_i.  Because P_i aliases S_i,
-//    S_i(j+1) is issued only after PV_i(j) has completed; the MMA order
-//    S0 S1 PV0 PV1 keeps the tensor pipe fed while it waits.
+//    S_i(j+1) is issued only after PV_i(j) has completed; the other Q
+//    tile's MMAs keep the tensor pipe fed meanwhile.
 //  * Every mbarrier wait is bounded; a timeout raises the CTA's abort flag,
 //    all roles leave their loops, in-flight copies and MMAs are drained, TMEM
 //    is freed and GC_ERR_TIMEOUT is recorded in the pool status word.
@@ -42,6 +48,10 @@ namespace {
 using namespace ptx;
 
 constexpr int kThreads = 384;
+constexpr int kRegsProducer = 88;   // warps 0-3 after setmaxnreg.dec
+constexpr int kRegsSoftmax = 200;   // warps 4-11 after setmaxnreg.inc
+static_assert(128 * kRegsProducer + 256 * kRegsSoftmax <= kThreads * 168,
+              "register split exceeds the launch allocation");
 constexpr int kTileM = 128;     // rows per Q tile
 constexpr int kTileN = 128;     // keys per K/V tile
 constexpr float kRescaleLog2 = 8.0f;
@@ -122,10 +132,8 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
   const int lane = threadIdx.x & 31;
   volatile int* abortp = &bar.abort_flag;
   uint32_t q_count = 0, kv_count = 0, vfix_count = 0;
-  int armed_slot_parity[C::kStages];
+  uint32_t armed = 0, armed_par = 0;  // per slot: a load in flight, and its phase parity
   int armed_q = -1, armed_vfix = -1;
-#pragma unroll
-  for (int s = 0; s < C::kStages; ++s) armed_slot_parity[s] = -1;
   bool ok = true;
   const uint32_t box_bytes = static_cast<uint32_t>(geo.ps) * 128;  // one page, one column block
 
@@ -157,6 +165,20 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
       const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
+      const int blk0 = key0 >> geo.ps_shift;
+      int pages[kTileN / 16];
+      int good = 0;
+#pragma unroll
+      for (int pg = 0; pg < kTileN / 16; ++pg) {
+        int page = -1;
+        if (pg < npages && blk0 + pg < geo.max_blocks) page = __ldg(block_table + bt_row + blk0 + pg);
+        if (pg < npages && (page < 0 || page >= geo.num_pages)) {
+          if (lane == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
+          page = -1;
+        }
+        pages[pg] = page;
+        good += page >= 0;
+      }
 #pragma unroll 1
       for (int kv = 0; kv < 2; ++kv) {
         const int slot = kv_count % C::kStages;
@@ -166,22 +188,12 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
         const bool fix = kv == 1 && nkeys < kTileN;
         uint64_t* full = fix ? &bar.vfix : &bar.kv_full[slot];
         if (lane == 0) {
-          int good = 0;
-          for (int pg = 0; pg < npages; ++pg) {
-            const int blk = (key0 >> geo.ps_shift) + pg;
-            const int page = blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
-            good += (page >= 0 && page < geo.num_pages);
-          }
           mbar_arrive_expect_tx(full, static_cast<uint32_t>(good) * box_bytes * C::kHalves);
-          for (int pg = 0; pg < npages; ++pg) {
-            const int blk = (key0 >> geo.ps_shift) + pg;
-            const int page = blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
-            if (page < 0 || page >= geo.num_pages) {
-              record_error(status, GC_ERR_OUT_OF_RANGE);
-              continue;
-            }
-            const int row = (((geo.layer * 2 + kv) * geo.num_pages + page) * geo.Hkv + w.g)
-                            << geo.ps_shift;
+          const int plane_row = (geo.layer * 2 + kv) * geo.num_pages;
+#pragma unroll
+          for (int pg = 0; pg < kTileN / 16; ++pg) {
+            if (pages[pg] < 0) continue;
+            const int row = (((plane_row + pages[pg]) * geo.Hkv + w.g) << geo.ps_shift);
 #pragma unroll
             for (int h = 0; h < C::kHalves; ++h)
               tma_load_2d(dst + h * C::kHalfBytes + pg * box_bytes, map_kv, full, h * 64, row);
@@ -192,7 +204,7 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
           // their P is zero but 0 * NaN would poison the PV product.
           ok = mbar_wait(&bar.vfix, vfix_count & 1, abortp);
           if (!ok) {
-            armed_slot_parity[slot] = -1;
+            armed &= ~(1u << slot);
             armed_vfix = vfix_count & 1;
             break;
           }
@@ -206,7 +218,8 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar.kv_full[slot]);
         } else {
-          armed_slot_parity[slot] = (kv_count / C::kStages) & 1;
+          armed |= 1u << slot;
+          armed_par = (armed_par & ~(1u << slot)) | (((kv_count / C::kStages) & 1u) << slot);
         }
         ++kv_count;
       }
@@ -218,7 +231,7 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
     if (armed_q >= 0) mbar_wait(&bar.q_full, armed_q, &no_abort);
     if (armed_vfix >= 0) mbar_wait(&bar.vfix, armed_vfix, &no_abort);
     for (int s = 0; s < C::kStages; ++s)
-      if (armed_slot_parity[s] >= 0) mbar_wait(&bar.kv_full[s], armed_slot_parity[s], &no_abort);
+      if (armed & (1u << s)) mbar_wait(&bar.kv_full[s], (armed_par >> s) & 1u, &no_abort);
   }
 }
 
@@ -231,11 +244,9 @@ __device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uin
   using C = Cfg<D>;
   volatile int* abortp = &bar.abort_flag;
   uint32_t q_count = 0, kv_count = 0;
-  uint32_t pv_issued[2] = {0, 0}, pv_waited[2] = {0, 0}, p_count[2] = {0, 0};
+  uint32_t p_cons[2] = {0, 0}, pv_issued[2] = {0, 0}, pv_acked[2] = {0, 0};
   bool ok = true;
-  const uint32_t q_base = smem_addr(smem_q), kv_base = smem_addr(smem_kv);
-  const uint32_t col_s[2] = {C::kColS0, C::kColS1};
-  const uint32_t col_o[2] = {C::kColO0, C::kColO1};
+  const uint32_t q_base = smem_addr(smem_q), kv_smem = smem_addr(smem_kv);
 
   for (int it = blockIdx.x; ok && it < total_items; it += gridDim.x) {
     Item w;
@@ -244,60 +255,87 @@ __device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uin
     ++q_count;
     if (!ok) break;
     tc_fence_after();
-    for (int j = 0; ok && j < w.nt; ++j) {
-      // ---- S_i = Q_i K_j^T
-      const int ks = kv_count % C::kStages;
-      ok = mbar_wait(&bar.kv_full[ks], (kv_count / C::kStages) & 1, abortp);
-      ++kv_count;
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t k_addr = kv_base + ks * C::kTileBytes;
+    // K_j sits in ring use kv_base + 2j, V_j in use kv_base + 2j + 1
+    const uint32_t kv_base = kv_count;
+    int s_next[2] = {0, 0}, pv_next[2] = {0, 0};
+    int kfront = 0, vfront = 0;
+    bool q_released = false;
+    long long last = clock64();
+    while (true) {
+      bool progressed = false;
 #pragma unroll
       for (int i = 0; i < 2; ++i) {
-        if (j >= w.nt_i[i]) continue;
-        if (pv_issued[i] > pv_waited[i]) {  // P_i aliases S_i: PV_i must be done
-          ok = mbar_wait(&bar.pv_done[i], (pv_issued[i] - 1) & 1, abortp);
-          if (!ok) break;
-          pv_waited[i] = pv_issued[i];
-          tc_fence_after();
+        const uint32_t col_s = i ? C::kColS1 : C::kColS0;
+        const uint32_t col_o = i ? C::kColO1 : C::kColO0;
+        // O_i += P_i V_j once the softmax has written P_i(j)
+        int j = pv_next[i];
+        if (j < s_next[i]) {
+          const uint32_t use = kv_base + 2 * j + 1;
+          if (mbar_test(&bar.p_full[i], p_cons[i] & 1) &&
+              mbar_test(&bar.kv_full[use % C::kStages], (use / C::kStages) & 1)) {
+            tc_fence_after();
+            const uint32_t v_addr = kv_smem + (use % C::kStages) * C::kTileBytes;
+#pragma unroll
+            for (int kk = 0; kk < kTileN / 16; ++kk)
+              mma_ts(tmem + col_o, tmem + col_s + kk * 8,
+                     sdesc_sw128(v_addr + kk * 16 * 128, C::kHalfBytes, 1024), C::kIdescPV,
+                     (j > 0 || kk > 0) ? 1u : 0u);
+            mma_commit(&bar.pv_done[i]);
+            ++pv_issued[i];
+            ++p_cons[i];
+            ++pv_next[i];
+            progressed = true;
+          }
         }
-        const uint32_t q_addr = q_base + i * C::kTileBytes;
+        // S_i = Q_i K_j^T once PV_i(j-1) has finished reading P_i (it aliases S_i)
+        j = s_next[i];
+        if (j < w.nt_i[i] && pv_next[i] == j) {
+          const uint32_t use = kv_base + 2 * j;
+          const bool alias_free = pv_acked[i] == pv_issued[i] ||
+                                  mbar_test(&bar.pv_done[i], (pv_issued[i] - 1) & 1);
+          if (alias_free && mbar_test(&bar.kv_full[use % C::kStages], (use / C::kStages) & 1)) {
+            pv_acked[i] = pv_issued[i];
+            tc_fence_after();
+            const uint32_t k_addr = kv_smem + (use % C::kStages) * C::kTileBytes;
+            const uint32_t q_addr = q_base + i * C::kTileBytes;
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * C::kHalfBytes + (kk & 3) * 32;
-          mma_ss(tmem + col_s[i], sdesc_sw128(q_addr + off, 16, 1024),
-                 sdesc_sw128(k_addr + off, 16, 1024), C::kIdescQK, kk > 0);
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * C::kHalfBytes + (kk & 3) * 32;
+              mma_ss(tmem + col_s, sdesc_sw128(q_addr + off, 16, 1024),
+                     sdesc_sw128(k_addr + off, 16, 1024), C::kIdescQK, kk > 0);
+            }
+            mma_commit(&bar.s_full[i]);
+            ++s_next[i];
+            progressed = true;
+          }
         }
-        mma_commit(&bar.s_full[i]);
       }
-      if (!ok) break;
-      mma_commit(&bar.kv_empty[ks]);
-      if (j == w.nt - 1) mma_commit(&bar.q_empty);
-      // ---- O_i += P_i V_j
-      const int vs = kv_count % C::kStages;
-      ok = mbar_wait(&bar.kv_full[vs], (kv_count / C::kStages) & 1, abortp);
-      ++kv_count;
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t v_addr = kv_base + vs * C::kTileBytes;
-#pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        if (j >= w.nt_i[i]) continue;
-        ok = mbar_wait(&bar.p_full[i], p_count[i] & 1, abortp);
-        ++p_count[i];
-        if (!ok) break;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < kTileN / 16; ++kk)
-          mma_ts(tmem + col_o[i], tmem + col_s[i] + kk * 8,
-                 sdesc_sw128(v_addr + kk * 16 * 128, C::kHalfBytes, 1024), C::kIdescPV,
-                 (j > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(&bar.pv_done[i]);
-        ++pv_issued[i];
+      // release ring slots whose last reader has been issued (the commit
+      // arrives once those MMAs complete), and the Q tiles after their last S
+      while (kfront < w.nt && (s_next[0] > kfront || kfront >= w.nt_i[0]) &&
+             (s_next[1] > kfront || kfront >= w.nt_i[1])) {
+        mma_commit(&bar.kv_empty[(kv_base + 2 * kfront) % C::kStages]);
+        ++kfront;
       }
-      if (!ok) break;
-      mma_commit(&bar.kv_empty[vs]);
+      while (vfront < w.nt && (pv_next[0] > vfront || vfront >= w.nt_i[0]) &&
+             (pv_next[1] > vfront || vfront >= w.nt_i[1])) {
+        mma_commit(&bar.kv_empty[(kv_base + 2 * vfront + 1) % C::kStages]);
+        ++vfront;
+      }
+      if (!q_released && s_next[0] == w.nt_i[0] && s_next[1] == w.nt_i[1]) {
+        mma_commit(&bar.q_empty);
+        q_released = true;
+      }
+      if (kfront == w.nt && vfront == w.nt) break;
+      if (progressed) {
+        last = clock64();
+      } else if (*abortp || clock64() - last > kWaitCycles) {
+        *abortp = 1;
+        ok = false;
+        break;
+      }
     }
+    kv_count = kv_base + 2 * w.nt;
   }
   // wait for every MMA this thread issued before TMEM is released
   mma_commit(&bar.drain);
@@ -305,8 +343,8 @@ __device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uin
   mbar_wait(&bar.drain, 0, &no_abort);
 }
 
-template <int D>
-__device__ void softmax_wg(int i, Barriers& bar, uint32_t tmem, const int* item_start,
+template <int D, int i>
+__device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
                            int total_items, const Geom& geo,
                            const int32_t* __restrict__ prefix_lens,
                            const int32_t* __restrict__ new_lens,
@@ -340,22 +378,24 @@ __device__ void softmax_wg(int i, Barriers& bar, uint32_t tmem, const int* item_
       for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
       tmem_wait_ld();
       const int key0 = j * kTileN;
-      float mt = -INFINITY;
       if (key0 + kTileN - 1 > kmax) {
 #pragma unroll
         for (int c = 0; c < 4; ++c)
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const float v = key0 + c * 32 + e > kmax ? -INFINITY : __uint_as_float(sr[c][e]);
-            sr[c][e] = __float_as_uint(v);
-            mt = fmaxf(mt, v);
-          }
-      } else {
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-#pragma unroll
-          for (int e = 0; e < 32; ++e) mt = fmaxf(mt, __uint_as_float(sr[c][e]));
+          for (int e = 0; e < 32; ++e)
+            if (key0 + c * 32 + e > kmax) sr[c][e] = __float_as_uint(-INFINITY);
       }
+      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+#pragma unroll
+        for (int e = 0; e < 32; e += 8) {
+          mx[0] = fmax3(mx[0], __uint_as_float(sr[c][e + 0]), __uint_as_float(sr[c][e + 1]));
+          mx[1] = fmax3(mx[1], __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
+          mx[2] = fmax3(mx[2], __uint_as_float(sr[c][e + 4]), __uint_as_float(sr[c][e + 5]));
+          mx[3] = fmax3(mx[3], __uint_as_float(sr[c][e + 6]), __uint_as_float(sr[c][e + 7]));
+        }
+      const float mt = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
       const float mt2 = mt * geo.scale_log2;
       if (__any_sync(0xffffffffu, mt2 > m_run + kRescaleLog2)) {
         const float m_new = fmaxf(m_run, mt2);
@@ -375,21 +415,32 @@ __device__ void softmax_wg(int i, Barriers& bar, uint32_t tmem, const int* item_
         l *= alpha;
         m_run = m_new;
       }
-      const float neg_m = -m_run;
-      float lsum0 = 0.f, lsum1 = 0.f;
+      // p = 2^(s * scale*log2(e) - m), two columns per paired FMA
+      const uint64_t sc2 = f2_pack(geo.scale_log2, geo.scale_log2);
+      const uint64_t nm2 = f2_pack(-m_run, -m_run);
+      uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         uint32_t pk[16];
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
-          const float p0 = ex2_approx(fmaf(__uint_as_float(sr[c][2 * e]), geo.scale_log2, neg_m));
-          const float p1 =
-              ex2_approx(fmaf(__uint_as_float(sr[c][2 * e + 1]), geo.scale_log2, neg_m));
-          lsum0 += p0;
-          lsum1 += p1;
+          const uint64_t t = f2_fma(f2_pack(__uint_as_float(sr[c][2 * e]),
+                                            __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
+          float t0, t1;
+          f2_unpack(t, t0, t1);
+          const float p0 = ex2_approx(t0), p1 = ex2_approx(t1);
+          acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
           pk[e] = pack_bf16x2(p0, p1);
         }
         tmem_st16(tS + c * 16, pk);
+      }
+      float lsum0, lsum1, lsum2, lsum3;
+      {
+        const uint64_t s01 = f2_add(acc[0], acc[1]), s23 = f2_add(acc[2], acc[3]);
+        f2_unpack(s01, lsum0, lsum1);
+        f2_unpack(s23, lsum2, lsum3);
+        lsum0 += lsum2;
+        lsum1 += lsum3;
       }
       l += lsum0 + lsum1;
       tmem_wait_st();
@@ -499,17 +550,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bar.tmem_base;
   const int total_items = item_start[geo.batch];
 
-  if (warp == 0) {
-    producer<D>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv, block_table,
-                prefix_lens, new_lens, cu_new_lens, status);
-  } else if (warp == 1) {
-    if (lane == 0)
-      mma_issuer<D>(smem_q, smem_kv, bar, tmem, item_start, total_items, geo, prefix_lens,
-                    new_lens, cu_new_lens);
-    __syncwarp();
-  } else if (warp >= 4) {
-    softmax_wg<D>((warp - 4) >> 2, bar, tmem, item_start, total_items, geo, prefix_lens, new_lens,
-                  cu_new_lens, out);
+  if (warp < 4) {
+    regs_dec<kRegsProducer>();
+    if (warp == 0) {
+      producer<D>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv,
+                  block_table, prefix_lens, new_lens, cu_new_lens, status);
+    } else if (warp == 1) {
+      if (lane == 0)
+        mma_issuer<D>(smem_q, smem_kv, bar, tmem, item_start, total_items, geo, prefix_lens,
+                      new_lens, cu_new_lens);
+      __syncwarp();
+    }
+  } else {
+    regs_inc<kRegsSoftmax>();
+    if (warp < 8)
+      softmax_wg<D, 0>(bar, tmem, item_start, total_items, geo, prefix_lens, new_lens,
+                       cu_new_lens, out);
+    else
+      softmax_wg<D, 1>(bar, tmem, item_start, total_items, geo, prefix_lens, new_lens,
+                       cu_new_lens, out);
   }
   tc_fence_before();
   __syncthreads();
