@@ -26,10 +26,12 @@
 //      warps 4-7     softmax of Q tile 0; warps 8-11 softmax of Q tile 1.
 //    Warps 0-3 give registers to the softmax warpgroups (setmaxnreg).
 //                    One thread per row: S row from TMEM, causal mask, online
-//                    softmax in the log2 domain with lazy rescaling (the
-//                    reference max moves only when a row max grows by more
-//                    than 2^8), P as bf16 written back over S in TMEM, final
-//                    1/l normalisation and the bf16 store of O.
+//                    softmax in the log2 domain against a running reference
+//                    max (the exact max of the row's first tile; recomputed,
+//                    with O and l rescaled, only if a later tile's terms
+//                    would approach fp32 overflow), P as bf16 written back
+//                    over S in TMEM, final 1/l normalisation and the bf16
+//                    store of O.
 //  * TMEM (512 columns): S0 [0,128) S1 [128,256) O0 [256,256+d) O1 [.., +d).
 //    P_i overwrites the first 64 columns of S_i.  Because P_i aliases S_i,
 //    S_i(j+1) is issued only after PV_i(j) has completed; the other Q
@@ -49,12 +51,17 @@ using namespace ptx;
 
 constexpr int kThreads = 384;
 constexpr int kRegsProducer = 88;   // warps 0-3 after setmaxnreg.dec
-constexpr int kRegsSoftmax = 200;   // warps 4-11 after setmaxnreg.inc
+constexpr int kRegsSoftmax = 208;   // warps 4-11 after setmaxnreg.inc
 static_assert(128 * kRegsProducer + 256 * kRegsSoftmax <= kThreads * 168,
               "register split exceeds the launch allocation");
 constexpr int kTileM = 128;     // rows per Q tile
 constexpr int kTileN = 128;     // keys per K/V tile
-constexpr float kRescaleLog2 = 8.0f;
+// The running row max is only recomputed when a tile's probabilities, taken
+// against the stale max, sum to 2^63 or more (a score grew by more than ~56
+// in log2 units).  Any reference value gives the same O = sum p v / sum p;
+// this bound only keeps p, l and O far from fp32 overflow.
+constexpr float kSpecLimit = 9.223372036854775808e18f;  // 2^63
+
 
 template <int D>
 struct Cfg {
@@ -343,6 +350,70 @@ __device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uin
   mbar_wait(&bar.drain, 0, &no_abort);
 }
 
+// Row max of a 128-column score tile (raw scores, masked columns -inf).
+__device__ __forceinline__ float tile_max(const uint32_t (&sr)[4][32]) {
+  float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+  for (int c = 0; c < 4; ++c)
+#pragma unroll
+    for (int e = 0; e < 32; e += 8) {
+      mx[0] = fmax3(mx[0], __uint_as_float(sr[c][e + 0]), __uint_as_float(sr[c][e + 1]));
+      mx[1] = fmax3(mx[1], __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
+      mx[2] = fmax3(mx[2], __uint_as_float(sr[c][e + 4]), __uint_as_float(sr[c][e + 5]));
+      mx[3] = fmax3(mx[3], __uint_as_float(sr[c][e + 6]), __uint_as_float(sr[c][e + 7]));
+    }
+  return fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
+}
+
+// p = 2^(s * scale*log2(e) - m) for one row of the tile, written to TMEM at
+// tS as bf16 pairs (the A operand of the PV product); returns sum p (fp32).
+__device__ __forceinline__ float tile_exp(const uint32_t (&sr)[4][32], uint32_t tS,
+                                          float scale_log2, float m) {
+  const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
+  const uint64_t nm2 = f2_pack(-m, -m);
+  uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    uint32_t pk[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      const uint64_t t = f2_fma(f2_pack(__uint_as_float(sr[c][2 * e]),
+                                        __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
+      float t0, t1;
+      f2_unpack(t, t0, t1);
+      const float p0 = ex2_approx(t0), p1 = ex2_approx(t1);
+      acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
+      pk[e] = pack_bf16x2(p0, p1);
+    }
+    tmem_st16(tS + c * 16, pk);
+  }
+  float s0, s1, s2, s3;
+  f2_unpack(f2_add(acc[0], acc[1]), s0, s1);
+  f2_unpack(f2_add(acc[2], acc[3]), s2, s3);
+  return (s0 + s2) + (s1 + s3);
+}
+
+// O row *= alpha in TMEM (D fp32 columns at tO).
+template <int D>
+__device__ __forceinline__ void rescale_o(uint32_t tO, float alpha) {
+#pragma unroll 1
+  for (int c = 0; c < D / 32; ++c) {
+    uint32_t o[32];
+    tmem_ld32(tO + c * 32, o);
+    tmem_wait_ld();
+#pragma unroll
+    for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+    tmem_st32(tO + c * 32, o);
+  }
+}
+
+// Make this thread's P writes visible to the MMA issuer and arrive.
+__device__ __forceinline__ void publish_p(uint64_t* bar) {
+  tmem_wait_st();
+  tc_fence_before();
+  mbar_arrive(bar);
+}
+
 template <int D, int i>
 __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
                            int total_items, const Geom& geo,
@@ -385,67 +456,28 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
           for (int e = 0; e < 32; ++e)
             if (key0 + c * 32 + e > kmax) sr[c][e] = __float_as_uint(-INFINITY);
       }
-      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-      for (int c = 0; c < 4; ++c)
-#pragma unroll
-        for (int e = 0; e < 32; e += 8) {
-          mx[0] = fmax3(mx[0], __uint_as_float(sr[c][e + 0]), __uint_as_float(sr[c][e + 1]));
-          mx[1] = fmax3(mx[1], __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
-          mx[2] = fmax3(mx[2], __uint_as_float(sr[c][e + 4]), __uint_as_float(sr[c][e + 5]));
-          mx[3] = fmax3(mx[3], __uint_as_float(sr[c][e + 6]), __uint_as_float(sr[c][e + 7]));
+      const float sl2 = geo.scale_log2;
+      float lt;
+      if (m_run == -INFINITY) {
+        // first tile of the row: exact max (key 0 is always visible)
+        m_run = tile_max(sr) * sl2;
+        lt = tile_exp(sr, tS, sl2, m_run);
+      } else {
+        // later tiles keep the running max unless the tile would overflow
+        lt = tile_exp(sr, tS, sl2, m_run);
+        if (__any_sync(0xffffffffu, !(lt < kSpecLimit))) {
+          // O is complete up to tile j-1: S_i(j) was issued after PV_i(j-1)
+          tmem_wait_st();
+          const float m_new = fmaxf(m_run, tile_max(sr) * sl2);
+          const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
+          rescale_o<D>(tO, alpha);
+          l *= alpha;
+          m_run = m_new;
+          lt = tile_exp(sr, tS, sl2, m_run);
         }
-      const float mt = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
-      const float mt2 = mt * geo.scale_log2;
-      if (__any_sync(0xffffffffu, mt2 > m_run + kRescaleLog2)) {
-        const float m_new = fmaxf(m_run, mt2);
-        const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;  // 0 if m_run = -inf
-        if (j > 0) {
-          // O_i is complete up to tile j-1: S_i(j) was issued after PV_i(j-1)
-#pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32(tO + c * 32, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-            tmem_st32(tO + c * 32, o);
-          }
-        }
-        l *= alpha;
-        m_run = m_new;
       }
-      // p = 2^(s * scale*log2(e) - m), two columns per paired FMA
-      const uint64_t sc2 = f2_pack(geo.scale_log2, geo.scale_log2);
-      const uint64_t nm2 = f2_pack(-m_run, -m_run);
-      uint64_t acc[4] = {0, 0, 0, 0};
-#pragma unroll
-      for (int c = 0; c < 4; ++c) {
-        uint32_t pk[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const uint64_t t = f2_fma(f2_pack(__uint_as_float(sr[c][2 * e]),
-                                            __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
-          float t0, t1;
-          f2_unpack(t, t0, t1);
-          const float p0 = ex2_approx(t0), p1 = ex2_approx(t1);
-          acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
-          pk[e] = pack_bf16x2(p0, p1);
-        }
-        tmem_st16(tS + c * 16, pk);
-      }
-      float lsum0, lsum1, lsum2, lsum3;
-      {
-        const uint64_t s01 = f2_add(acc[0], acc[1]), s23 = f2_add(acc[2], acc[3]);
-        f2_unpack(s01, lsum0, lsum1);
-        f2_unpack(s23, lsum2, lsum3);
-        lsum0 += lsum2;
-        lsum1 += lsum3;
-      }
-      l += lsum0 + lsum1;
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(&bar.p_full[i]);
+      l += lt;
+      publish_p(&bar.p_full[i]);
     }
     if (!ok) break;
     // ---- epilogue: O / l -> bf16

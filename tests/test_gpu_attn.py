@@ -209,3 +209,17 @@ def test_bad_block_table_entry_is_reported_not_faulted():
     db.attn()
     assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
     db.close()
+
+
+def test_large_score_jumps_take_the_exact_path():
+    """Keys whose scores jump far above the running row max (by more than
+    the overflow guard, in the second half of one tile and the first half of
+    a later one) must still give the softmax definition."""
+    w = wl.custom("jumps", 1, 8, 1, 128, 16, [512], [64], seed=12)
+    src = wl.bf16_bits_to_f32(w.host_src())          # [32 blocks][1][2][1][16][128]
+    keys = src[:, 0, 0, 0].reshape(-1, 128)            # prefix keys in order
+    keys[192:256] *= 256.0                             # tile 1, second half
+    keys[256:320] *= 1024.0                            # tile 2, first half
+    src[:, 0, 0, 0] = keys.reshape(-1, 16, 128)
+    w._cache["src"] = wl.f32_to_bf16_bits(src)
+    full_parity(w)
