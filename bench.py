@@ -207,7 +207,7 @@ def run_reference(args):
     w = make_workload(args.config, args.seed)
     rng = np.random.default_rng(args.seed)
     pool = None
-    per_step = max(1.0, min(6.0, 150.0 / max(args.steps + args.warmup, 1)))
+    per_step = args.ref_step_seconds or max(1.0, min(6.0, 150.0 / max(args.steps + args.warmup, 1)))
     for _ in range(args.warmup):
         s = oracle_sample(w, per_step / 2, rng, pool)
         pool = s["pool"]
@@ -472,6 +472,9 @@ def main():
     ap.add_argument("--no-restore80", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--ref-step-seconds", type=float, default=None,
+                    help="oracle seconds per step of --impl reference (default: sized so "
+                         "the whole run takes about 2.5 minutes)")
     ap.add_argument("--profile", action="store_true",
                     help="timed loop only (for ncu launch lists): no e2e, clocks or baselines")
     args = ap.parse_args()
