@@ -34,6 +34,8 @@
  *  - Zero sizes (n_blocks = 0, batch = 0, a request with no new tokens) are
  *    valid no-ops.
  *  - A pool handle is not thread-safe; distinct pools are independent.
+ *    Attention calls on one pool must not run concurrently on the GPU: they
+ *    share the work counter in the pool's control block.
  *  - bf16 is the only element type.  All tensors are dense and row-major.
  *
  * Layouts (element = bf16 unless stated)
@@ -89,7 +91,8 @@ typedef struct gc_pool_config {
 } gc_pool_config;
 
 /* Device bytes a pool of this shape needs: the KV planes
- * (L*2*num_pages*Hkv*ps*d*2 bytes) plus a 256-byte status trailer.
+ * (L*2*num_pages*Hkv*ps*d*2 bytes) plus a 256-byte control block (device
+ * status word, attention work counter).
  * Returns 0 for an invalid configuration. */
 GC_API size_t gc_kv_pool_bytes(const gc_pool_config* cfg);
 
@@ -109,7 +112,7 @@ GC_API gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, siz
  * caller must make sure no stream still uses the pool. */
 GC_API gc_status gc_kv_pool_destroy(gc_kv_pool* pool);
 
-/* Device address and byte size of the KV planes (status trailer excluded). */
+/* Device address and byte size of the KV planes (control block excluded). */
 GC_API gc_status gc_kv_pool_data(const gc_kv_pool* pool, void** dev_ptr, size_t* bytes);
 
 /* Synchronise `stream`, then read and clear the pool's device status word:

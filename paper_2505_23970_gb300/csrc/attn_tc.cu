@@ -7,7 +7,9 @@
 // with keys read from the paged pool through block_table[b].
 //
 // Design
-//  * Work item = (request b, kv head g, pair of 128-row Q tiles).  A Q tile
+//  * Work item = (request b, kv head g, pair of 128-row Q tiles), handed out
+//    dynamically (an atomic counter in the pool's control block; items of a
+//    request are numbered later rows first, so long items start early).  A Q tile
 //    packs 128/G new tokens x the G q heads of one kv group (row = token*G +
 //    head), so every K/V tile fetched from the pool feeds all G heads, and
 //    the two Q tiles of a CTA share each K/V tile as well.
@@ -83,9 +85,15 @@ struct Barriers {
   uint64_t q_full, q_empty, vfix, drain;
   uint64_t kv_full[8], kv_empty[8];
   uint64_t s_full[2], p_full[2], pv_done[2];
+  uint64_t item_full[2], item_empty[2];  // work-item ring, producer -> other roles
+  int item_slot[2];
   uint32_t tmem_base;
   int abort_flag;
 };
+
+// Consumers of the work-item ring: the MMA issuer thread and one elected
+// thread per softmax warp.
+constexpr int kItemConsumers = 1 + 2 * kTileM / 32;
 
 // A work item and the quantities every role derives from it.
 struct Item {
@@ -127,6 +135,31 @@ __device__ __forceinline__ bool decode_item(int it, const int* item_start, const
   return true;
 }
 
+// Work items are handed out dynamically: the producer warp claims the next
+// one from the launch's counter and publishes it to the other roles through a
+// 2-slot ring in shared memory; -1 ends the CTA's work.
+__device__ __forceinline__ int claim_item(Barriers& bar, uint32_t k, int* work_counter,
+                                          int total_items, volatile int* abortp, bool& ok) {
+  const int s = k & 1;
+  ok = mbar_wait(&bar.item_empty[s], ((k >> 1) & 1) ^ 1, abortp);
+  int it = -1;
+  if ((threadIdx.x & 31) == 0 && ok) {
+    it = atomicAdd(work_counter, 1);
+    if (it >= total_items) it = -1;
+    bar.item_slot[s] = it;
+    mbar_arrive(&bar.item_full[s]);
+  }
+  return __shfl_sync(0xffffffffu, it, 0);
+}
+
+// Read item k of the ring (all consumer threads); the caller releases the
+// slot with one arrival per consumer (see kItemConsumers).
+__device__ __forceinline__ int read_item(Barriers& bar, uint32_t k, volatile int* abortp,
+                                         bool& ok) {
+  ok = mbar_wait(&bar.item_full[k & 1], (k >> 1) & 1, abortp);
+  return ok ? *reinterpret_cast<volatile int*>(&bar.item_slot[k & 1]) : -1;
+}
+
 // ------------------------------------------------------------------ roles
 template <int D>
 __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const int* item_start,
@@ -134,7 +167,8 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
                          const CUtensorMap* map_kv, const int32_t* __restrict__ block_table,
                          const int32_t* __restrict__ prefix_lens,
                          const int32_t* __restrict__ new_lens,
-                         const int32_t* __restrict__ cu_new_lens, int32_t* status) {
+                         const int32_t* __restrict__ cu_new_lens, int32_t* status,
+                         int* work_counter) {
   using C = Cfg<D>;
   const int lane = threadIdx.x & 31;
   volatile int* abortp = &bar.abort_flag;
@@ -144,7 +178,9 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
   bool ok = true;
   const uint32_t box_bytes = static_cast<uint32_t>(geo.ps) * 128;  // one page, one column block
 
-  for (int it = blockIdx.x; ok && it < total_items; it += gridDim.x) {
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = claim_item(bar, k, work_counter, total_items, abortp, ok);
+    if (!ok || it < 0) break;
     Item w;
     decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
     // ---- Q tiles
@@ -255,7 +291,11 @@ __device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uin
   bool ok = true;
   const uint32_t q_base = smem_addr(smem_q), kv_smem = smem_addr(smem_kv);
 
-  for (int it = blockIdx.x; ok && it < total_items; it += gridDim.x) {
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = read_item(bar, k, abortp, ok);
+    if (!ok) break;
+    mbar_arrive(&bar.item_empty[k & 1]);
+    if (it < 0) break;
     Item w;
     decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
     ok = mbar_wait(&bar.q_full, q_count & 1, abortp);
@@ -431,7 +471,12 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
   uint32_t s_count = 0, pv_total = 0;
   bool ok = true;
 
-  for (int it = blockIdx.x; ok && it < total_items; it += gridDim.x) {
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = read_item(bar, k, abortp, ok);
+    if (!ok) break;
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) mbar_arrive(&bar.item_empty[k & 1]);
+    if (it < 0) break;
     Item w;
     decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
     if (!w.valid[i]) continue;
@@ -516,7 +561,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                    const __grid_constant__ CUtensorMap map_kv,
                    const int32_t* __restrict__ block_table, const int32_t* __restrict__ prefix_lens,
                    const int32_t* __restrict__ new_lens, const int32_t* __restrict__ cu_new_lens,
-                   __nv_bfloat16* __restrict__ out, Geom geo, int32_t* status) {
+                   __nv_bfloat16* __restrict__ out, Geom geo, int32_t* status,
+                   int* work_counter) {
   using C = Cfg<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>(
@@ -540,6 +586,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.s_full[i], 1);
       mbar_init(&bar.p_full[i], kTileM);
       mbar_init(&bar.pv_done[i], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&bar.item_full[s], 1);
+      mbar_init(&bar.item_empty[s], kItemConsumers);
     }
     bar.abort_flag = 0;
     fence_barrier_init();
@@ -586,7 +636,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     regs_dec<kRegsProducer>();
     if (warp == 0) {
       producer<D>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv,
-                  block_table, prefix_lens, new_lens, cu_new_lens, status);
+                  block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
     } else if (warp == 1) {
       if (lane == 0)
         mma_issuer<D>(smem_q, smem_kv, bar, tmem, item_start, total_items, geo, prefix_lens,
@@ -681,9 +731,12 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream)
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: smem attribute");
+  // the work items are claimed from a counter in the pool's control block
+  e = cudaMemsetAsync(pool->work_counter, 0, sizeof(int), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: clearing the work counter");
   attn_tc_kernel<D><<<pool->num_sms, kThreads, smem, stream>>>(
       map_q, map_kv, a.block_table, a.prefix_lens, a.new_lens, a.cu_new_lens,
-      static_cast<__nv_bfloat16*>(a.out), geo, pool->status);
+      static_cast<__nv_bfloat16*>(a.out), geo, pool->status, pool->work_counter);
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: launch");
   return GC_OK;

@@ -14,6 +14,7 @@ struct gc_kv_pool {
   uint8_t* data;          // KV planes [L][2][num_pages][Hkv][ps][d] bf16
   size_t data_bytes;
   int32_t* status;        // device status word (first error recorded by a kernel)
+  int32_t* work_counter;  // attention work-item counter (control block, zeroed per launch)
   void* owned;            // cudaMalloc'd block, or nullptr if caller-owned
   int device;
   int num_sms;
