@@ -52,6 +52,9 @@ namespace {
 using namespace ptx;
 
 constexpr int kThreads = 384;
+// Batches up to this size are numbered longest request first (ranked in
+// shared memory by every CTA); larger batches keep the given order.
+constexpr int kSortMax = 512;
 constexpr int kRegsProducer = 88;   // warps 0-3 after setmaxnreg.dec
 constexpr int kRegsSoftmax = 208;   // warps 4-11 after setmaxnreg.inc
 static_assert(128 * kRegsProducer + 256 * kRegsSoftmax <= kThreads * 168,
@@ -102,6 +105,8 @@ struct Item {
   bool valid[2];
 };
 
+// item_start[p] = first item of the p-th request in work order; the request
+// itself is order[p] when the batch was sorted (order != nullptr), else p.
 __device__ __forceinline__ bool decode_item(int it, const int* item_start, const Geom& geo,
                                             const int32_t* __restrict__ prefix_lens,
                                             const int32_t* __restrict__ new_lens,
@@ -111,14 +116,17 @@ __device__ __forceinline__ bool decode_item(int it, const int* item_start, const
     const int mid = (lo + hi) >> 1;
     if (item_start[mid] <= it) lo = mid; else hi = mid;
   }
-  w.b = lo;
+  const int b = geo.batch <= kSortMax ? static_cast<int>(
+                    reinterpret_cast<const int16_t*>(item_start + geo.batch + 1)[lo])
+                                       : lo;
+  w.b = b;
   const int local = it - item_start[lo];
   const int pairs = (item_start[lo + 1] - item_start[lo]) / geo.Hkv;
   const int pair = pairs - 1 - local / geo.Hkv;  // later rows (more keys) first
   w.g = local % geo.Hkv;
-  w.P = __ldg(prefix_lens + lo);
-  w.n = __ldg(new_lens + lo);
-  w.cu = __ldg(cu_new_lens + lo);
+  w.P = __ldg(prefix_lens + b);
+  w.n = __ldg(new_lens + b);
+  w.cu = __ldg(cu_new_lens + b);
   w.T = w.P + w.n;
   const int rows = w.n * geo.G;
   w.nt = 0;
@@ -571,6 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem_kv = base + 2 * C::kTileBytes;
   Barriers& bar = *reinterpret_cast<Barriers*>(smem_kv + C::kStages * C::kTileBytes);
   int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
+  int16_t* order = reinterpret_cast<int16_t*>(item_start + geo.batch + 1);  // [min(batch, kSortMax)]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
@@ -602,13 +611,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(&bar.tmem_base, 512);
     tmem_relinquish();
   }
+  if (geo.batch <= kSortMax) {
+    // rank requests by total length, longest first (ties by index)
+    for (int b = threadIdx.x; b < geo.batch; b += kThreads) {
+      const int tb = __ldg(prefix_lens + b) + __ldg(new_lens + b);
+      int rank = 0;
+      for (int o = 0; o < geo.batch; ++o) {
+        const int to = __ldg(prefix_lens + o) + __ldg(new_lens + o);
+        rank += (to > tb) || (to == tb && o < b);
+      }
+      order[rank] = static_cast<int16_t>(b);
+    }
+  }
+  __syncthreads();
   if (warp == 2) {
-    // work items per request: Hkv * ceil(n_b * G / 256); exclusive scan
+    // work items per request: Hkv * ceil(n_b * G / 256); exclusive scan in work order
     int running = 0;
     for (int b0 = 0; b0 < geo.batch; b0 += 32) {
-      const int b = b0 + lane;
+      const int p = b0 + lane;
+      const int b = p < geo.batch ? (geo.batch <= kSortMax ? order[p] : p) : p;
       int cnt = 0;
-      if (b < geo.batch) {
+      if (p < geo.batch) {
         const int n = __ldg(new_lens + b), P = __ldg(prefix_lens + b);
         const int cu = __ldg(cu_new_lens + b);
         const bool sane = n >= 0 && P >= 0 && cu >= 0 && cu + n <= geo.total_new;
@@ -621,7 +644,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int y = __shfl_up_sync(0xffffffffu, incl, o);
         if (lane >= o) incl += y;
       }
-      if (b < geo.batch) item_start[b] = running + incl - cnt;
+      if (p < geo.batch) item_start[p] = running + incl - cnt;
       running += __shfl_sync(0xffffffffu, incl, 31);
     }
     if (lane == 0) item_start[geo.batch] = running;
@@ -726,7 +749,8 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream)
       return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: pool tensor map (CUresult %d)", (int)r);
   }
   const size_t smem = 1024 + 2 * C::kTileBytes + C::kStages * C::kTileBytes + sizeof(Barriers) +
-                      (static_cast<size_t>(a.batch) + 1) * sizeof(int);
+                      (static_cast<size_t>(a.batch) + 1) * sizeof(int) +
+                      kSortMax * sizeof(int16_t);
   cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
