@@ -199,6 +199,35 @@ GC_API gc_status gc_prefix_prefill_attn(const void* q, const gc_kv_pool* pool, c
                                  int32_t batch, int32_t max_blocks_per_seq, int32_t num_q_heads,
                                  float softmax_scale, int32_t total_new_tokens);
 
+/* Same operation, arguments and result as gc_prefix_prefill_attn, for
+ * callers that cannot allocate device memory.  The paper has no counterpart:
+ * this entry point serves code that runs inside a device-memory budget it
+ * does not control, for example a plugin living in a framework whose caching
+ * allocator has reserved the GPU's memory, or a runtime that forbids
+ * allocation while it serves.  Such a caller creates its pool in memory it
+ * already owns (gc_kv_pool_create with dev_mem) and calls this function.
+ *   It allocates nothing: the only scratch the kernel needs (its work-item
+ *   counter) is a 256-byte array inside libgc's device image, which every GPU
+ *   that loads the library holds until the process exits.  The first call on
+ *   a device looks up the array's device address (cudaGetSymbolAddress) with
+ *   that device current; make that first call before any stream capture.
+ *   Each call clears the counter with a stream-ordered memset.
+ *   All calls share the array, on every pool: two calls that overlap on the
+ *   GPU race on it and give wrong results.  Serialise them.
+ *   Limit: at most 2^31 - 1 work items per call, i.e.
+ *   Hkv * (total_new_tokens * (Hq/Hkv) / 256 + batch) <= 2^31 - 1; larger
+ *   calls fail with GC_ERR_UNSUPPORTED before anything is launched.
+ *   The current device must be the pool's device (GC_ERR_INVALID_ARG).
+ * Other errors as gc_prefix_prefill_attn. */
+GC_API gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool* pool,
+                                                const int32_t* block_table,
+                                                const int32_t* prefix_lens,
+                                                const int32_t* new_lens, void* out,
+                                                cudaStream_t stream, int32_t layer,
+                                                const int32_t* cu_new_lens, int32_t batch,
+                                                int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                                float softmax_scale, int32_t total_new_tokens);
+
 /* Same operation and arguments as gc_prefix_prefill_attn, computed by a
  * plain CUDA-core kernel (one warp per row, fp32 throughout, no tensor
  * cores).  Slow; kept as an independent GPU cross-check of the indexing. */

@@ -32,7 +32,8 @@ GC_RESTORE_VECTOR = 2
 EXPORTED = (
     "gc_kv_pool_bytes", "gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
     "gc_kv_pool_check", "gc_kv_restore", "gc_kv_append", "gc_prefix_prefill_attn",
-    "gc_prefix_prefill_attn_simt", "gc_last_error", "gc_status_string",
+    "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc", "gc_last_error",
+    "gc_status_string",
 )
 
 
@@ -75,9 +76,11 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         attn = [vp, vp, vp, vp, vp, vp, vp, i32, vp, i32, i32, i32, ctypes.c_float, i32]
         lib.gc_prefix_prefill_attn.argtypes = attn
         lib.gc_prefix_prefill_attn_simt.argtypes = attn
+        lib.gc_prefix_prefill_attn_noalloc.argtypes = attn
         for f in ("gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
                   "gc_kv_pool_check", "gc_kv_restore", "gc_kv_append",
-                  "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt"):
+                  "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt",
+                  "gc_prefix_prefill_attn_noalloc"):
             getattr(lib, f).restype = ctypes.c_int
         lib.gc_last_error.argtypes = []
         lib.gc_last_error.restype = ctypes.c_char_p
@@ -189,6 +192,20 @@ def gc_prefix_prefill_attn_simt(q, pool, block_table, prefix_lens, new_lens, out
                                               _stream(stream), layer, _addr(cu_new_lens), batch,
                                               max_blocks_per_seq, num_q_heads, softmax_scale,
                                               total_new_tokens), "gc_prefix_prefill_attn_simt")
+
+
+def gc_prefix_prefill_attn_noalloc(q, pool, block_table, prefix_lens, new_lens, out, stream,
+                                   layer: int, cu_new_lens, batch: int, max_blocks_per_seq: int,
+                                   num_q_heads: int, softmax_scale: float,
+                                   total_new_tokens: int) -> None:
+    """gc_prefix_prefill_attn for callers that cannot allocate device memory:
+    its only scratch is a static array inside libgc (see include/gc.h)."""
+    _check(load().gc_prefix_prefill_attn_noalloc(_addr(q), pool, _addr(block_table),
+                                                 _addr(prefix_lens), _addr(new_lens), _addr(out),
+                                                 _stream(stream), layer, _addr(cu_new_lens),
+                                                 batch, max_blocks_per_seq, num_q_heads,
+                                                 softmax_scale, total_new_tokens),
+           "gc_prefix_prefill_attn_noalloc")
 
 
 @dataclass

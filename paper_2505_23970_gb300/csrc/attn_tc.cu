@@ -42,6 +42,7 @@
 //    all roles leave their loops, in-flight copies and MMAs are drained, TMEM
 //    is freed and GC_ERR_TIMEOUT is recorded in the pool status word.
 #include <cmath>
+#include <mutex>
 
 #include "gc_internal.cuh"
 #include "sm103_ptx.cuh"
@@ -698,7 +699,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 }
 
 template <int D>
-gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
+gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
+                 int* work_counter) {
   using C = Cfg<D>;
   auto enc = encode_fn();
   if (!enc) return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: cuTensorMapEncodeTiled unavailable");
@@ -756,11 +758,11 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream)
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: smem attribute");
   // the work items are claimed from a counter in the pool's control block
-  e = cudaMemsetAsync(pool->work_counter, 0, sizeof(int), stream);
+  e = cudaMemsetAsync(work_counter, 0, sizeof(int), stream);
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: clearing the work counter");
   attn_tc_kernel<D><<<pool->num_sms, kThreads, smem, stream>>>(
       map_q, map_kv, a.block_table, a.prefix_lens, a.new_lens, a.cu_new_lens,
-      static_cast<__nv_bfloat16*>(a.out), geo, pool->status, pool->work_counter);
+      static_cast<__nv_bfloat16*>(a.out), geo, pool->status, work_counter);
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: launch");
   return GC_OK;
@@ -769,8 +771,71 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream)
 }  // namespace
 
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
-  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream);
-  return launch<64>(pool, a, stream);
+  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter);
+  return launch<64>(pool, a, stream, pool->work_counter);
+}
+
+}  // namespace gc
+
+// ------------------------------------------------------- allocation-free variant
+// Scratch of gc_prefix_prefill_attn_noalloc: element 0 is the work-item
+// counter the kernel's CTAs claim items from.  It lives in the library's own
+// device memory, so that entry point needs no buffer from anyone; every GPU
+// that loads the library keeps these 256 bytes until the process exits, and
+// all calls share them.
+static __device__ __align__(256) int32_t g_attn_noalloc_scratch[64];
+
+namespace gc {
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+// Device address of the static scratch on `device`, looked up once per device
+// with that device current (host code cannot use the symbol itself: it only
+// names a host-side stand-in).
+gc_status noalloc_scratch(int device, int** out) {
+  static std::mutex mu;
+  static int* addr[kMaxDevices] = {};
+  if (device < 0 || device >= kMaxDevices)
+    return fail(GC_ERR_UNSUPPORTED, "gc_prefix_prefill_attn_noalloc: device %d >= %d", device,
+                kMaxDevices);
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_attn_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn_noalloc: cudaGetSymbolAddress");
+    addr[device] = static_cast<int*>(p);
+  }
+  *out = addr[device];
+  return GC_OK;
+}
+
+}  // namespace
+
+gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a,
+                                 cudaStream_t stream) {
+  // the items of a call must fit the 32-bit counter: Hkv * sum ceil(n_b*G/256)
+  const long long G = a.num_q_heads / pool->cfg.num_kv_heads;
+  const long long items_max =
+      static_cast<long long>(pool->cfg.num_kv_heads) *
+      (static_cast<long long>(a.total_new_tokens) * G / (2 * kTileM) + a.batch);
+  if (items_max > 2147483647LL)
+    return fail(GC_ERR_UNSUPPORTED,
+                "gc_prefix_prefill_attn_noalloc: up to %lld work items exceed the 2^31-1 the "
+                "static work counter can hand out",
+                items_max);
+  int device = -1;
+  cudaError_t e = cudaGetDevice(&device);
+  if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn_noalloc: cudaGetDevice");
+  if (device != pool->device)
+    return fail(GC_ERR_INVALID_ARG,
+                "gc_prefix_prefill_attn_noalloc: current device %d is not the pool's device %d",
+                device, pool->device);
+  int* counter = nullptr;
+  const gc_status st = noalloc_scratch(device, &counter);
+  if (st != GC_OK) return st;
+  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, counter);
+  return launch<64>(pool, a, stream, counter);
 }
 
 }  // namespace gc

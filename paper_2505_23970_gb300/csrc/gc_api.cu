@@ -278,6 +278,22 @@ gc_status gc_prefix_prefill_attn(const void* q, const gc_kv_pool* pool, const in
   return gc::launch_attn_tc(pool, a, stream);
 }
 
+gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool* pool,
+                                         const int32_t* block_table, const int32_t* prefix_lens,
+                                         const int32_t* new_lens, void* out, cudaStream_t stream,
+                                         int32_t layer, const int32_t* cu_new_lens, int32_t batch,
+                                         int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                         float softmax_scale, int32_t total_new_tokens) {
+  g_msg[0] = 0;
+  gc::AttnArgs a;
+  bool noop;
+  gc_status s = attn_common("gc_prefix_prefill_attn_noalloc", q, pool, block_table, prefix_lens,
+                            new_lens, out, layer, cu_new_lens, batch, max_blocks_per_seq,
+                            num_q_heads, softmax_scale, total_new_tokens, &a, &noop);
+  if (s != GC_OK || noop) return s;
+  return gc::launch_attn_tc_noalloc(pool, a, stream);
+}
+
 gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* pool,
                                       const int32_t* block_table, const int32_t* prefix_lens,
                                       const int32_t* new_lens, void* out, cudaStream_t stream,
