@@ -406,7 +406,9 @@ def bench_restore80(args, pk):
     """Restore of the 80-layer KV of one 8192-token prefix (2.68 GB): the
     scatter from a device staging buffer (read + write bytes vs HBM) and the
     whole pinned host -> pool path (payload bytes), next to a plain pinned
-    host -> device cudaMemcpyAsync of the same bytes."""
+    host -> device cudaMemcpyAsync of the same bytes; then the inverse save
+    (pool -> device staging gather, pool -> pinned host) beside a plain
+    device -> host copy."""
     import torch
 
     from paper_2505_23970_gb300 import binding as gcb
@@ -443,6 +445,16 @@ def bench_restore80(args, pk):
     zc_ms = timed(lambda: gcb.gc_kv_restore(db.pool.handle, db.host_src, db.block_ids,
                                             db.n_blocks, stream, None, 0))
     h2d_ms = timed(lambda: db.staging.copy_(db.host_src, non_blocking=True))
+    # the inverse path: save the same pages back to the cache tier
+    host_dst = torch.empty_like(db.host_src).pin_memory()
+    save_dev_ms = timed(lambda: gcb.gc_kv_save(db.pool.handle, db.staging, db.block_ids,
+                                               db.n_blocks, stream, None,
+                                               gcb.GC_SAVE_DST_DEVICE))
+    save_staged_ms = timed(lambda: gcb.gc_kv_save(db.pool.handle, host_dst, db.block_ids,
+                                                  db.n_blocks, stream, db.staging, 0))
+    save_zc_ms = timed(lambda: gcb.gc_kv_save(db.pool.handle, host_dst, db.block_ids,
+                                              db.n_blocks, stream, None, 0))
+    d2h_ms = timed(lambda: host_dst.copy_(db.staging, non_blocking=True))
     ok = db.check(stream) == gcb.GC_OK
     db.close()
     gbs = lambda nbytes, ms: nbytes / (ms / 1e3) / 1e9  # noqa: E731
@@ -454,8 +466,15 @@ def bench_restore80(args, pk):
         "host_to_pool_staged_gbs": gbs(payload, staged_ms),
         "host_to_pool_zero_copy_gbs": gbs(payload, zc_ms),
         "pinned_h2d_memcpy_gbs": gbs(payload, h2d_ms),
+        "save_gather_gbs": gbs(2 * payload, save_dev_ms),
+        "save_gather_frac_hbm": gbs(2 * payload, save_dev_ms) / pk["hbm_gbs"],
+        "pool_to_host_staged_gbs": gbs(payload, save_staged_ms),
+        "pool_to_host_zero_copy_gbs": gbs(payload, save_zc_ms),
+        "pinned_d2h_memcpy_gbs": gbs(payload, d2h_ms),
         "ms": {"scatter_bulk": scatter_ms, "scatter_vector": vec_ms, "staged": staged_ms,
-               "zero_copy": zc_ms, "h2d_memcpy": h2d_ms},
+               "zero_copy": zc_ms, "h2d_memcpy": h2d_ms, "save_gather": save_dev_ms,
+               "save_staged": save_staged_ms, "save_zero_copy": save_zc_ms,
+               "d2h_memcpy": d2h_ms},
     }
 
 

@@ -12,6 +12,8 @@
  *
  *   gc_kv_restore           cached pages (pinned host or device staging)
  *                           -> paged HBM KV pool                  (load)
+ *   gc_kv_save              paged HBM KV pool -> pinned host / device
+ *                           staging image; the inverse of restore  (save)
  *   gc_kv_append            new tokens' K,V -> pool slots after each
  *                           request's cached prefix                (stitch)
  *   gc_prefix_prefill_attn  causal GQA attention of the new tokens over
@@ -147,6 +149,34 @@ GC_API gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t
  * zero-copy path), GC_ERR_CUDA. */
 GC_API gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
                         int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags);
+
+/* gc_kv_save flags */
+#define GC_SAVE_DST_DEVICE 1u /* host_dst is device memory (gather only) */
+#define GC_SAVE_VECTOR 2u     /* 16-byte vector-copy kernel instead of bulk copies */
+
+/* Save pool pages to the cache tier (Sec. 2.2, Fig. 2a step 1: once a
+ * request has been processed its KV is saved to storage); the inverse of
+ * gc_kv_restore.  For i < n_blocks and every layer l and plane kv:
+ *     host_dst[i][l][kv] <- pool[l][kv][block_ids[i]]
+ * a byte-exact copy of Hkv*ps*d*2 bytes per (i, l, kv).
+ *   host_dst   [n_blocks][L][2][Hkv][ps][d] bf16.  Pinned host memory, or
+ *              device memory when flags has GC_SAVE_DST_DEVICE.  The caller
+ *              reads it after the stream has passed the call.
+ *   block_ids  int32 [n_blocks], DEVICE memory.  Ids outside [0, num_pages)
+ *              are skipped and recorded as GC_ERR_OUT_OF_RANGE in the status
+ *              word: their chunk of the written image (host_dst, or
+ *              dev_staging on the staged path, which is then copied to
+ *              host_dst whole) is not written.
+ *   dev_staging  NULL: the kernel writes host_dst directly over the
+ *              host-device link (zero copy).  Otherwise device memory of at
+ *              least n_blocks*L*2*Hkv*ps*d*2 bytes: the pages are gathered
+ *              there, then copied to host_dst with one cudaMemcpyAsync.
+ *              Ignored with GC_SAVE_DST_DEVICE.
+ * Errors: GC_ERR_INVALID_ARG (null/negative, unaligned, or host_dst not
+ * pinned), GC_ERR_CUDA. */
+GC_API gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
+                            int32_t n_blocks, cudaStream_t stream, void* dev_staging,
+                            uint32_t flags);
 
 /* Append the new tokens' K and V after each request's cached prefix
  * (Sec. 2.2: the KV of the cached tokens and of the new tokens is stitched

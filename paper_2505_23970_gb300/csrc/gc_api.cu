@@ -198,8 +198,57 @@ gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* b
   }
   if (reinterpret_cast<uintptr_t>(src) % 16)
     return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: source not 16-byte aligned");
-  return vector ? gc::launch_restore_vector(pool, src, block_ids, n_blocks, stream)
-                : gc::launch_restore_bulk(pool, src, block_ids, n_blocks, stream);
+  uint8_t* stg = const_cast<uint8_t*>(src);  // read only when restoring
+  return vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, false, stream)
+                : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, false, stream);
+}
+
+gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
+                     int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  g_msg[0] = 0;
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_kv_save: pool is NULL");
+  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "gc_kv_save: n_blocks < 0");
+  if (flags & ~(GC_SAVE_DST_DEVICE | GC_SAVE_VECTOR))
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_save: unknown flags 0x%x", flags);
+  if (n_blocks == 0) return GC_OK;
+  if (!host_dst || !block_ids)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_save: host_dst / block_ids is NULL");
+  const size_t bytes = static_cast<size_t>(n_blocks) * pool->cfg.num_layers * 2 *
+                       gc::page_bytes(pool->cfg);
+  bool vector = (flags & GC_SAVE_VECTOR) != 0;
+  if (flags & GC_SAVE_DST_DEVICE) {
+    if (reinterpret_cast<uintptr_t>(host_dst) % 16)
+      return fail(GC_ERR_INVALID_ARG, "gc_kv_save: destination not 16-byte aligned");
+    uint8_t* dst = static_cast<uint8_t*>(host_dst);
+    return vector ? gc::launch_restore_vector(pool, dst, block_ids, n_blocks, true, stream)
+                  : gc::launch_restore_bulk(pool, dst, block_ids, n_blocks, true, stream);
+  }
+  cudaPointerAttributes attr;
+  cudaError_t e = cudaPointerGetAttributes(&attr, host_dst);
+  if (e != cudaSuccess || attr.type != cudaMemoryTypeHost) {
+    cudaGetLastError();
+    return fail(GC_ERR_INVALID_ARG,
+                "gc_kv_save: host_dst must be pinned host memory "
+                "(cudaHostAlloc / cudaHostRegister) unless GC_SAVE_DST_DEVICE is set");
+  }
+  if (!dev_staging) {
+    // zero copy: the kernel writes the pinned buffer through its device alias
+    if (!attr.devicePointer)
+      return fail(GC_ERR_INVALID_ARG, "gc_kv_save: host_dst has no device mapping");
+    if (reinterpret_cast<uintptr_t>(attr.devicePointer) % 16)
+      return fail(GC_ERR_INVALID_ARG, "gc_kv_save: host_dst not 16-byte aligned");
+    return gc::launch_restore_vector(pool, static_cast<uint8_t*>(attr.devicePointer), block_ids,
+                                     n_blocks, true, stream);
+  }
+  if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
+    return fail(GC_ERR_INVALID_ARG, "gc_kv_save: dev_staging not 16-byte aligned");
+  uint8_t* stg = static_cast<uint8_t*>(dev_staging);
+  gc_status st = vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, true, stream)
+                        : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, true, stream);
+  if (st != GC_OK) return st;
+  e = cudaMemcpyAsync(host_dst, dev_staging, bytes, cudaMemcpyDeviceToHost, stream);
+  if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_save: copy to host");
+  return GC_OK;
 }
 
 gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v_new,

@@ -6,6 +6,8 @@
 //
 // Restore moves chunks of C = Hkv*ps*d*2 bytes: chunk c = (i, l, kv) of the
 // staging image [n_blocks][L][2][chunk] goes to pool[l][kv][block_ids[i]].
+// Save (Sec. 2.2, Fig. 2a step 1: a processed request's KV is saved to the
+// cache tier) is the same map run backwards: pool pages -> staging image.
 // The bulk kernel streams 16 KB pieces global -> shared -> global with
 // cp.async.bulk (one issuing thread per CTA, a ring of mbarrier-tracked
 // stages); the vector kernel uses 16-byte loads/stores and is also the
@@ -25,9 +27,10 @@ struct RestoreGeom {
   uint32_t pieces;          // ceil(C / kPiece)
   int32_t L, num_pages;
   int32_t n_blocks;
+  int32_t gather;           // 0: staging -> pool (restore), 1: pool -> staging (save)
 };
 
-__device__ __forceinline__ bool piece_addr(const RestoreGeom& g, const uint8_t* src, uint8_t* pool,
+__device__ __forceinline__ bool piece_addr(const RestoreGeom& g, uint8_t* staging, uint8_t* pool,
                                            const int32_t* block_ids, int32_t* status, uint64_t u,
                                            const uint8_t** s_out, uint8_t** d_out,
                                            uint32_t* bytes) {
@@ -44,12 +47,14 @@ __device__ __forceinline__ bool piece_addr(const RestoreGeom& g, const uint8_t* 
   const uint64_t off = static_cast<uint64_t>(piece) * kPiece;
   const uint64_t rem = g.chunk_bytes - off;
   *bytes = static_cast<uint32_t>(rem < kPiece ? rem : kPiece);
-  *s_out = src + c * g.chunk_bytes + off;
-  *d_out = pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) * g.chunk_bytes + off;
+  uint8_t* stg = staging + c * g.chunk_bytes + off;
+  uint8_t* pl = pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) * g.chunk_bytes + off;
+  *s_out = g.gather ? pl : stg;
+  *d_out = g.gather ? stg : pl;
   return true;
 }
 
-__global__ void __launch_bounds__(32) restore_bulk_kernel(const uint8_t* __restrict__ src,
+__global__ void __launch_bounds__(32) restore_bulk_kernel(uint8_t* __restrict__ staging,
                                                           uint8_t* __restrict__ pool,
                                                           const int32_t* __restrict__ block_ids,
                                                           RestoreGeom g, int32_t* status) {
@@ -72,7 +77,7 @@ __global__ void __launch_bounds__(32) restore_bulk_kernel(const uint8_t* __restr
       const uint8_t* s;
       uint8_t* d;
       uint32_t b;
-      const bool ok = piece_addr(g, src, pool, block_ids, status, next, &s, &d, &b);
+      const bool ok = piece_addr(g, staging, pool, block_ids, status, next, &s, &d, &b);
       next += gridDim.x;
       if (!ok) continue;
       dst_of[slot] = d;
@@ -112,7 +117,7 @@ __global__ void __launch_bounds__(32) restore_bulk_kernel(const uint8_t* __restr
   }
 }
 
-__global__ void __launch_bounds__(256) restore_vector_kernel(const uint4* __restrict__ src,
+__global__ void __launch_bounds__(256) restore_vector_kernel(uint4* __restrict__ staging,
                                                              uint8_t* __restrict__ pool,
                                                              const int32_t* __restrict__ block_ids,
                                                              RestoreGeom g, int32_t* status) {
@@ -123,7 +128,7 @@ __global__ void __launch_bounds__(256) restore_vector_kernel(const uint4* __rest
   for (uint64_t base = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x; base < total;
        base += stride * U) {
     uint4 v[U];
-    uint4* dst[U];
+    uint4* dst[U];  // destination word; the source was read into v
 #pragma unroll
     for (int k = 0; k < U; ++k) {
       const uint64_t w = base + k * stride;
@@ -139,11 +144,17 @@ __global__ void __launch_bounds__(256) restore_vector_kernel(const uint4* __rest
           if (off == 0 && l == 0 && kv == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
           continue;
         }
-        v[k] = src[w];
-        dst[k] = reinterpret_cast<uint4*>(
-                     pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) *
-                                g.chunk_bytes) +
-                 off;
+        uint4* pl = reinterpret_cast<uint4*>(
+                        pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) *
+                                   g.chunk_bytes) +
+                    off;
+        if (g.gather) {
+          v[k] = *pl;
+          dst[k] = staging + w;
+        } else {
+          v[k] = staging[w];
+          dst[k] = pl;
+        }
       }
     }
 #pragma unroll
@@ -214,9 +225,11 @@ int ilog2(int x) {
 
 }  // namespace
 
-gc_status launch_restore_bulk(const gc_kv_pool* pool, const uint8_t* src,
-                              const int32_t* block_ids, int32_t n_blocks, cudaStream_t stream) {
+gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
+                              const int32_t* block_ids, int32_t n_blocks, bool gather,
+                              cudaStream_t stream) {
   RestoreGeom g;
+  g.gather = gather ? 1 : 0;
   g.chunk_bytes = page_bytes(pool->cfg);
   g.pieces = static_cast<uint32_t>((g.chunk_bytes + kPiece - 1) / kPiece);
   g.L = pool->cfg.num_layers;
@@ -229,16 +242,19 @@ gc_status launch_restore_bulk(const gc_kv_pool* pool, const uint8_t* src,
   cudaError_t ea =
       cudaFuncSetAttribute(restore_bulk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (ea != cudaSuccess) return cuda_fail(ea, "gc_kv_restore: smem attribute");
-  restore_bulk_kernel<<<static_cast<unsigned>(grid), 32, smem, stream>>>(src, pool->data, block_ids,
-                                                                           g, pool->status);
+  restore_bulk_kernel<<<static_cast<unsigned>(grid), 32, smem, stream>>>(staging, pool->data,
+                                                                           block_ids, g,
+                                                                           pool->status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "gc_kv_restore: bulk kernel launch");
   return GC_OK;
 }
 
-gc_status launch_restore_vector(const gc_kv_pool* pool, const uint8_t* src,
-                                const int32_t* block_ids, int32_t n_blocks, cudaStream_t stream) {
+gc_status launch_restore_vector(const gc_kv_pool* pool, uint8_t* staging,
+                                const int32_t* block_ids, int32_t n_blocks, bool gather,
+                                cudaStream_t stream) {
   RestoreGeom g;
+  g.gather = gather ? 1 : 0;
   g.chunk_bytes = page_bytes(pool->cfg);
   g.pieces = 1;
   g.L = pool->cfg.num_layers;
@@ -249,7 +265,7 @@ gc_status launch_restore_vector(const gc_kv_pool* pool, const uint8_t* src,
   const uint64_t cap = static_cast<uint64_t>(pool->num_sms) * 8;
   if (grid > cap) grid = cap;
   restore_vector_kernel<<<static_cast<unsigned>(grid), 256, 0, stream>>>(
-      reinterpret_cast<const uint4*>(src), pool->data, block_ids, g, pool->status);
+      reinterpret_cast<uint4*>(staging), pool->data, block_ids, g, pool->status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "gc_kv_restore: vector kernel launch");
   return GC_OK;

@@ -80,6 +80,32 @@ class DeviceBatch:
         else:
             raise ValueError(mode)
 
+    def save(self, block_ids, mode: str = "staged", vector: bool = False, stream=None,
+             fill=0x7FC0) -> np.ndarray:
+        """gc_kv_save of pages `block_ids` into a fresh image [n][L][2][Hkv][ps][d]
+        pre-filled with `fill`; mode 'staged' (device staging, then a copy to
+        pinned host), 'device' (device destination) or 'zerocopy' (kernel writes
+        pinned host memory). Returns the image's bf16 bit patterns."""
+        import torch
+        w = self.w
+        ids = _i32(block_ids, self.device)
+        n = int(ids.numel())
+        shape = (n, w.L, 2, w.Hkv, w.ps, w.d)
+        flags = gcb.GC_SAVE_VECTOR if vector else 0
+        fill_i16 = int(np.uint16(fill).view(np.int16))
+        if mode == "device":
+            dst = torch.full(shape, fill_i16, dtype=torch.int16, device=self.device)
+            flags |= gcb.GC_SAVE_DST_DEVICE
+        else:
+            dst = torch.full(shape, fill_i16, dtype=torch.int16).pin_memory()
+        staging = (torch.empty(shape, dtype=torch.int16, device=self.device)
+                   if mode == "staged" else None)
+        if mode not in ("staged", "device", "zerocopy"):
+            raise ValueError(mode)
+        gcb.gc_kv_save(self.pool.handle, dst, ids, n, stream, staging, flags)
+        torch.cuda.synchronize()
+        return dst.cpu().numpy().view(np.uint16)
+
     def stage(self, stream=None):
         """Copy the pinned image into the device staging buffer (torch copy)."""
         if self.n_blocks:

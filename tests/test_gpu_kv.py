@@ -144,3 +144,64 @@ def test_library_owned_pool_matches_caller_owned():
     gcb.gc_kv_pool_destroy(h)
     assert torch.equal(out.view(torch.int16), ref.view(torch.int16))
     db.close()
+
+
+def _used_pages(w):
+    ids = []
+    for b in range(w.B):
+        ids.extend(w.block_table[b, :-(-int(w.total_lens[b]) // w.ps)].tolist())
+    return np.asarray(ids[::-1], dtype=np.int32)  # reversed: not pool order
+
+
+@pytest.mark.parametrize("mode,vector", [("staged", False), ("staged", True), ("device", False),
+                                         ("zerocopy", False)])
+@pytest.mark.parametrize("make", [wl.tiny, lambda: wl.llama3_8b_layer(seed=1, B=6)])
+def test_save_bit_exact(make, mode, vector):
+    """Sec. 2.2 step 1: the pages of processed requests saved to the cache
+    tier are byte-for-byte the pool pages (oracle gather of the same ids)."""
+    w = make()
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    ids = _used_pages(w)
+    got = db.save(ids, mode=mode, vector=vector)
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(got, oracle.kv_gather_blocks(oracle_pool(w), ids))
+    db.close()
+
+
+def test_save_then_restore_round_trip():
+    """Saving pages and restoring them elsewhere reproduces them exactly."""
+    w = wl.custom("roundtrip", 3, 8, 2, 128, 32, [70, 0, 300], [10, 40, 3], seed=13)
+    a = DeviceBatch(w)
+    a.restore()
+    a.append()
+    ids = _used_pages(w)
+    image = a.save(ids, mode="staged")
+    b = DeviceBatch(w, with_restore=False)
+    new_ids = np.random.default_rng(1).permutation(w.num_pages)[:ids.size].astype(np.int32)
+    import torch
+    src = torch.from_numpy(image.view(np.int16)).pin_memory()
+    staging = torch.empty_like(src, device="cuda")
+    gcb.gc_kv_restore(b.pool.handle, src, _i32(new_ids, "cuda"), ids.size, None, staging, 0)
+    assert b.check() == gcb.GC_OK and a.check() == gcb.GC_OK
+    pa, pb = a.pool_bits(), b.pool_bits()
+    assert np.array_equal(pa[:, :, ids], pb[:, :, new_ids])
+    a.close()
+    b.close()
+
+
+def test_save_skips_out_of_range_block_and_reports_it():
+    w = wl.tiny()
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    ids = _used_pages(w)
+    ids[2] = -3
+    got = db.save(ids, mode="device", fill=0x1234)
+    assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
+    keep = np.ones(ids.size, bool)
+    keep[2] = False
+    assert np.array_equal(got[keep], oracle.kv_gather_blocks(oracle_pool(w), ids[keep]))
+    assert np.all(got[2] == 0x1234)
+    db.close()
