@@ -7,13 +7,15 @@
  * GPU memory, the KV of the new tokens is stitched after it, and the new
  * tokens are prefilled against [cached context ++ new tokens] instead of
  * recomputing the whole context.  Sec. 2.1 defines the KV cache as the keys
- * and values of processed tokens kept for reuse.  The three calls below are
- * that step:
+ * and values of processed tokens kept for reuse.  The calls below are that
+ * step:
  *
  *   gc_kv_restore           cached pages (pinned host or device staging)
  *                           -> paged HBM KV pool                  (load)
  *   gc_kv_save              paged HBM KV pool -> pinned host / device
  *                           staging image; the inverse of restore  (save)
+ *   gc_kv_restore_layers,   the same for a range of layers, for restores
+ *   gc_kv_save_layers       and saves pipelined with per-layer compute
  *   gc_kv_append            new tokens' K,V -> pool slots after each
  *                           request's cached prefix                (stitch)
  *   gc_prefix_prefill_attn  causal GQA attention of the new tokens over
@@ -150,6 +152,27 @@ GC_API gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t
 GC_API gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
                         int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags);
 
+/* Restore layers [layer_begin, layer_begin + layer_count) of the cached
+ * pages only: the same map as gc_kv_restore restricted to those layers
+ * (gc_kv_restore is layer_begin 0, layer_count L).  A serving loop calls
+ * it once per layer on a side stream, each call followed by an event that
+ * the layer's compute waits on, so the restore of later layers overlaps the
+ * attention of earlier ones (Sec. 2.2, Fig. 2b: loading the cached KV
+ * costs far less time than recomputing it, so the load can hide behind the
+ * prefill of the new tokens).
+ *   host_src, dev_staging  the whole image [n_blocks][L][2][Hkv][ps][d] and
+ *              a device buffer of the same size, as for gc_kv_restore; only
+ *              the slices of the chosen layers are read (and, on the staged
+ *              path, copied into the same offsets of dev_staging with one
+ *              cudaMemcpy2DAsync), so calls for disjoint layer ranges touch
+ *              disjoint bytes and may run on different streams.
+ * Errors: as gc_kv_restore; GC_ERR_OUT_OF_RANGE for a layer range outside
+ * [0, L) (layer_count 0 is a no-op). */
+GC_API gc_status gc_kv_restore_layers(gc_kv_pool* pool, const void* host_src,
+                                      const int32_t* block_ids, int32_t n_blocks,
+                                      int32_t layer_begin, int32_t layer_count,
+                                      cudaStream_t stream, void* dev_staging, uint32_t flags);
+
 /* gc_kv_save flags */
 #define GC_SAVE_DST_DEVICE 1u /* host_dst is device memory (gather only) */
 #define GC_SAVE_VECTOR 2u     /* 16-byte vector-copy kernel instead of bulk copies */
@@ -177,6 +200,18 @@ GC_API gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int
 GC_API gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
                             int32_t n_blocks, cudaStream_t stream, void* dev_staging,
                             uint32_t flags);
+
+/* Save layers [layer_begin, layer_begin + layer_count) of the pages only:
+ * gc_kv_save restricted to those layers, written into the same offsets of
+ * the whole image [n_blocks][L][2][Hkv][ps][d] (host_dst, and dev_staging
+ * on the staged path, are whole-image buffers; other layers' bytes are not
+ * written).  Lets a request's KV be offloaded layer by layer as each layer
+ * finishes (Sec. 2.2, Fig. 2a step 1).
+ * Errors: as gc_kv_save; GC_ERR_OUT_OF_RANGE for a layer range outside
+ * [0, L) (layer_count 0 is a no-op). */
+GC_API gc_status gc_kv_save_layers(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
+                                   int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
+                                   cudaStream_t stream, void* dev_staging, uint32_t flags);
 
 /* Append the new tokens' K and V after each request's cached prefix
  * (Sec. 2.2: the KV of the cached tokens and of the new tokens is stitched

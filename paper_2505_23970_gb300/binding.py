@@ -33,7 +33,8 @@ GC_SAVE_VECTOR = 2
 
 EXPORTED = (
     "gc_kv_pool_bytes", "gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
-    "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_append", "gc_prefix_prefill_attn",
+    "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
+    "gc_kv_save_layers", "gc_kv_append", "gc_prefix_prefill_attn",
     "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc", "gc_last_error",
     "gc_status_string",
 )
@@ -75,13 +76,16 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_kv_pool_check.argtypes = [vp, vp, ctypes.POINTER(i32)]
         lib.gc_kv_restore.argtypes = [vp, vp, vp, i32, vp, vp, u32]
         lib.gc_kv_save.argtypes = [vp, vp, vp, i32, vp, vp, u32]
+        lib.gc_kv_restore_layers.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
+        lib.gc_kv_save_layers.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
         lib.gc_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, i32, vp, i32, i32, i32]
         attn = [vp, vp, vp, vp, vp, vp, vp, i32, vp, i32, i32, i32, ctypes.c_float, i32]
         lib.gc_prefix_prefill_attn.argtypes = attn
         lib.gc_prefix_prefill_attn_simt.argtypes = attn
         lib.gc_prefix_prefill_attn_noalloc.argtypes = attn
         for f in ("gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
-                  "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_append",
+                  "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
+                  "gc_kv_save_layers", "gc_kv_append",
                   "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt",
                   "gc_prefix_prefill_attn_noalloc"):
             getattr(lib, f).restype = ctypes.c_int
@@ -173,6 +177,20 @@ def gc_kv_save(pool, host_dst, block_ids, n_blocks: int, stream=None, dev_stagin
                flags: int = 0) -> None:
     _check(load().gc_kv_save(pool, _addr(host_dst), _addr(block_ids), n_blocks, _stream(stream),
                              _addr(dev_staging), flags), "gc_kv_save")
+
+
+def gc_kv_restore_layers(pool, host_src, block_ids, n_blocks: int, layer_begin: int,
+                         layer_count: int, stream=None, dev_staging=None, flags: int = 0) -> None:
+    _check(load().gc_kv_restore_layers(pool, _addr(host_src), _addr(block_ids), n_blocks,
+                                       layer_begin, layer_count, _stream(stream),
+                                       _addr(dev_staging), flags), "gc_kv_restore_layers")
+
+
+def gc_kv_save_layers(pool, host_dst, block_ids, n_blocks: int, layer_begin: int,
+                      layer_count: int, stream=None, dev_staging=None, flags: int = 0) -> None:
+    _check(load().gc_kv_save_layers(pool, _addr(host_dst), _addr(block_ids), n_blocks,
+                                    layer_begin, layer_count, _stream(stream), _addr(dev_staging),
+                                    flags), "gc_kv_save_layers")
 
 
 def gc_kv_append(pool, k_new, v_new, block_table, seq_lens, stream, layer: int, cu_new_lens,

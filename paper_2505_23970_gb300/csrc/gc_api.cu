@@ -159,18 +159,54 @@ gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t* devic
   return GC_OK;
 }
 
-gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
-                        int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+namespace {
+
+// Copy layers [lb, lb + lc) of every block between two whole images
+// [n][L][2][chunk] (same offsets on both sides): one copy when the range is
+// all layers, else one strided 2-D copy (rows = blocks).
+gc_status copy_layers(const char* who, void* dst, const void* src, int32_t n, int32_t L,
+                      int32_t lb, int32_t lc, size_t layer_bytes, cudaMemcpyKind kind,
+                      cudaStream_t stream) {
+  const size_t off = static_cast<size_t>(lb) * layer_bytes;
+  const size_t pitch = static_cast<size_t>(L) * layer_bytes;
+  const size_t width = static_cast<size_t>(lc) * layer_bytes;
+  cudaError_t e;
+  if (lc == L) {
+    e = cudaMemcpyAsync(dst, src, static_cast<size_t>(n) * pitch, kind, stream);
+  } else if (pitch <= 0x7fffffffu) {
+    e = cudaMemcpy2DAsync(static_cast<uint8_t*>(dst) + off, pitch,
+                          static_cast<const uint8_t*>(src) + off, pitch, width, n, kind, stream);
+  } else {  // beyond the 2-D copy's pitch limit: one copy per block
+    e = cudaSuccess;
+    for (int32_t i = 0; i < n && e == cudaSuccess; ++i)
+      e = cudaMemcpyAsync(static_cast<uint8_t*>(dst) + i * pitch + off,
+                          static_cast<const uint8_t*>(src) + i * pitch + off, width, kind, stream);
+  }
+  if (e != cudaSuccess) return gc::cuda_fail(e, who);
+  return GC_OK;
+}
+
+gc_status check_layers(const char* who, const gc_kv_pool* pool, int32_t lb, int32_t lc) {
+  const int32_t L = pool->cfg.num_layers;
+  if (lb < 0 || lc < 0 || lb > L || lc > L - lb)
+    return fail(GC_ERR_OUT_OF_RANGE, "%s: layers [%d, %d + %d) outside [0, %d)", who, lb, lb, lc,
+                L);
+  return GC_OK;
+}
+
+gc_status restore_impl(const char* who, gc_kv_pool* pool, const void* host_src,
+                       const int32_t* block_ids, int32_t n_blocks, int32_t lb, int32_t lc,
+                       cudaStream_t stream, void* dev_staging, uint32_t flags) {
   g_msg[0] = 0;
-  if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: pool is NULL");
-  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: n_blocks < 0");
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "%s: n_blocks < 0", who);
   if (flags & ~(GC_RESTORE_SRC_DEVICE | GC_RESTORE_VECTOR))
-    return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: unknown flags 0x%x", flags);
-  if (n_blocks == 0) return GC_OK;
-  if (!host_src || !block_ids)
-    return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: host_src / block_ids is NULL");
-  const size_t bytes = static_cast<size_t>(n_blocks) * pool->cfg.num_layers * 2 *
-                       gc::page_bytes(pool->cfg);
+    return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
+  gc_status st = check_layers(who, pool, lb, lc);
+  if (st != GC_OK) return st;
+  if (n_blocks == 0 || lc == 0) return GC_OK;
+  if (!host_src || !block_ids) return fail(GC_ERR_INVALID_ARG, "%s: host_src / block_ids is NULL", who);
+  const size_t layer_bytes = 2 * gc::page_bytes(pool->cfg);
   const uint8_t* src = static_cast<const uint8_t*>(host_src);
   bool vector = (flags & GC_RESTORE_VECTOR) != 0;
   if (!(flags & GC_RESTORE_SRC_DEVICE)) {
@@ -179,76 +215,104 @@ gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* b
     if (e != cudaSuccess || attr.type != cudaMemoryTypeHost) {
       cudaGetLastError();
       return fail(GC_ERR_INVALID_ARG,
-                  "gc_kv_restore: host_src must be pinned host memory "
-                  "(cudaHostAlloc / cudaHostRegister) unless GC_RESTORE_SRC_DEVICE is set");
+                  "%s: host_src must be pinned host memory "
+                  "(cudaHostAlloc / cudaHostRegister) unless GC_RESTORE_SRC_DEVICE is set", who);
     }
     if (dev_staging) {
       if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
-        return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: dev_staging not 16-byte aligned");
-      e = cudaMemcpyAsync(dev_staging, host_src, bytes, cudaMemcpyHostToDevice, stream);
-      if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_restore: staging copy");
+        return fail(GC_ERR_INVALID_ARG, "%s: dev_staging not 16-byte aligned", who);
+      st = copy_layers(who, dev_staging, host_src, n_blocks, pool->cfg.num_layers, lb, lc,
+                       layer_bytes, cudaMemcpyHostToDevice, stream);
+      if (st != GC_OK) return st;
       src = static_cast<const uint8_t*>(dev_staging);
     } else {
       // zero copy: the kernel reads the pinned buffer through its device alias
       void* dptr = attr.devicePointer;
-      if (!dptr) return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: host_src has no device mapping");
+      if (!dptr) return fail(GC_ERR_INVALID_ARG, "%s: host_src has no device mapping", who);
       src = static_cast<const uint8_t*>(dptr);
       vector = true;
     }
   }
   if (reinterpret_cast<uintptr_t>(src) % 16)
-    return fail(GC_ERR_INVALID_ARG, "gc_kv_restore: source not 16-byte aligned");
+    return fail(GC_ERR_INVALID_ARG, "%s: source not 16-byte aligned", who);
   uint8_t* stg = const_cast<uint8_t*>(src);  // read only when restoring
-  return vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, false, stream)
-                : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, false, stream);
+  return vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, lb, lc, false, stream)
+                : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, lb, lc, false, stream);
 }
 
-gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
-                     int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+gc_status save_impl(const char* who, gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
+                    int32_t n_blocks, int32_t lb, int32_t lc, cudaStream_t stream,
+                    void* dev_staging, uint32_t flags) {
   g_msg[0] = 0;
-  if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_kv_save: pool is NULL");
-  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "gc_kv_save: n_blocks < 0");
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "%s: n_blocks < 0", who);
   if (flags & ~(GC_SAVE_DST_DEVICE | GC_SAVE_VECTOR))
-    return fail(GC_ERR_INVALID_ARG, "gc_kv_save: unknown flags 0x%x", flags);
-  if (n_blocks == 0) return GC_OK;
-  if (!host_dst || !block_ids)
-    return fail(GC_ERR_INVALID_ARG, "gc_kv_save: host_dst / block_ids is NULL");
-  const size_t bytes = static_cast<size_t>(n_blocks) * pool->cfg.num_layers * 2 *
-                       gc::page_bytes(pool->cfg);
+    return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
+  gc_status st = check_layers(who, pool, lb, lc);
+  if (st != GC_OK) return st;
+  if (n_blocks == 0 || lc == 0) return GC_OK;
+  if (!host_dst || !block_ids) return fail(GC_ERR_INVALID_ARG, "%s: host_dst / block_ids is NULL", who);
+  const size_t layer_bytes = 2 * gc::page_bytes(pool->cfg);
   bool vector = (flags & GC_SAVE_VECTOR) != 0;
   if (flags & GC_SAVE_DST_DEVICE) {
     if (reinterpret_cast<uintptr_t>(host_dst) % 16)
-      return fail(GC_ERR_INVALID_ARG, "gc_kv_save: destination not 16-byte aligned");
+      return fail(GC_ERR_INVALID_ARG, "%s: destination not 16-byte aligned", who);
     uint8_t* dst = static_cast<uint8_t*>(host_dst);
-    return vector ? gc::launch_restore_vector(pool, dst, block_ids, n_blocks, true, stream)
-                  : gc::launch_restore_bulk(pool, dst, block_ids, n_blocks, true, stream);
+    return vector ? gc::launch_restore_vector(pool, dst, block_ids, n_blocks, lb, lc, true, stream)
+                  : gc::launch_restore_bulk(pool, dst, block_ids, n_blocks, lb, lc, true, stream);
   }
   cudaPointerAttributes attr;
   cudaError_t e = cudaPointerGetAttributes(&attr, host_dst);
   if (e != cudaSuccess || attr.type != cudaMemoryTypeHost) {
     cudaGetLastError();
     return fail(GC_ERR_INVALID_ARG,
-                "gc_kv_save: host_dst must be pinned host memory "
-                "(cudaHostAlloc / cudaHostRegister) unless GC_SAVE_DST_DEVICE is set");
+                "%s: host_dst must be pinned host memory "
+                "(cudaHostAlloc / cudaHostRegister) unless GC_SAVE_DST_DEVICE is set", who);
   }
   if (!dev_staging) {
     // zero copy: the kernel writes the pinned buffer through its device alias
-    if (!attr.devicePointer)
-      return fail(GC_ERR_INVALID_ARG, "gc_kv_save: host_dst has no device mapping");
+    if (!attr.devicePointer) return fail(GC_ERR_INVALID_ARG, "%s: host_dst has no device mapping", who);
     if (reinterpret_cast<uintptr_t>(attr.devicePointer) % 16)
-      return fail(GC_ERR_INVALID_ARG, "gc_kv_save: host_dst not 16-byte aligned");
+      return fail(GC_ERR_INVALID_ARG, "%s: host_dst not 16-byte aligned", who);
     return gc::launch_restore_vector(pool, static_cast<uint8_t*>(attr.devicePointer), block_ids,
-                                     n_blocks, true, stream);
+                                     n_blocks, lb, lc, true, stream);
   }
   if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
-    return fail(GC_ERR_INVALID_ARG, "gc_kv_save: dev_staging not 16-byte aligned");
+    return fail(GC_ERR_INVALID_ARG, "%s: dev_staging not 16-byte aligned", who);
   uint8_t* stg = static_cast<uint8_t*>(dev_staging);
-  gc_status st = vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, true, stream)
-                        : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, true, stream);
+  st = vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, lb, lc, true, stream)
+              : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, lb, lc, true, stream);
   if (st != GC_OK) return st;
-  e = cudaMemcpyAsync(host_dst, dev_staging, bytes, cudaMemcpyDeviceToHost, stream);
-  if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_save: copy to host");
-  return GC_OK;
+  return copy_layers(who, host_dst, dev_staging, n_blocks, pool->cfg.num_layers, lb, lc,
+                     layer_bytes, cudaMemcpyDeviceToHost, stream);
+}
+
+}  // namespace
+
+gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
+                        int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  return restore_impl("gc_kv_restore", pool, host_src, block_ids, n_blocks, 0,
+                      pool ? pool->cfg.num_layers : 0, stream, dev_staging, flags);
+}
+
+gc_status gc_kv_restore_layers(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
+                               int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
+                               cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  return restore_impl("gc_kv_restore_layers", pool, host_src, block_ids, n_blocks, layer_begin,
+                      layer_count, stream, dev_staging, flags);
+}
+
+gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
+                     int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  return save_impl("gc_kv_save", pool, host_dst, block_ids, n_blocks, 0,
+                   pool ? pool->cfg.num_layers : 0, stream, dev_staging, flags);
+}
+
+gc_status gc_kv_save_layers(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
+                            int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
+                            cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  return save_impl("gc_kv_save_layers", pool, host_dst, block_ids, n_blocks, layer_begin,
+                   layer_count, stream, dev_staging, flags);
 }
 
 gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v_new,

@@ -37,13 +37,15 @@ __device__ __forceinline__ void record_error(int32_t* status, int32_t code) {
 
 // ---------------------------------------------------------------- launchers
 // Each returns GC_OK or a status with the message already set.
-// Page copies between a staging image [n_blocks][L][2][chunk] and the pool;
-// gather = false restores (staging -> pool), gather = true saves.
+// Page copies between a staging image [n_blocks][L][2][chunk] and the pool,
+// layers [layer0, layer0 + layers) only; gather = false restores
+// (staging -> pool), gather = true saves.
 gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging, const int32_t* block_ids,
-                              int32_t n_blocks, bool gather, cudaStream_t stream);
+                              int32_t n_blocks, int32_t layer0, int32_t layers, bool gather,
+                              cudaStream_t stream);
 gc_status launch_restore_vector(const gc_kv_pool* pool, uint8_t* staging,
-                                const int32_t* block_ids, int32_t n_blocks, bool gather,
-                                cudaStream_t stream);
+                                const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
+                                int32_t layers, bool gather, cudaStream_t stream);
 gc_status launch_append(const gc_kv_pool* pool, const void* k_new, const void* v_new,
                         const int32_t* block_table, const int32_t* prefix_lens,
                         const int32_t* cu_new_lens, int32_t batch, int32_t max_blocks,

@@ -4,8 +4,11 @@
 // new tokens' KV is stitched after it), so the kernels are bandwidth-bound
 // and bit-exact.
 //
-// Restore moves chunks of C = Hkv*ps*d*2 bytes: chunk c = (i, l, kv) of the
-// staging image [n_blocks][L][2][chunk] goes to pool[l][kv][block_ids[i]].
+// Restore moves chunks of C = Hkv*ps*d*2 bytes: chunk (i, l, kv) of the
+// staging image [n_blocks][L][2][chunk] goes to pool[l][kv][block_ids[i]],
+// for the layers l of one contiguous range [layer0, layer0 + layers) (all L
+// for a whole-request restore, one layer when restores are pipelined with
+// the layers' compute).
 // Save (Sec. 2.2, Fig. 2a step 1: a processed request's KV is saved to the
 // cache tier) is the same map run backwards: pool pages -> staging image.
 // The bulk kernel streams 16 KB pieces global -> shared -> global with
@@ -25,7 +28,8 @@ constexpr int kBulkCtasPerSm = 2;
 struct RestoreGeom {
   uint64_t chunk_bytes;     // C
   uint32_t pieces;          // ceil(C / kPiece)
-  int32_t L, num_pages;
+  int32_t L, num_pages;     // layers of the pool and of the image; pages of the pool
+  int32_t layer0, layers;   // the layer range moved
   int32_t n_blocks;
   int32_t gather;           // 0: staging -> pool (restore), 1: pool -> staging (save)
 };
@@ -36,18 +40,19 @@ __device__ __forceinline__ bool piece_addr(const RestoreGeom& g, uint8_t* stagin
                                            uint32_t* bytes) {
   const uint64_t c = u / g.pieces;
   const uint32_t piece = static_cast<uint32_t>(u - c * g.pieces);
-  const int64_t i = static_cast<int64_t>(c / (2 * g.L));
-  const int l = static_cast<int>((c / 2) % g.L);
+  const int64_t i = static_cast<int64_t>(c / (2 * g.layers));
+  const int lr = static_cast<int>((c / 2) % g.layers);
+  const int l = g.layer0 + lr;
   const int kv = static_cast<int>(c % 2);
   const int32_t id = __ldg(block_ids + i);
   if (id < 0 || id >= g.num_pages) {
-    if (piece == 0 && l == 0 && kv == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
+    if (piece == 0 && lr == 0 && kv == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
     return false;
   }
   const uint64_t off = static_cast<uint64_t>(piece) * kPiece;
   const uint64_t rem = g.chunk_bytes - off;
   *bytes = static_cast<uint32_t>(rem < kPiece ? rem : kPiece);
-  uint8_t* stg = staging + c * g.chunk_bytes + off;
+  uint8_t* stg = staging + ((static_cast<uint64_t>(i) * g.L + l) * 2 + kv) * g.chunk_bytes + off;
   uint8_t* pl = pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) * g.chunk_bytes + off;
   *s_out = g.gather ? pl : stg;
   *d_out = g.gather ? stg : pl;
@@ -66,7 +71,7 @@ __global__ void __launch_bounds__(32) restore_bulk_kernel(uint8_t* __restrict__ 
   abort_flag = 0;
   ptx::fence_barrier_init();
 
-  const uint64_t units = static_cast<uint64_t>(g.n_blocks) * g.L * 2 * g.pieces;
+  const uint64_t units = static_cast<uint64_t>(g.n_blocks) * g.layers * 2 * g.pieces;
   uint64_t next = blockIdx.x;  // next candidate unit of this CTA
   uint8_t* dst_of[kStages];
   uint32_t bytes_of[kStages];
@@ -122,7 +127,7 @@ __global__ void __launch_bounds__(256) restore_vector_kernel(uint4* __restrict__
                                                              const int32_t* __restrict__ block_ids,
                                                              RestoreGeom g, int32_t* status) {
   const uint64_t words_per_chunk = g.chunk_bytes / 16;
-  const uint64_t total = static_cast<uint64_t>(g.n_blocks) * g.L * 2 * words_per_chunk;
+  const uint64_t total = static_cast<uint64_t>(g.n_blocks) * g.layers * 2 * words_per_chunk;
   const uint64_t stride = static_cast<uint64_t>(gridDim.x) * blockDim.x;
   constexpr int U = 4;
   for (uint64_t base = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x; base < total;
@@ -136,23 +141,25 @@ __global__ void __launch_bounds__(256) restore_vector_kernel(uint4* __restrict__
       if (w < total) {
         const uint64_t c = w / words_per_chunk;
         const uint64_t off = w - c * words_per_chunk;
-        const int64_t i = static_cast<int64_t>(c / (2 * g.L));
-        const int l = static_cast<int>((c / 2) % g.L);
+        const int64_t i = static_cast<int64_t>(c / (2 * g.layers));
+        const int lr = static_cast<int>((c / 2) % g.layers);
+        const int l = g.layer0 + lr;
         const int kv = static_cast<int>(c % 2);
         const int32_t id = __ldg(block_ids + i);
         if (id < 0 || id >= g.num_pages) {
-          if (off == 0 && l == 0 && kv == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
+          if (off == 0 && lr == 0 && kv == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
           continue;
         }
+        uint4* sw = staging + ((static_cast<uint64_t>(i) * g.L + l) * 2 + kv) * words_per_chunk + off;
         uint4* pl = reinterpret_cast<uint4*>(
                         pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) *
                                    g.chunk_bytes) +
                     off;
         if (g.gather) {
           v[k] = *pl;
-          dst[k] = staging + w;
+          dst[k] = sw;
         } else {
-          v[k] = staging[w];
+          v[k] = *sw;
           dst[k] = pl;
         }
       }
@@ -226,8 +233,8 @@ int ilog2(int x) {
 }  // namespace
 
 gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
-                              const int32_t* block_ids, int32_t n_blocks, bool gather,
-                              cudaStream_t stream) {
+                              const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
+                              int32_t layers, bool gather, cudaStream_t stream) {
   RestoreGeom g;
   g.gather = gather ? 1 : 0;
   g.chunk_bytes = page_bytes(pool->cfg);
@@ -235,7 +242,9 @@ gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
   g.L = pool->cfg.num_layers;
   g.num_pages = pool->cfg.num_pages;
   g.n_blocks = n_blocks;
-  const uint64_t units = static_cast<uint64_t>(n_blocks) * g.L * 2 * g.pieces;
+  g.layer0 = layer0;
+  g.layers = layers;
+  const uint64_t units = static_cast<uint64_t>(n_blocks) * layers * 2 * g.pieces;
   uint64_t grid = static_cast<uint64_t>(pool->num_sms) * kBulkCtasPerSm;
   if (grid > units) grid = units;
   const int smem = kStages * kPiece;
@@ -251,8 +260,8 @@ gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
 }
 
 gc_status launch_restore_vector(const gc_kv_pool* pool, uint8_t* staging,
-                                const int32_t* block_ids, int32_t n_blocks, bool gather,
-                                cudaStream_t stream) {
+                                const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
+                                int32_t layers, bool gather, cudaStream_t stream) {
   RestoreGeom g;
   g.gather = gather ? 1 : 0;
   g.chunk_bytes = page_bytes(pool->cfg);
@@ -260,7 +269,9 @@ gc_status launch_restore_vector(const gc_kv_pool* pool, uint8_t* staging,
   g.L = pool->cfg.num_layers;
   g.num_pages = pool->cfg.num_pages;
   g.n_blocks = n_blocks;
-  const uint64_t words = static_cast<uint64_t>(n_blocks) * g.L * 2 * (g.chunk_bytes / 16);
+  g.layer0 = layer0;
+  g.layers = layers;
+  const uint64_t words = static_cast<uint64_t>(n_blocks) * layers * 2 * (g.chunk_bytes / 16);
   uint64_t grid = (words + 256 * 4 - 1) / (256 * 4);
   const uint64_t cap = static_cast<uint64_t>(pool->num_sms) * 8;
   if (grid > cap) grid = cap;

@@ -141,3 +141,99 @@ class DeviceBatch:
 
     def close(self):
         self.pool.close()
+
+
+class LayerStack:
+    """One batch of requests through all `w.L` layers of one pool, the way a
+    serving loop prefills with reused context: per layer, the cached pages
+    of that layer are restored, the layer's new K/V appended and its
+    attention run.
+
+    ``run(pipelined=True)`` issues every layer's restore
+    (gc_kv_restore_layers, one layer per call) on a side stream with one
+    CUDA event per layer; the main stream waits for layer l's event before
+    layer l's append and attention, so the restore of later layers overlaps
+    the attention of earlier ones.  ``run(pipelined=False)`` restores all
+    layers first (one gc_kv_restore) and then computes layer by layer on one
+    stream.  Q and the new tokens' K/V are the same tensors for every layer
+    (inputs of the attention step, not produced here); the cached pages
+    differ per layer.  Only streams, events and buffers are handled here:
+    every byte is moved or computed by libgc."""
+
+    def __init__(self, w: Workload, device: str = "cuda", fill=BF16_NAN, keep_outputs=False,
+                 staging: bool = True):
+        import torch
+        self.w, self.device = w, device
+        self.pool = gcb.KVPool.create(w.L, w.Hkv, w.d, w.ps, w.num_pages, device=device)
+        self.pool.planes().view(torch.int16).fill_(int(np.uint16(fill).view(np.int16)))
+        self.block_table = _i32(w.block_table, device)
+        self.prefix_lens = _i32(w.prefix_lens, device)
+        self.new_lens = _i32(w.new_lens, device)
+        self.cu_new_lens = _i32(w.cu_new_lens, device)
+        ids = w.prefix_blocks()
+        self.n_blocks = int(ids.size)
+        self.block_ids = _i32(ids, device)
+        self.host_src = bf16_tensor(w.host_src(), pin=True) if self.n_blocks else None
+        self.staging = (torch.empty_like(self.host_src, device=device)
+                        if staging and self.n_blocks else None)
+        k, v = w.kv_new()
+        self.k_new, self.v_new = bf16_tensor(k, device), bf16_tensor(v, device)
+        self.q = bf16_tensor(w.q(), device)
+        n_out = w.L if keep_outputs else 1
+        self.outs = [torch.empty((w.T_new, w.Hq, w.d), dtype=torch.bfloat16, device=device)
+                     for _ in range(n_out)]
+        self.side = torch.cuda.Stream(device=device)
+        self.events = [torch.cuda.Event() for _ in range(w.L)]
+
+    def restore_layer(self, l, stream):
+        if self.n_blocks:
+            gcb.gc_kv_restore_layers(self.pool.handle, self.host_src, self.block_ids,
+                                     self.n_blocks, l, 1, stream, self.staging, 0)
+
+    def restore_all(self, stream):
+        if self.n_blocks:
+            gcb.gc_kv_restore(self.pool.handle, self.host_src, self.block_ids, self.n_blocks,
+                              stream, self.staging, 0)
+
+    def prefill_layer(self, l, stream):
+        w = self.w
+        h = self.pool.handle
+        gcb.gc_kv_append(h, self.k_new, self.v_new, self.block_table, self.prefix_lens, stream, l,
+                         self.cu_new_lens, w.B, w.max_blocks, w.T_new)
+        gcb.gc_prefix_prefill_attn(self.q, h, self.block_table, self.prefix_lens, self.new_lens,
+                                   self.outs[l % len(self.outs)], stream, l, self.cu_new_lens,
+                                   w.B, w.max_blocks, w.Hq, w.scale, w.T_new)
+
+    def run(self, pipelined: bool = True):
+        """Restore + append + attention of every layer, issued on the current
+        stream (and, when pipelined, the side stream for the restores)."""
+        import torch
+        main = torch.cuda.current_stream(self.device)
+        if not pipelined:
+            self.restore_all(main)
+            for l in range(self.w.L):
+                self.prefill_layer(l, main)
+            return
+        self.side.wait_stream(main)  # the restores may not pass earlier work on main
+        for l in range(self.w.L):
+            self.restore_layer(l, self.side)
+            self.events[l].record(self.side)
+        for l in range(self.w.L):
+            main.wait_event(self.events[l])
+            self.prefill_layer(l, main)
+
+    def prefill_only(self):
+        """Append + attention of every layer (the compute half alone)."""
+        import torch
+        main = torch.cuda.current_stream(self.device)
+        for l in range(self.w.L):
+            self.prefill_layer(l, main)
+
+    def check(self) -> int:
+        return self.pool.check(None)
+
+    def pool_bits(self) -> np.ndarray:
+        return bf16_bits(self.pool.planes())
+
+    def close(self):
+        self.pool.close()

@@ -223,6 +223,21 @@ def llama3_70b_restore_80layer(seed: int = 0, prefix: int = 8192) -> Workload:
     return w
 
 
+def llama3_70b_80layer_prefill(seed: int = 0, prefix: int = 8192, new: int = 1024,
+                               recompute: bool = False, B: int = 1) -> Workload:
+    """All 80 layers of the 70B-shaped model for B requests with an
+    8192-token cached prefix and 1024 new tokens each (restore of every
+    layer's cached pages + append + attention); recompute=True gives the
+    same context prefilled from scratch (prefix 0, prefix + new tokens)."""
+    if recompute:
+        w = _mk("llama3-70b-80layer-recompute", B, 64, 8, 128, 16, [0] * B, [prefix + new] * B,
+                seed)
+    else:
+        w = _mk("llama3-70b-80layer-prefill", B, 64, 8, 128, 16, [prefix] * B, [new] * B, seed)
+    w.L = 80
+    return w
+
+
 def conversation_mix(seed: int = 0, hit_p: float = 1.0, B: int = 64) -> Workload:
     """Multi-turn mix on the 70B-shaped layer: prefix ~ LogNormal(ln 2048, 1.0)
     clipped to [0, 32768], new ~ LogNormal(ln 200, 0.8) clipped to

@@ -223,3 +223,34 @@ def test_large_score_jumps_take_the_exact_path():
     src[:, 0, 0, 0] = keys.reshape(-1, 16, 128)
     w._cache["src"] = wl.f32_to_bf16_bits(src)
     full_parity(w)
+
+
+def test_layer_pipelined_schedule_matches_serial_and_oracle():
+    """Restoring layer l on a side stream (one gc_kv_restore_layers call per
+    layer, event-chained to the layer's append and attention) leaves the
+    pool and every layer's output bit-identical to restoring all layers
+    first; the pool equals the oracle's and the outputs match its attention."""
+    import torch
+    from paper_2505_23970_gb300.harness import LayerStack
+    w = wl.custom("layers", 2, 16, 2, 128, 16, [700, 33], [64, 130], seed=14)
+    w.L = 4
+    serial = LayerStack(w, keep_outputs=True)
+    serial.run(pipelined=False)
+    piped = LayerStack(w, keep_outputs=True)
+    piped.run(pipelined=True)
+    assert serial.check() == gcb.GC_OK and piped.check() == gcb.GC_OK
+    for a, b in zip(serial.outs, piped.outs):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    pool = w.empty_pool()
+    oracle.kv_restore(pool, w.host_src(), w.prefix_blocks())
+    k, v = w.kv_new()
+    for l in range(w.L):
+        oracle.kv_append(pool, l, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
+    assert np.array_equal(piped.pool_bits(), pool)
+    assert np.array_equal(serial.pool_bits(), pool)
+    for l in (0, 3):
+        ref = oracle.prefix_attn(w.q(), pool, l, w.block_table, w.prefix_lens, w.cu_new_lens,
+                                 w.scale)
+        assert_attn_close(piped.outs[l].to(torch.float64).cpu().numpy(), ref, f"layer {l}")
+    serial.close()
+    piped.close()

@@ -205,3 +205,90 @@ def test_save_skips_out_of_range_block_and_reports_it():
     assert np.array_equal(got[keep], oracle.kv_gather_blocks(oracle_pool(w), ids[keep]))
     assert np.all(got[2] == 0x1234)
     db.close()
+
+
+def _layered(seed=15):
+    w = wl.custom("layered", 3, 8, 2, 64, 16, [90, 0, 257], [7, 3, 20], seed=seed)
+    w.L = 5
+    return w
+
+
+@pytest.mark.parametrize("mode,vector", [("staged", False), ("staged", True), ("device", False),
+                                         ("zerocopy", False)])
+@pytest.mark.parametrize("lb,lc", [(0, 5), (1, 2), (4, 1)])
+def test_restore_layers_bit_exact(mode, vector, lb, lc):
+    """gc_kv_restore_layers writes exactly the chosen layers' pages of the
+    cached image and leaves every other layer untouched."""
+    w = _layered()
+    db = DeviceBatch(w)
+    if mode == "device":
+        db.stage()
+    src = db.staging if mode == "device" else db.host_src
+    staging = db.staging if mode == "staged" else None
+    flags = (gcb.GC_RESTORE_VECTOR if vector else 0) | (
+        gcb.GC_RESTORE_SRC_DEVICE if mode == "device" else 0)
+    gcb.gc_kv_restore_layers(db.pool.handle, src, db.block_ids, db.n_blocks, lb, lc, None,
+                             staging, flags)
+    assert db.check() == gcb.GC_OK
+    full = oracle_pool(w, append=False)
+    want = w.empty_pool()
+    want[lb:lb + lc] = full[lb:lb + lc]
+    assert np.array_equal(db.pool_bits(), want)
+    db.close()
+
+
+def test_restore_layers_one_call_per_layer_equals_whole_restore():
+    w = _layered(16)
+    db = DeviceBatch(w)
+    for l in range(w.L):
+        gcb.gc_kv_restore_layers(db.pool.handle, db.host_src, db.block_ids, db.n_blocks, l, 1,
+                                 None, db.staging, 0)
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(db.pool_bits(), oracle_pool(w, append=False))
+    db.close()
+
+
+@pytest.mark.parametrize("mode", ["staged", "device", "zerocopy"])
+@pytest.mark.parametrize("lb,lc", [(0, 5), (2, 3), (3, 1)])
+def test_save_layers_bit_exact(mode, lb, lc):
+    """gc_kv_save_layers writes the chosen layers' slices of the image (the
+    oracle's gather) and no other byte of it."""
+    import torch
+    w = _layered(17)
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    ids = _used_pages(w)
+    n = ids.size
+    shape = (n, w.L, 2, w.Hkv, w.ps, w.d)
+    fill = int(np.uint16(0x1234).view(np.int16))
+    flags = gcb.GC_SAVE_DST_DEVICE if mode == "device" else 0
+    if mode == "device":
+        dst = torch.full(shape, fill, dtype=torch.int16, device="cuda")
+    else:
+        dst = torch.full(shape, fill, dtype=torch.int16).pin_memory()
+    staging = torch.empty(shape, dtype=torch.int16, device="cuda") if mode == "staged" else None
+    gcb.gc_kv_save_layers(db.pool.handle, dst, _i32(ids, "cuda"), n, lb, lc, None, staging, flags)
+    assert db.check() == gcb.GC_OK
+    got = dst.cpu().numpy().view(np.uint16)
+    want = np.full(shape, 0x1234, dtype=np.uint16)
+    want[:, lb:lb + lc] = oracle.kv_gather_blocks(oracle_pool(w), ids)[:, lb:lb + lc]
+    assert np.array_equal(got, want)
+    db.close()
+
+
+def test_layer_range_checks():
+    w = _layered(18)
+    db = DeviceBatch(w)
+    before = db.pool_bits()
+    for lb, lc in [(-1, 1), (0, 6), (5, 1), (2, -1), (4, 2)]:
+        for fn, buf in ((gcb.gc_kv_restore_layers, db.host_src),
+                        (gcb.gc_kv_save_layers, db.host_src)):
+            with pytest.raises(gcb.GcError) as e:
+                fn(db.pool.handle, buf, db.block_ids, db.n_blocks, lb, lc, None, db.staging, 0)
+            assert e.value.status == gcb.GC_ERR_OUT_OF_RANGE
+    gcb.gc_kv_restore_layers(db.pool.handle, db.host_src, db.block_ids, db.n_blocks, 5, 0, None,
+                             db.staging, 0)  # empty range at the end: a no-op
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(db.pool_bits(), before)
+    db.close()
