@@ -457,6 +457,25 @@ def bench_restore80(args, pk):
     save_zc_ms = timed(lambda: gcb.gc_kv_save(db.pool.handle, host_dst, db.block_ids,
                                               db.n_blocks, stream, None, 0))
     d2h_ms = timed(lambda: host_dst.copy_(db.staging, non_blocking=True))
+    del host_dst
+    # the 8-bit cache tier: INT8 image of the same pages
+    n, L = db.n_blocks, w.L
+    q8_bytes = n * L * 2 * gcb.gc_kv_q8_chunk_bytes(db.pool.cfg)
+    q8_dev = torch.empty(q8_bytes, dtype=torch.uint8, device=db.staging.device)
+    q8_stg = torch.empty_like(q8_dev)
+    q8_host = torch.empty(q8_bytes, dtype=torch.uint8).pin_memory()
+    q8_save_ms = timed(lambda: gcb.gc_kv_save_q8(db.pool.handle, q8_dev, db.block_ids, n, 0, L,
+                                                 stream, None, gcb.GC_SAVE_DST_DEVICE))
+    q8_restore_ms = timed(lambda: gcb.gc_kv_restore_q8(db.pool.handle, q8_dev, db.block_ids, n, 0,
+                                                       L, stream, None,
+                                                       gcb.GC_RESTORE_SRC_DEVICE))
+    q8_save_host_ms = timed(lambda: gcb.gc_kv_save_q8(db.pool.handle, q8_host, db.block_ids, n, 0,
+                                                      L, stream, q8_stg, 0))
+    q8_staged_ms = timed(lambda: gcb.gc_kv_restore_q8(db.pool.handle, q8_host, db.block_ids, n, 0,
+                                                      L, stream, q8_stg, 0))
+    q8_zc_ms = timed(lambda: gcb.gc_kv_restore_q8(db.pool.handle, q8_host, db.block_ids, n, 0, L,
+                                                  stream, None, 0))
+    del q8_dev, q8_stg, q8_host
     ok = db.check(stream) == gcb.GC_OK
     db.close()
     gbs = lambda nbytes, ms: nbytes / (ms / 1e3) / 1e9  # noqa: E731
@@ -473,6 +492,20 @@ def bench_restore80(args, pk):
         "pool_to_host_staged_gbs": gbs(payload, save_staged_ms),
         "pool_to_host_zero_copy_gbs": gbs(payload, save_zc_ms),
         "pinned_d2h_memcpy_gbs": gbs(payload, d2h_ms),
+        "q8": {
+            "image_bytes": q8_bytes,
+            "dequant_scatter_gbs": gbs(q8_bytes + payload, q8_restore_ms),
+            "dequant_scatter_frac_hbm": gbs(q8_bytes + payload, q8_restore_ms) / pk["hbm_gbs"],
+            "quant_gather_gbs": gbs(payload + q8_bytes, q8_save_ms),
+            "quant_gather_frac_hbm": gbs(payload + q8_bytes, q8_save_ms) / pk["hbm_gbs"],
+            "host_to_pool_staged_image_gbs": gbs(q8_bytes, q8_staged_ms),
+            "host_to_pool_staged_bf16_equiv_gbs": gbs(payload, q8_staged_ms),
+            "host_to_pool_zero_copy_bf16_equiv_gbs": gbs(payload, q8_zc_ms),
+            "pool_to_host_staged_image_gbs": gbs(q8_bytes, q8_save_host_ms),
+            "ms": {"dequant_scatter": q8_restore_ms, "quant_gather": q8_save_ms,
+                   "staged": q8_staged_ms, "zero_copy": q8_zc_ms,
+                   "save_staged": q8_save_host_ms},
+        },
         "ms": {"scatter_bulk": scatter_ms, "scatter_vector": vec_ms, "staged": staged_ms,
                "zero_copy": zc_ms, "h2d_memcpy": h2d_ms, "save_gather": save_dev_ms,
                "save_staged": save_staged_ms, "save_zero_copy": save_zc_ms,
@@ -519,14 +552,20 @@ def bench_ttft80(args, image=None):
         for l in range(w.L):
             cached.restore_layer(l, stream)
 
-    ms = {
+    ms = {}
+    cached.restore_all(stream)
+    cached.use_q8()      # 8-bit cache tier: the same pages as an INT8 image
+    ms["pipelined_q8"] = timed(lambda: cached.run(pipelined=True))
+    ms["restore_per_layer_only_q8"] = timed(restore_layers)
+    cached.q8 = False
+    ms.update({
         "pipelined": timed(lambda: cached.run(pipelined=True)),
         "sequential": timed(lambda: cached.run(pipelined=False)),
         "restore_per_layer_only": timed(restore_layers),
         "restore_whole_only": timed(lambda: cached.restore_all(stream)),
         "prefill_only": timed(cached.prefill_only),
         "recompute": timed(scratch.prefill_only),
-    }
+    })
     ok = cached.check() == gcb.GC_OK and scratch.check() == gcb.GC_OK
     cached.close()
     scratch.close()
@@ -537,6 +576,7 @@ def bench_ttft80(args, image=None):
         "device_status_ok": ok, "ms": ms,
         "restore_hidden_frac": hidden / ms["restore_per_layer_only"],
         "speedup_vs_recompute": ms["recompute"] / ms["pipelined"],
+        "speedup_vs_recompute_q8": ms["recompute"] / ms["pipelined_q8"],
         "restore_bytes": int(w.prefix_blocks().size) * w.page_bytes,
         "gpu_launches_pipelined": 3 * w.L,
     }

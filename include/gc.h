@@ -16,6 +16,8 @@
  *                           staging image; the inverse of restore  (save)
  *   gc_kv_restore_layers,   the same for a range of layers, for restores
  *   gc_kv_save_layers       and saves pipelined with per-layer compute
+ *   gc_kv_save_q8,          the same with an 8-bit (INT8 + scales) image
+ *   gc_kv_restore_q8        in the cache tier
  *   gc_kv_append            new tokens' K,V -> pool slots after each
  *                           request's cached prefix                (stitch)
  *   gc_prefix_prefill_attn  causal GQA attention of the new tokens over
@@ -129,6 +131,7 @@ GC_API gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t
 /* gc_kv_restore flags */
 #define GC_RESTORE_SRC_DEVICE 1u /* host_src is device memory (already staged) */
 #define GC_RESTORE_VECTOR 2u     /* 16-byte vector-copy kernel instead of bulk copies */
+#define GC_RESTORE_LAYER_MAJOR 4u /* image is [L][n_blocks][2][Hkv][ps][d] (see below) */
 
 /* Restore cached prefix pages into the pool (Sec. 2.2, Fig. 2a: on a hit
  * the cached KV of the context is loaded instead of recomputed).
@@ -166,6 +169,15 @@ GC_API gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int
  *              path, copied into the same offsets of dev_staging with one
  *              cudaMemcpy2DAsync), so calls for disjoint layer ranges touch
  *              disjoint bytes and may run on different streams.
+ *   GC_RESTORE_LAYER_MAJOR  (any restore or save call, with the matching
+ *              GC_SAVE_LAYER_MAJOR) the image is laid out [L][n_blocks][2]
+ *              [Hkv][ps][d] instead: element (i, l, kv) of the map above sits
+ *              at chunk (l*n_blocks + i)*2 + kv.  A layer range is then one
+ *              contiguous span and the staged path copies it with one
+ *              cudaMemcpyAsync; for the block-major image the strided 2-D
+ *              copy of one layer runs at about a third of the contiguous
+ *              copy's rate on a GB300 host link, so per-layer callers should
+ *              keep their cache images layer-major.
  * Errors: as gc_kv_restore; GC_ERR_OUT_OF_RANGE for a layer range outside
  * [0, L) (layer_count 0 is a no-op). */
 GC_API gc_status gc_kv_restore_layers(gc_kv_pool* pool, const void* host_src,
@@ -176,6 +188,7 @@ GC_API gc_status gc_kv_restore_layers(gc_kv_pool* pool, const void* host_src,
 /* gc_kv_save flags */
 #define GC_SAVE_DST_DEVICE 1u /* host_dst is device memory (gather only) */
 #define GC_SAVE_VECTOR 2u     /* 16-byte vector-copy kernel instead of bulk copies */
+#define GC_SAVE_LAYER_MAJOR 4u /* image is [L][n_blocks][2][Hkv][ps][d] */
 
 /* Save pool pages to the cache tier (Sec. 2.2, Fig. 2a step 1: once a
  * request has been processed its KV is saved to storage); the inverse of
@@ -212,6 +225,40 @@ GC_API gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* blo
 GC_API gc_status gc_kv_save_layers(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
                                    int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
                                    cudaStream_t stream, void* dev_staging, uint32_t flags);
+
+/* ---- 8-bit cache tier.  The 70B runs of Sec. 6.1 use INT8; keeping the
+ * cached KV in 8 bits halves what the cache tier stores (the storage whose
+ * embodied carbon Sec. 3.2, Eq. 4 charges per allocated byte) and what the
+ * host link carries on a restore.  The pool stays bf16.
+ * Quantisation is symmetric absmax INT8 with one binary32 scale per
+ * (block, layer, plane kv, kv head g) group of ps*d values x:
+ *     amax = max |x| over the group's finite values
+ *     s    = amax / 127
+ *     c    = clamp(round_half_even(x * (127 / amax)), -127, 127)
+ *            (c = 0 for NaN x; every c = 0 when amax = 0)
+ * each product and quotient rounded once in binary32; restore writes
+ *     pool value = bf16_round_half_even(c * s).
+ * Image: [n_blocks][L][2][chunk] (or [L][n_blocks][2][chunk] with the
+ * LAYER_MAJOR flag), chunk = gc_kv_q8_chunk_bytes(cfg) bytes: Hkv binary32
+ * scales, zero bytes up to a multiple of 16, then codes [Hkv][ps][d] int8.
+ * Both calls take the same layer range, source / destination modes
+ * (pinned host through dev_staging, zero copy with dev_staging NULL, or a
+ * device image with GC_RESTORE_SRC_DEVICE / GC_SAVE_DST_DEVICE), block-id
+ * checks and errors as gc_kv_restore_layers / gc_kv_save_layers; the
+ * *_VECTOR flags do not apply. */
+GC_API size_t gc_kv_q8_chunk_bytes(const gc_pool_config* cfg);  /* 0 if invalid */
+
+/* Quantise pages block_ids[i], layers [layer_begin, layer_begin+layer_count),
+ * into the 8-bit image (chunks of other layers are not written). */
+GC_API gc_status gc_kv_save_q8(gc_kv_pool* pool, void* dst, const int32_t* block_ids,
+                               int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
+                               cudaStream_t stream, void* dev_staging, uint32_t flags);
+
+/* Dequantise the 8-bit image's chunks of those layers into pool pages
+ * block_ids[i]; no other page or layer changes. */
+GC_API gc_status gc_kv_restore_q8(gc_kv_pool* pool, const void* src, const int32_t* block_ids,
+                                  int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
+                                  cudaStream_t stream, void* dev_staging, uint32_t flags);
 
 /* Append the new tokens' K and V after each request's cached prefix
  * (Sec. 2.2: the KV of the cached tokens and of the new tokens is stitched

@@ -57,6 +57,10 @@ def _load():
             lib.oracle_bf16_to_double.restype = dbl
             lib.oracle_kv_restore.argtypes = [p, i32, i32, i32, i32, i32, p, p, i32]
             lib.oracle_kv_gather_blocks.argtypes = [p, i32, i32, i32, i32, i32, p, i32, p]
+            lib.oracle_q8_chunk_bytes.argtypes = [i32, i32, i32]
+            lib.oracle_q8_chunk_bytes.restype = ctypes.c_size_t
+            lib.oracle_kv_save_q8.argtypes = [p, i32, i32, i32, i32, i32, p, i32, i32, i32, p]
+            lib.oracle_kv_restore_q8.argtypes = [p, i32, i32, i32, i32, i32, p, p, i32, i32, i32]
             lib.oracle_kv_append.argtypes = [p, i32, i32, i32, i32, i32, i32, p, p, p, i32, p, p, i32]
             lib.oracle_prefix_attn.argtypes = [p, p, i32, i32, i32, i32, i32, i32, p, i32, p, p,
                                                i32, i32, dbl, p, i32]
@@ -128,6 +132,55 @@ def kv_gather_blocks(pool: np.ndarray, block_ids) -> np.ndarray:
     _check(_load().oracle_kv_gather_blocks(_ptr(_u16(pool)), L, Hkv, ps, d, NP, _ptr(ids),
                                            ids.size, _ptr(out)), "kv_gather_blocks")
     return out
+
+
+def q8_chunk_bytes(Hkv: int, ps: int, d: int) -> int:
+    """Bytes of one (block, layer, plane) chunk of the 8-bit image."""
+    return int(_load().oracle_q8_chunk_bytes(Hkv, ps, d))
+
+
+def kv_save_q8(pool: np.ndarray, block_ids, layer_begin: int = 0, layer_count=None,
+               out: np.ndarray | None = None) -> np.ndarray:
+    """8-bit image [n_blocks][L][2][chunk] (uint8) of pages block_ids, layers
+    [layer_begin, layer_begin + layer_count) written (into `out` if given,
+    else into a zero image)."""
+    L, _, NP, Hkv, ps, d = pool.shape
+    if layer_count is None:
+        layer_count = L - layer_begin
+    ids = _i32(block_ids)
+    chunk = q8_chunk_bytes(Hkv, ps, d)
+    if out is None:
+        out = np.zeros((ids.size, L, 2, chunk), dtype=np.uint8)
+    assert out.dtype == np.uint8 and out.flags.c_contiguous and out.shape == (ids.size, L, 2, chunk)
+    _check(_load().oracle_kv_save_q8(_ptr(_u16(pool)), L, Hkv, ps, d, NP, _ptr(ids), ids.size,
+                                     layer_begin, layer_count, _ptr(out)), "kv_save_q8")
+    return out
+
+
+def kv_restore_q8(pool: np.ndarray, image: np.ndarray, block_ids, layer_begin: int = 0,
+                  layer_count=None) -> None:
+    """In place: dequantise the 8-bit image's chunks into the pool pages."""
+    assert pool.dtype == np.uint16 and pool.flags.c_contiguous
+    L, _, NP, Hkv, ps, d = pool.shape
+    if layer_count is None:
+        layer_count = L - layer_begin
+    ids = _i32(block_ids)
+    img = np.ascontiguousarray(image, dtype=np.uint8)
+    assert img.size == ids.size * L * 2 * q8_chunk_bytes(Hkv, ps, d)
+    _check(_load().oracle_kv_restore_q8(_ptr(pool), L, Hkv, ps, d, NP, _ptr(img), _ptr(ids),
+                                        ids.size, layer_begin, layer_count), "kv_restore_q8")
+
+
+def q8_split(image: np.ndarray, Hkv: int, ps: int, d: int):
+    """(scales [n][L][2][Hkv] float32, codes [n][L][2][Hkv][ps][d] int8) views
+    of an 8-bit image (layout plumbing, no arithmetic)."""
+    n, L = image.shape[:2]
+    chunk = q8_chunk_bytes(Hkv, ps, d)
+    hdr = chunk - Hkv * ps * d
+    flat = image.reshape(n, L, 2, chunk)
+    scales = np.ascontiguousarray(flat[..., :4 * Hkv]).view(np.float32)
+    codes = np.ascontiguousarray(flat[..., hdr:]).view(np.int8).reshape(n, L, 2, Hkv, ps, d)
+    return scales, codes
 
 
 def kv_append(pool: np.ndarray, layer: int, k_new, v_new, block_table, prefix_lens,

@@ -100,6 +100,109 @@ int oracle_kv_gather_blocks(const uint16_t *pool, int L, int Hkv, int ps, int d,
     return OR_OK;
 }
 
+/* ------------------------------------------------------ 8-bit cache tier */
+/* An 8-bit copy of the cached pages for the cache tier (the 70B runs of
+ * Sec. 6.1 use INT8; an 8-bit image halves the bytes the tier stores and
+ * the host link carries).  Symmetric absmax INT8 with one scale per
+ * (block, layer, plane, kv head) group of ps*d values:
+ *   amax = max |x| over the group's finite values
+ *   s    = amax / 127                      (stored, binary32)
+ *   c    = clamp(round_half_even(x * (127 / amax)), -127, 127), 0 for NaN
+ *          (all codes 0 when amax is 0)
+ *   x'   = bf16_round_half_even(c * s)     (restore)
+ * The code is an integer decided by floating point, so it is decided here
+ * in binary32 like the kernel does (x * inv and 127 / amax each rounded
+ * once), not in float64.
+ * Image chunk of one (block, layer, plane): Hkv binary32 scales, zero padding
+ * to a multiple of 16 bytes, then the codes [Hkv][ps][d] as int8; the image
+ * is [n_blocks][L][2][chunk]. */
+size_t oracle_q8_chunk_bytes(int Hkv, int ps, int d) {
+    size_t hdr = ((size_t)Hkv * 4 + 15) / 16 * 16;
+    return hdr + (size_t)Hkv * ps * d;
+}
+
+static float bf16_to_float(uint16_t bits) {
+    uint32_t u = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return f;
+}
+
+/* binary32 -> bf16 bits, round half to even (finite inputs only here). */
+static uint16_t float_to_bf16_rne(float f) {
+    uint32_t u;
+    memcpy(&u, &f, sizeof u);
+    uint32_t lsb = (u >> 16) & 1u;
+    u += 0x7fffu + lsb;
+    return (uint16_t)(u >> 16);
+}
+
+static int8_t q8_code(float x, float inv) {
+    if (isnan(x)) return 0;
+    float v = x * inv;
+    if (isnan(v)) return 0;          /* inf * 0 when amax is 0 */
+    if (v > 127.0f) v = 127.0f;
+    if (v < -127.0f) v = -127.0f;
+    return (int8_t)rintf(v);         /* default rounding: half to even */
+}
+
+int oracle_kv_save_q8(const uint16_t *pool, int L, int Hkv, int ps, int d, int num_pages,
+                      const int32_t *block_ids, int n_blocks, int layer_begin, int layer_count,
+                      uint8_t *dst) {
+    if (layer_begin < 0 || layer_count < 0 || layer_begin + layer_count > L) return OR_ERR_ARG;
+    size_t chunk = oracle_q8_chunk_bytes(Hkv, ps, d);
+    size_t hdr = chunk - (size_t)Hkv * ps * d;
+    size_t group = (size_t)ps * d;
+    for (int i = 0; i < n_blocks; ++i) {
+        int page = block_ids[i];
+        if (page < 0 || page >= num_pages) return OR_ERR_RANGE;
+        for (int l = layer_begin; l < layer_begin + layer_count; ++l)
+            for (int kv = 0; kv < 2; ++kv) {
+                uint8_t *c = dst + (((size_t)i * L + l) * 2 + kv) * chunk;
+                memset(c, 0, hdr);
+                for (int g = 0; g < Hkv; ++g) {
+                    const uint16_t *x = pool + pool_index(L, Hkv, ps, d, num_pages, l, kv, page, g, 0, 0);
+                    float amax = 0.0f;
+                    for (size_t e = 0; e < group; ++e) {
+                        float a = fabsf(bf16_to_float(x[e]));
+                        if (isfinite(a) && a > amax) amax = a;
+                    }
+                    float scale = amax / 127.0f;
+                    float inv = amax > 0.0f ? 127.0f / amax : 0.0f;
+                    memcpy(c + (size_t)g * 4, &scale, 4);
+                    int8_t *codes = (int8_t *)(c + hdr) + (size_t)g * group;
+                    for (size_t e = 0; e < group; ++e) codes[e] = q8_code(bf16_to_float(x[e]), inv);
+                }
+            }
+    }
+    return OR_OK;
+}
+
+int oracle_kv_restore_q8(uint16_t *pool, int L, int Hkv, int ps, int d, int num_pages,
+                         const uint8_t *src, const int32_t *block_ids, int n_blocks,
+                         int layer_begin, int layer_count) {
+    if (layer_begin < 0 || layer_count < 0 || layer_begin + layer_count > L) return OR_ERR_ARG;
+    size_t chunk = oracle_q8_chunk_bytes(Hkv, ps, d);
+    size_t hdr = chunk - (size_t)Hkv * ps * d;
+    size_t group = (size_t)ps * d;
+    for (int i = 0; i < n_blocks; ++i)
+        if (block_ids[i] < 0 || block_ids[i] >= num_pages) return OR_ERR_RANGE;
+    for (int i = 0; i < n_blocks; ++i)
+        for (int l = layer_begin; l < layer_begin + layer_count; ++l)
+            for (int kv = 0; kv < 2; ++kv) {
+                const uint8_t *c = src + (((size_t)i * L + l) * 2 + kv) * chunk;
+                for (int g = 0; g < Hkv; ++g) {
+                    float scale;
+                    memcpy(&scale, c + (size_t)g * 4, 4);
+                    const int8_t *codes = (const int8_t *)(c + hdr) + (size_t)g * group;
+                    uint16_t *y = pool + pool_index(L, Hkv, ps, d, num_pages, l, kv, block_ids[i], g, 0, 0);
+                    for (size_t e = 0; e < group; ++e)
+                        y[e] = float_to_bf16_rne((float)codes[e] * scale);
+                }
+            }
+    return OR_OK;
+}
+
 /* ----------------------------------------------------------------- append */
 /* Sec. 2.2: stitch the new tokens' KV after the cached prefix.  Token t of
  * request b sits at absolute position prefix_lens[b] + t of its sequence. */

@@ -30,11 +30,14 @@ GC_RESTORE_SRC_DEVICE = 1
 GC_RESTORE_VECTOR = 2
 GC_SAVE_DST_DEVICE = 1
 GC_SAVE_VECTOR = 2
+GC_RESTORE_LAYER_MAJOR = 4
+GC_SAVE_LAYER_MAJOR = 4
 
 EXPORTED = (
     "gc_kv_pool_bytes", "gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
     "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
-    "gc_kv_save_layers", "gc_kv_append", "gc_prefix_prefill_attn",
+    "gc_kv_save_layers", "gc_kv_q8_chunk_bytes", "gc_kv_save_q8", "gc_kv_restore_q8",
+    "gc_kv_append", "gc_prefix_prefill_attn",
     "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc", "gc_last_error",
     "gc_status_string",
 )
@@ -78,6 +81,10 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_kv_save.argtypes = [vp, vp, vp, i32, vp, vp, u32]
         lib.gc_kv_restore_layers.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
         lib.gc_kv_save_layers.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
+        lib.gc_kv_q8_chunk_bytes.argtypes = [ctypes.POINTER(gc_pool_config)]
+        lib.gc_kv_q8_chunk_bytes.restype = ctypes.c_size_t
+        lib.gc_kv_save_q8.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
+        lib.gc_kv_restore_q8.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
         lib.gc_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, i32, vp, i32, i32, i32]
         attn = [vp, vp, vp, vp, vp, vp, vp, i32, vp, i32, i32, i32, ctypes.c_float, i32]
         lib.gc_prefix_prefill_attn.argtypes = attn
@@ -85,7 +92,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_prefix_prefill_attn_noalloc.argtypes = attn
         for f in ("gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
                   "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
-                  "gc_kv_save_layers", "gc_kv_append",
+                  "gc_kv_save_layers", "gc_kv_save_q8", "gc_kv_restore_q8", "gc_kv_append",
                   "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt",
                   "gc_prefix_prefill_attn_noalloc"):
             getattr(lib, f).restype = ctypes.c_int
@@ -191,6 +198,24 @@ def gc_kv_save_layers(pool, host_dst, block_ids, n_blocks: int, layer_begin: int
     _check(load().gc_kv_save_layers(pool, _addr(host_dst), _addr(block_ids), n_blocks,
                                     layer_begin, layer_count, _stream(stream), _addr(dev_staging),
                                     flags), "gc_kv_save_layers")
+
+
+def gc_kv_q8_chunk_bytes(cfg: gc_pool_config) -> int:
+    return int(load().gc_kv_q8_chunk_bytes(ctypes.byref(cfg)))
+
+
+def gc_kv_save_q8(pool, dst, block_ids, n_blocks: int, layer_begin: int, layer_count: int,
+                  stream=None, dev_staging=None, flags: int = 0) -> None:
+    _check(load().gc_kv_save_q8(pool, _addr(dst), _addr(block_ids), n_blocks, layer_begin,
+                                layer_count, _stream(stream), _addr(dev_staging), flags),
+           "gc_kv_save_q8")
+
+
+def gc_kv_restore_q8(pool, src, block_ids, n_blocks: int, layer_begin: int, layer_count: int,
+                     stream=None, dev_staging=None, flags: int = 0) -> None:
+    _check(load().gc_kv_restore_q8(pool, _addr(src), _addr(block_ids), n_blocks, layer_begin,
+                                   layer_count, _stream(stream), _addr(dev_staging), flags),
+           "gc_kv_restore_q8")
 
 
 def gc_kv_append(pool, k_new, v_new, block_table, seq_lens, stream, layer: int, cu_new_lens,

@@ -161,26 +161,33 @@ gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t* devic
 
 namespace {
 
-// Copy layers [lb, lb + lc) of every block between two whole images
-// [n][L][2][chunk] (same offsets on both sides): one copy when the range is
-// all layers, else one strided 2-D copy (rows = blocks).
+// Copy layers [lb, lb + lc) of every block between two whole images (same
+// offsets on both sides).  Layer-major images [L][n][2][chunk], or a range
+// of all layers: one contiguous copy.  Block-major images [n][L][2][chunk]:
+// one strided 2-D copy (rows = blocks).
 gc_status copy_layers(const char* who, void* dst, const void* src, int32_t n, int32_t L,
-                      int32_t lb, int32_t lc, size_t layer_bytes, cudaMemcpyKind kind,
-                      cudaStream_t stream) {
-  const size_t off = static_cast<size_t>(lb) * layer_bytes;
-  const size_t pitch = static_cast<size_t>(L) * layer_bytes;
-  const size_t width = static_cast<size_t>(lc) * layer_bytes;
+                      int32_t lb, int32_t lc, size_t layer_bytes, bool layer_major,
+                      cudaMemcpyKind kind, cudaStream_t stream) {
   cudaError_t e;
-  if (lc == L) {
-    e = cudaMemcpyAsync(dst, src, static_cast<size_t>(n) * pitch, kind, stream);
-  } else if (pitch <= 0x7fffffffu) {
-    e = cudaMemcpy2DAsync(static_cast<uint8_t*>(dst) + off, pitch,
-                          static_cast<const uint8_t*>(src) + off, pitch, width, n, kind, stream);
-  } else {  // beyond the 2-D copy's pitch limit: one copy per block
-    e = cudaSuccess;
-    for (int32_t i = 0; i < n && e == cudaSuccess; ++i)
-      e = cudaMemcpyAsync(static_cast<uint8_t*>(dst) + i * pitch + off,
-                          static_cast<const uint8_t*>(src) + i * pitch + off, width, kind, stream);
+  if (layer_major || lc == L) {
+    const size_t off = layer_major ? static_cast<size_t>(lb) * n * layer_bytes : 0;
+    const size_t len = static_cast<size_t>(lc) * n * layer_bytes;
+    e = cudaMemcpyAsync(static_cast<uint8_t*>(dst) + off, static_cast<const uint8_t*>(src) + off,
+                        len, kind, stream);
+  } else {
+    const size_t off = static_cast<size_t>(lb) * layer_bytes;
+    const size_t pitch = static_cast<size_t>(L) * layer_bytes;
+    const size_t width = static_cast<size_t>(lc) * layer_bytes;
+    if (pitch <= 0x7fffffffu) {
+      e = cudaMemcpy2DAsync(static_cast<uint8_t*>(dst) + off, pitch,
+                            static_cast<const uint8_t*>(src) + off, pitch, width, n, kind, stream);
+    } else {  // beyond the 2-D copy's pitch limit: one copy per block
+      e = cudaSuccess;
+      for (int32_t i = 0; i < n && e == cudaSuccess; ++i)
+        e = cudaMemcpyAsync(static_cast<uint8_t*>(dst) + i * pitch + off,
+                            static_cast<const uint8_t*>(src) + i * pitch + off, width, kind,
+                            stream);
+    }
   }
   if (e != cudaSuccess) return gc::cuda_fail(e, who);
   return GC_OK;
@@ -200,7 +207,7 @@ gc_status restore_impl(const char* who, gc_kv_pool* pool, const void* host_src,
   g_msg[0] = 0;
   if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
   if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "%s: n_blocks < 0", who);
-  if (flags & ~(GC_RESTORE_SRC_DEVICE | GC_RESTORE_VECTOR))
+  if (flags & ~(GC_RESTORE_SRC_DEVICE | GC_RESTORE_VECTOR | GC_RESTORE_LAYER_MAJOR))
     return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
   gc_status st = check_layers(who, pool, lb, lc);
   if (st != GC_OK) return st;
@@ -209,6 +216,7 @@ gc_status restore_impl(const char* who, gc_kv_pool* pool, const void* host_src,
   const size_t layer_bytes = 2 * gc::page_bytes(pool->cfg);
   const uint8_t* src = static_cast<const uint8_t*>(host_src);
   bool vector = (flags & GC_RESTORE_VECTOR) != 0;
+  const bool lm = (flags & GC_RESTORE_LAYER_MAJOR) != 0;
   if (!(flags & GC_RESTORE_SRC_DEVICE)) {
     cudaPointerAttributes attr;
     cudaError_t e = cudaPointerGetAttributes(&attr, host_src);
@@ -222,7 +230,7 @@ gc_status restore_impl(const char* who, gc_kv_pool* pool, const void* host_src,
       if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
         return fail(GC_ERR_INVALID_ARG, "%s: dev_staging not 16-byte aligned", who);
       st = copy_layers(who, dev_staging, host_src, n_blocks, pool->cfg.num_layers, lb, lc,
-                       layer_bytes, cudaMemcpyHostToDevice, stream);
+                       layer_bytes, lm, cudaMemcpyHostToDevice, stream);
       if (st != GC_OK) return st;
       src = static_cast<const uint8_t*>(dev_staging);
     } else {
@@ -236,8 +244,9 @@ gc_status restore_impl(const char* who, gc_kv_pool* pool, const void* host_src,
   if (reinterpret_cast<uintptr_t>(src) % 16)
     return fail(GC_ERR_INVALID_ARG, "%s: source not 16-byte aligned", who);
   uint8_t* stg = const_cast<uint8_t*>(src);  // read only when restoring
-  return vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, lb, lc, false, stream)
-                : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, lb, lc, false, stream);
+  return vector
+             ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, lb, lc, lm, false, stream)
+             : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, lb, lc, lm, false, stream);
 }
 
 gc_status save_impl(const char* who, gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
@@ -246,7 +255,7 @@ gc_status save_impl(const char* who, gc_kv_pool* pool, void* host_dst, const int
   g_msg[0] = 0;
   if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
   if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "%s: n_blocks < 0", who);
-  if (flags & ~(GC_SAVE_DST_DEVICE | GC_SAVE_VECTOR))
+  if (flags & ~(GC_SAVE_DST_DEVICE | GC_SAVE_VECTOR | GC_SAVE_LAYER_MAJOR))
     return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
   gc_status st = check_layers(who, pool, lb, lc);
   if (st != GC_OK) return st;
@@ -254,12 +263,14 @@ gc_status save_impl(const char* who, gc_kv_pool* pool, void* host_dst, const int
   if (!host_dst || !block_ids) return fail(GC_ERR_INVALID_ARG, "%s: host_dst / block_ids is NULL", who);
   const size_t layer_bytes = 2 * gc::page_bytes(pool->cfg);
   bool vector = (flags & GC_SAVE_VECTOR) != 0;
+  const bool lm = (flags & GC_SAVE_LAYER_MAJOR) != 0;
   if (flags & GC_SAVE_DST_DEVICE) {
     if (reinterpret_cast<uintptr_t>(host_dst) % 16)
       return fail(GC_ERR_INVALID_ARG, "%s: destination not 16-byte aligned", who);
     uint8_t* dst = static_cast<uint8_t*>(host_dst);
-    return vector ? gc::launch_restore_vector(pool, dst, block_ids, n_blocks, lb, lc, true, stream)
-                  : gc::launch_restore_bulk(pool, dst, block_ids, n_blocks, lb, lc, true, stream);
+    return vector
+               ? gc::launch_restore_vector(pool, dst, block_ids, n_blocks, lb, lc, lm, true, stream)
+               : gc::launch_restore_bulk(pool, dst, block_ids, n_blocks, lb, lc, lm, true, stream);
   }
   cudaPointerAttributes attr;
   cudaError_t e = cudaPointerGetAttributes(&attr, host_dst);
@@ -275,16 +286,101 @@ gc_status save_impl(const char* who, gc_kv_pool* pool, void* host_dst, const int
     if (reinterpret_cast<uintptr_t>(attr.devicePointer) % 16)
       return fail(GC_ERR_INVALID_ARG, "%s: host_dst not 16-byte aligned", who);
     return gc::launch_restore_vector(pool, static_cast<uint8_t*>(attr.devicePointer), block_ids,
-                                     n_blocks, lb, lc, true, stream);
+                                     n_blocks, lb, lc, lm, true, stream);
   }
   if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
     return fail(GC_ERR_INVALID_ARG, "%s: dev_staging not 16-byte aligned", who);
   uint8_t* stg = static_cast<uint8_t*>(dev_staging);
-  st = vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, lb, lc, true, stream)
-              : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, lb, lc, true, stream);
+  st = vector ? gc::launch_restore_vector(pool, stg, block_ids, n_blocks, lb, lc, lm, true, stream)
+              : gc::launch_restore_bulk(pool, stg, block_ids, n_blocks, lb, lc, lm, true, stream);
   if (st != GC_OK) return st;
   return copy_layers(who, host_dst, dev_staging, n_blocks, pool->cfg.num_layers, lb, lc,
-                     layer_bytes, cudaMemcpyDeviceToHost, stream);
+                     layer_bytes, lm, cudaMemcpyDeviceToHost, stream);
+}
+
+// The 8-bit image: the same movement as restore / save (pinned host via a
+// device staging copy, zero copy, or a device image), with the INT8 kernels.
+gc_status restore_q8_impl(const char* who, gc_kv_pool* pool, const void* src_img,
+                          const int32_t* block_ids, int32_t n_blocks, int32_t lb, int32_t lc,
+                          cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  g_msg[0] = 0;
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "%s: n_blocks < 0", who);
+  if (flags & ~(GC_RESTORE_SRC_DEVICE | GC_RESTORE_LAYER_MAJOR))
+    return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
+  gc_status st = check_layers(who, pool, lb, lc);
+  if (st != GC_OK) return st;
+  if (n_blocks == 0 || lc == 0) return GC_OK;
+  if (!src_img || !block_ids) return fail(GC_ERR_INVALID_ARG, "%s: image / block_ids is NULL", who);
+  const bool lm = (flags & GC_RESTORE_LAYER_MAJOR) != 0;
+  const size_t layer_bytes = 2 * gc::q8_chunk_bytes(pool->cfg);
+  const uint8_t* src = static_cast<const uint8_t*>(src_img);
+  if (!(flags & GC_RESTORE_SRC_DEVICE)) {
+    cudaPointerAttributes attr;
+    cudaError_t e = cudaPointerGetAttributes(&attr, src_img);
+    if (e != cudaSuccess || attr.type != cudaMemoryTypeHost) {
+      cudaGetLastError();
+      return fail(GC_ERR_INVALID_ARG,
+                  "%s: image must be pinned host memory unless GC_RESTORE_SRC_DEVICE is set", who);
+    }
+    if (dev_staging) {
+      if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
+        return fail(GC_ERR_INVALID_ARG, "%s: dev_staging not 16-byte aligned", who);
+      st = copy_layers(who, dev_staging, src_img, n_blocks, pool->cfg.num_layers, lb, lc,
+                       layer_bytes, lm, cudaMemcpyHostToDevice, stream);
+      if (st != GC_OK) return st;
+      src = static_cast<const uint8_t*>(dev_staging);
+    } else {
+      if (!attr.devicePointer) return fail(GC_ERR_INVALID_ARG, "%s: image has no device mapping", who);
+      src = static_cast<const uint8_t*>(attr.devicePointer);
+    }
+  }
+  if (reinterpret_cast<uintptr_t>(src) % 16)
+    return fail(GC_ERR_INVALID_ARG, "%s: image not 16-byte aligned", who);
+  return gc::launch_restore_q8(pool, src, block_ids, n_blocks, lb, lc, lm, stream);
+}
+
+gc_status save_q8_impl(const char* who, gc_kv_pool* pool, void* dst_img, const int32_t* block_ids,
+                       int32_t n_blocks, int32_t lb, int32_t lc, cudaStream_t stream,
+                       void* dev_staging, uint32_t flags) {
+  g_msg[0] = 0;
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "%s: n_blocks < 0", who);
+  if (flags & ~(GC_SAVE_DST_DEVICE | GC_SAVE_LAYER_MAJOR))
+    return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
+  gc_status st = check_layers(who, pool, lb, lc);
+  if (st != GC_OK) return st;
+  if (n_blocks == 0 || lc == 0) return GC_OK;
+  if (!dst_img || !block_ids) return fail(GC_ERR_INVALID_ARG, "%s: image / block_ids is NULL", who);
+  const bool lm = (flags & GC_SAVE_LAYER_MAJOR) != 0;
+  const size_t layer_bytes = 2 * gc::q8_chunk_bytes(pool->cfg);
+  if (flags & GC_SAVE_DST_DEVICE) {
+    if (reinterpret_cast<uintptr_t>(dst_img) % 16)
+      return fail(GC_ERR_INVALID_ARG, "%s: image not 16-byte aligned", who);
+    return gc::launch_save_q8(pool, static_cast<uint8_t*>(dst_img), block_ids, n_blocks, lb, lc,
+                              lm, stream);
+  }
+  cudaPointerAttributes attr;
+  cudaError_t e = cudaPointerGetAttributes(&attr, dst_img);
+  if (e != cudaSuccess || attr.type != cudaMemoryTypeHost) {
+    cudaGetLastError();
+    return fail(GC_ERR_INVALID_ARG,
+                "%s: image must be pinned host memory unless GC_SAVE_DST_DEVICE is set", who);
+  }
+  if (!dev_staging) {
+    if (!attr.devicePointer) return fail(GC_ERR_INVALID_ARG, "%s: image has no device mapping", who);
+    if (reinterpret_cast<uintptr_t>(attr.devicePointer) % 16)
+      return fail(GC_ERR_INVALID_ARG, "%s: image not 16-byte aligned", who);
+    return gc::launch_save_q8(pool, static_cast<uint8_t*>(attr.devicePointer), block_ids, n_blocks,
+                              lb, lc, lm, stream);
+  }
+  if (reinterpret_cast<uintptr_t>(dev_staging) % 16)
+    return fail(GC_ERR_INVALID_ARG, "%s: dev_staging not 16-byte aligned", who);
+  st = gc::launch_save_q8(pool, static_cast<uint8_t*>(dev_staging), block_ids, n_blocks, lb, lc,
+                          lm, stream);
+  if (st != GC_OK) return st;
+  return copy_layers(who, dst_img, dev_staging, n_blocks, pool->cfg.num_layers, lb, lc,
+                     layer_bytes, lm, cudaMemcpyDeviceToHost, stream);
 }
 
 }  // namespace
@@ -313,6 +409,25 @@ gc_status gc_kv_save_layers(gc_kv_pool* pool, void* host_dst, const int32_t* blo
                             cudaStream_t stream, void* dev_staging, uint32_t flags) {
   return save_impl("gc_kv_save_layers", pool, host_dst, block_ids, n_blocks, layer_begin,
                    layer_count, stream, dev_staging, flags);
+}
+
+size_t gc_kv_q8_chunk_bytes(const gc_pool_config* cfg) {
+  if (!pool_config_ok(cfg)) return 0;
+  return gc::q8_chunk_bytes(*cfg);
+}
+
+gc_status gc_kv_save_q8(gc_kv_pool* pool, void* dst, const int32_t* block_ids, int32_t n_blocks,
+                        int32_t layer_begin, int32_t layer_count, cudaStream_t stream,
+                        void* dev_staging, uint32_t flags) {
+  return save_q8_impl("gc_kv_save_q8", pool, dst, block_ids, n_blocks, layer_begin, layer_count,
+                      stream, dev_staging, flags);
+}
+
+gc_status gc_kv_restore_q8(gc_kv_pool* pool, const void* src, const int32_t* block_ids,
+                           int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
+                           cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  return restore_q8_impl("gc_kv_restore_q8", pool, src, block_ids, n_blocks, layer_begin,
+                         layer_count, stream, dev_staging, flags);
 }
 
 gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v_new,

@@ -37,15 +37,27 @@ __device__ __forceinline__ void record_error(int32_t* status, int32_t code) {
 
 // ---------------------------------------------------------------- launchers
 // Each returns GC_OK or a status with the message already set.
-// Page copies between a staging image [n_blocks][L][2][chunk] and the pool,
-// layers [layer0, layer0 + layers) only; gather = false restores
+// Page copies between a staging image [n_blocks][L][2][chunk] (or, with
+// layer_major, [L][n_blocks][2][chunk]) and the pool, layers
+// [layer0, layer0 + layers) only; gather = false restores
 // (staging -> pool), gather = true saves.
 gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging, const int32_t* block_ids,
-                              int32_t n_blocks, int32_t layer0, int32_t layers, bool gather,
-                              cudaStream_t stream);
+                              int32_t n_blocks, int32_t layer0, int32_t layers, bool layer_major,
+                              bool gather, cudaStream_t stream);
 gc_status launch_restore_vector(const gc_kv_pool* pool, uint8_t* staging,
                                 const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
-                                int32_t layers, bool gather, cudaStream_t stream);
+                                int32_t layers, bool layer_major, bool gather,
+                                cudaStream_t stream);
+// 8-bit cache tier (INT8 codes + one binary32 scale per (block, layer, plane,
+// kv head)); image chunk = scales padded to 16 bytes, then [Hkv][ps][d] int8.
+size_t q8_header_bytes(const gc_pool_config& c);
+size_t q8_chunk_bytes(const gc_pool_config& c);
+gc_status launch_save_q8(const gc_kv_pool* pool, uint8_t* image, const int32_t* block_ids,
+                         int32_t n_blocks, int32_t layer0, int32_t layers, bool layer_major,
+                         cudaStream_t stream);
+gc_status launch_restore_q8(const gc_kv_pool* pool, const uint8_t* image,
+                            const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
+                            int32_t layers, bool layer_major, cudaStream_t stream);
 gc_status launch_append(const gc_kv_pool* pool, const void* k_new, const void* v_new,
                         const int32_t* block_table, const int32_t* prefix_lens,
                         const int32_t* cu_new_lens, int32_t batch, int32_t max_blocks,

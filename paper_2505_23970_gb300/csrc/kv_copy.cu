@@ -8,7 +8,8 @@
 // staging image [n_blocks][L][2][chunk] goes to pool[l][kv][block_ids[i]],
 // for the layers l of one contiguous range [layer0, layer0 + layers) (all L
 // for a whole-request restore, one layer when restores are pipelined with
-// the layers' compute).
+// the layers' compute).  A layer-major image [L][n_blocks][2][chunk] is
+// also accepted (one contiguous span per layer range).
 // Save (Sec. 2.2, Fig. 2a step 1: a processed request's KV is saved to the
 // cache tier) is the same map run backwards: pool pages -> staging image.
 // The bulk kernel streams 16 KB pieces global -> shared -> global with
@@ -30,9 +31,17 @@ struct RestoreGeom {
   uint32_t pieces;          // ceil(C / kPiece)
   int32_t L, num_pages;     // layers of the pool and of the image; pages of the pool
   int32_t layer0, layers;   // the layer range moved
+  int32_t layer_major;      // image is [L][n_blocks][2][chunk] instead of [n_blocks][L][2][chunk]
   int32_t n_blocks;
   int32_t gather;           // 0: staging -> pool (restore), 1: pool -> staging (save)
 };
+
+// Index of chunk (block i, layer l, plane kv) in the staging image.
+__device__ __forceinline__ uint64_t image_chunk(const RestoreGeom& g, int64_t i, int l, int kv) {
+  const uint64_t il = g.layer_major ? static_cast<uint64_t>(l) * g.n_blocks + i
+                                    : static_cast<uint64_t>(i) * g.L + l;
+  return il * 2 + kv;
+}
 
 __device__ __forceinline__ bool piece_addr(const RestoreGeom& g, uint8_t* staging, uint8_t* pool,
                                            const int32_t* block_ids, int32_t* status, uint64_t u,
@@ -52,7 +61,7 @@ __device__ __forceinline__ bool piece_addr(const RestoreGeom& g, uint8_t* stagin
   const uint64_t off = static_cast<uint64_t>(piece) * kPiece;
   const uint64_t rem = g.chunk_bytes - off;
   *bytes = static_cast<uint32_t>(rem < kPiece ? rem : kPiece);
-  uint8_t* stg = staging + ((static_cast<uint64_t>(i) * g.L + l) * 2 + kv) * g.chunk_bytes + off;
+  uint8_t* stg = staging + image_chunk(g, i, l, kv) * g.chunk_bytes + off;
   uint8_t* pl = pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) * g.chunk_bytes + off;
   *s_out = g.gather ? pl : stg;
   *d_out = g.gather ? stg : pl;
@@ -150,7 +159,7 @@ __global__ void __launch_bounds__(256) restore_vector_kernel(uint4* __restrict__
           if (off == 0 && lr == 0 && kv == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
           continue;
         }
-        uint4* sw = staging + ((static_cast<uint64_t>(i) * g.L + l) * 2 + kv) * words_per_chunk + off;
+        uint4* sw = staging + image_chunk(g, i, l, kv) * words_per_chunk + off;
         uint4* pl = reinterpret_cast<uint4*>(
                         pool + ((static_cast<uint64_t>(l) * 2 + kv) * g.num_pages + id) *
                                    g.chunk_bytes) +
@@ -234,7 +243,8 @@ int ilog2(int x) {
 
 gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
                               const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
-                              int32_t layers, bool gather, cudaStream_t stream) {
+                              int32_t layers, bool layer_major, bool gather,
+                              cudaStream_t stream) {
   RestoreGeom g;
   g.gather = gather ? 1 : 0;
   g.chunk_bytes = page_bytes(pool->cfg);
@@ -244,6 +254,7 @@ gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
   g.n_blocks = n_blocks;
   g.layer0 = layer0;
   g.layers = layers;
+  g.layer_major = layer_major ? 1 : 0;
   const uint64_t units = static_cast<uint64_t>(n_blocks) * layers * 2 * g.pieces;
   uint64_t grid = static_cast<uint64_t>(pool->num_sms) * kBulkCtasPerSm;
   if (grid > units) grid = units;
@@ -261,7 +272,8 @@ gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
 
 gc_status launch_restore_vector(const gc_kv_pool* pool, uint8_t* staging,
                                 const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
-                                int32_t layers, bool gather, cudaStream_t stream) {
+                                int32_t layers, bool layer_major, bool gather,
+                                cudaStream_t stream) {
   RestoreGeom g;
   g.gather = gather ? 1 : 0;
   g.chunk_bytes = page_bytes(pool->cfg);
@@ -271,6 +283,7 @@ gc_status launch_restore_vector(const gc_kv_pool* pool, uint8_t* staging,
   g.n_blocks = n_blocks;
   g.layer0 = layer0;
   g.layers = layers;
+  g.layer_major = layer_major ? 1 : 0;
   const uint64_t words = static_cast<uint64_t>(n_blocks) * layers * 2 * (g.chunk_bytes / 16);
   uint64_t grid = (words + 256 * 4 - 1) / (256 * 4);
   const uint64_t cap = static_cast<uint64_t>(pool->num_sms) * 8;

@@ -161,7 +161,7 @@ class LayerStack:
     every byte is moved or computed by libgc."""
 
     def __init__(self, w: Workload, device: str = "cuda", fill=BF16_NAN, keep_outputs=False,
-                 staging: bool = True):
+                 staging: bool = True, layer_major: bool = True):
         import torch
         self.w, self.device = w, device
         self.pool = gcb.KVPool.create(w.L, w.Hkv, w.d, w.ps, w.num_pages, device=device)
@@ -173,7 +173,14 @@ class LayerStack:
         ids = w.prefix_blocks()
         self.n_blocks = int(ids.size)
         self.block_ids = _i32(ids, device)
-        self.host_src = bf16_tensor(w.host_src(), pin=True) if self.n_blocks else None
+        # the cached image, layer-major [L][n][2][Hkv][ps][d] by default so
+        # that each layer's slice is one contiguous host span
+        self.flags = gcb.GC_RESTORE_LAYER_MAJOR if layer_major else 0
+        img = w.host_src()
+        if layer_major and self.n_blocks:
+            img = np.ascontiguousarray(img.swapaxes(0, 1))
+        self.host_src = bf16_tensor(img, pin=True) if self.n_blocks else None
+        del img
         self.staging = (torch.empty_like(self.host_src, device=device)
                         if staging and self.n_blocks else None)
         k, v = w.kv_new()
@@ -185,15 +192,38 @@ class LayerStack:
         self.side = torch.cuda.Stream(device=device)
         self.events = [torch.cuda.Event() for _ in range(w.L)]
 
+    def use_q8(self):
+        """Switch the cache tier to the 8-bit image: quantise what the pool
+        holds now (after a restore) into a pinned layer-major INT8 image with
+        gc_kv_save_q8; later restores dequantise it with gc_kv_restore_q8."""
+        import torch
+        w = self.w
+        chunk = gcb.gc_kv_q8_chunk_bytes(self.pool.cfg)
+        shape = (w.L, self.n_blocks, 2, chunk)
+        self.q8_staging = torch.empty(shape, dtype=torch.uint8, device=self.device)
+        self.q8_host = torch.empty(shape, dtype=torch.uint8).pin_memory()
+        gcb.gc_kv_save_q8(self.pool.handle, self.q8_host, self.block_ids, self.n_blocks, 0, w.L,
+                          None, self.q8_staging, gcb.GC_SAVE_LAYER_MAJOR)
+        torch.cuda.synchronize()
+        self.q8 = True
+
+    q8 = False
+
     def restore_layer(self, l, stream):
-        if self.n_blocks:
+        if self.n_blocks and self.q8:
+            gcb.gc_kv_restore_q8(self.pool.handle, self.q8_host, self.block_ids, self.n_blocks,
+                                 l, 1, stream, self.q8_staging, gcb.GC_RESTORE_LAYER_MAJOR)
+        elif self.n_blocks:
             gcb.gc_kv_restore_layers(self.pool.handle, self.host_src, self.block_ids,
-                                     self.n_blocks, l, 1, stream, self.staging, 0)
+                                     self.n_blocks, l, 1, stream, self.staging, self.flags)
 
     def restore_all(self, stream):
-        if self.n_blocks:
+        if self.n_blocks and self.q8:
+            gcb.gc_kv_restore_q8(self.pool.handle, self.q8_host, self.block_ids, self.n_blocks,
+                                 0, self.w.L, stream, self.q8_staging, gcb.GC_RESTORE_LAYER_MAJOR)
+        elif self.n_blocks:
             gcb.gc_kv_restore(self.pool.handle, self.host_src, self.block_ids, self.n_blocks,
-                              stream, self.staging, 0)
+                              stream, self.staging, self.flags)
 
     def prefill_layer(self, l, stream):
         w = self.w

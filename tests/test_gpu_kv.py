@@ -6,7 +6,7 @@ import pytest
 import oracle
 from paper_2505_23970_gb300 import binding as gcb
 from paper_2505_23970_gb300 import workloads as wl
-from paper_2505_23970_gb300.harness import DeviceBatch, _i32
+from paper_2505_23970_gb300.harness import DeviceBatch, _i32, bf16_tensor
 
 pytestmark = pytest.mark.gpu
 
@@ -216,17 +216,24 @@ def _layered(seed=15):
 @pytest.mark.parametrize("mode,vector", [("staged", False), ("staged", True), ("device", False),
                                          ("zerocopy", False)])
 @pytest.mark.parametrize("lb,lc", [(0, 5), (1, 2), (4, 1)])
-def test_restore_layers_bit_exact(mode, vector, lb, lc):
+@pytest.mark.parametrize("layer_major", [False, True])
+def test_restore_layers_bit_exact(mode, vector, lb, lc, layer_major):
     """gc_kv_restore_layers writes exactly the chosen layers' pages of the
-    cached image and leaves every other layer untouched."""
+    cached image (block-major or layer-major) and leaves every other layer
+    untouched."""
     w = _layered()
     db = DeviceBatch(w)
+    if layer_major:  # the same image with its first two axes swapped (layout only)
+        img = np.ascontiguousarray(w.host_src().swapaxes(0, 1))
+        db.host_src = bf16_tensor(img, pin=True)
+        db.staging = db.staging.view(db.host_src.shape)
     if mode == "device":
         db.stage()
     src = db.staging if mode == "device" else db.host_src
     staging = db.staging if mode == "staged" else None
     flags = (gcb.GC_RESTORE_VECTOR if vector else 0) | (
-        gcb.GC_RESTORE_SRC_DEVICE if mode == "device" else 0)
+        gcb.GC_RESTORE_SRC_DEVICE if mode == "device" else 0) | (
+        gcb.GC_RESTORE_LAYER_MAJOR if layer_major else 0)
     gcb.gc_kv_restore_layers(db.pool.handle, src, db.block_ids, db.n_blocks, lb, lc, None,
                              staging, flags)
     assert db.check() == gcb.GC_OK
@@ -250,9 +257,10 @@ def test_restore_layers_one_call_per_layer_equals_whole_restore():
 
 @pytest.mark.parametrize("mode", ["staged", "device", "zerocopy"])
 @pytest.mark.parametrize("lb,lc", [(0, 5), (2, 3), (3, 1)])
-def test_save_layers_bit_exact(mode, lb, lc):
+@pytest.mark.parametrize("layer_major", [False, True])
+def test_save_layers_bit_exact(mode, lb, lc, layer_major):
     """gc_kv_save_layers writes the chosen layers' slices of the image (the
-    oracle's gather) and no other byte of it."""
+    oracle's gather; block-major or layer-major) and no other byte of it."""
     import torch
     w = _layered(17)
     db = DeviceBatch(w)
@@ -260,9 +268,10 @@ def test_save_layers_bit_exact(mode, lb, lc):
     db.append()
     ids = _used_pages(w)
     n = ids.size
-    shape = (n, w.L, 2, w.Hkv, w.ps, w.d)
+    shape = (w.L, n, 2, w.Hkv, w.ps, w.d) if layer_major else (n, w.L, 2, w.Hkv, w.ps, w.d)
     fill = int(np.uint16(0x1234).view(np.int16))
-    flags = gcb.GC_SAVE_DST_DEVICE if mode == "device" else 0
+    flags = (gcb.GC_SAVE_DST_DEVICE if mode == "device" else 0) | (
+        gcb.GC_SAVE_LAYER_MAJOR if layer_major else 0)
     if mode == "device":
         dst = torch.full(shape, fill, dtype=torch.int16, device="cuda")
     else:
@@ -271,7 +280,9 @@ def test_save_layers_bit_exact(mode, lb, lc):
     gcb.gc_kv_save_layers(db.pool.handle, dst, _i32(ids, "cuda"), n, lb, lc, None, staging, flags)
     assert db.check() == gcb.GC_OK
     got = dst.cpu().numpy().view(np.uint16)
-    want = np.full(shape, 0x1234, dtype=np.uint16)
+    if layer_major:
+        got = got.swapaxes(0, 1)
+    want = np.full((n, w.L, 2, w.Hkv, w.ps, w.d), 0x1234, dtype=np.uint16)
     want[:, lb:lb + lc] = oracle.kv_gather_blocks(oracle_pool(w), ids)[:, lb:lb + lc]
     assert np.array_equal(got, want)
     db.close()
@@ -292,3 +303,136 @@ def test_layer_range_checks():
     assert db.check() == gcb.GC_OK
     assert np.array_equal(db.pool_bits(), before)
     db.close()
+
+
+# ------------------------------------------------------ 8-bit cache tier
+def _q8_image_shape(w, n, layer_major):
+    import oracle as _o
+    chunk = _o.q8_chunk_bytes(w.Hkv, w.ps, w.d)
+    return (w.L, n, 2, chunk) if layer_major else (n, w.L, 2, chunk)
+
+
+@pytest.mark.parametrize("mode", ["staged", "device", "zerocopy"])
+@pytest.mark.parametrize("lb,lc", [(0, 5), (1, 3)])
+@pytest.mark.parametrize("layer_major", [False, True])
+def test_save_q8_bit_exact(mode, lb, lc, layer_major):
+    """INT8 codes and scales of the chosen layers equal the oracle's, bit for
+    bit (pages carry NaN in their unused tail slots); other chunks untouched."""
+    import torch
+    w = _layered(19)
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    ids = _used_pages(w)
+    n = ids.size
+    shape = _q8_image_shape(w, n, layer_major)
+    flags = (gcb.GC_SAVE_DST_DEVICE if mode == "device" else 0) | (
+        gcb.GC_SAVE_LAYER_MAJOR if layer_major else 0)
+    if mode == "device":
+        dst = torch.full(shape, 0xAB, dtype=torch.uint8, device="cuda")
+    else:
+        dst = torch.full(shape, 0xAB, dtype=torch.uint8).pin_memory()
+    staging = torch.empty(shape, dtype=torch.uint8, device="cuda") if mode == "staged" else None
+    gcb.gc_kv_save_q8(db.pool.handle, dst, _i32(ids, "cuda"), n, lb, lc, None, staging, flags)
+    assert db.check() == gcb.GC_OK
+    got = dst.cpu().numpy()
+    if layer_major:
+        got = got.swapaxes(0, 1)
+    want = np.full((n, w.L, 2, shape[-1]), 0xAB, dtype=np.uint8)
+    oracle.kv_save_q8(oracle_pool(w), ids, lb, lc, out=want)
+    assert np.array_equal(got, want)
+    db.close()
+
+
+@pytest.mark.parametrize("mode", ["staged", "device", "zerocopy"])
+@pytest.mark.parametrize("lb,lc", [(0, 5), (2, 1)])
+@pytest.mark.parametrize("layer_major", [False, True])
+def test_restore_q8_bit_exact(mode, lb, lc, layer_major):
+    """Dequantising an oracle-made INT8 image into the pool gives the
+    oracle's pool bit for bit; other layers and pages are untouched."""
+    import torch
+    w = _layered(20)
+    ids = w.prefix_blocks()
+    src_pool = w.empty_pool()
+    oracle.kv_restore(src_pool, w.host_src(), ids)
+    img = oracle.kv_save_q8(src_pool, ids)                    # [n][L][2][chunk]
+    want = w.empty_pool()
+    oracle.kv_restore_q8(want, img, ids, lb, lc)
+    db = DeviceBatch(w)
+    if layer_major:
+        img = np.ascontiguousarray(img.swapaxes(0, 1))
+    host = torch.from_numpy(img).pin_memory()
+    flags = gcb.GC_RESTORE_LAYER_MAJOR if layer_major else 0
+    if mode == "device":
+        src, staging, flags = host.cuda(), None, flags | gcb.GC_RESTORE_SRC_DEVICE
+    elif mode == "staged":
+        src, staging = host, torch.empty_like(host, device="cuda")
+    else:
+        src, staging = host, None
+    gcb.gc_kv_restore_q8(db.pool.handle, src, db.block_ids, db.n_blocks, lb, lc, None, staging,
+                         flags)
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(db.pool_bits(), want)
+    db.close()
+
+
+def test_q8_gpu_round_trip_and_bad_id():
+    """GPU save then GPU restore reproduces the oracle's round trip; a bad
+    block id is skipped and reported by both calls."""
+    import torch
+    w = _layered(21)
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    ids = _used_pages(w)
+    n = ids.size
+    img = torch.zeros(_q8_image_shape(w, n, False), dtype=torch.uint8, device="cuda")
+    gcb.gc_kv_save_q8(db.pool.handle, img, _i32(ids, "cuda"), n, 0, w.L, None, None,
+                      gcb.GC_SAVE_DST_DEVICE)
+    b = DeviceBatch(w, with_restore=False)
+    gcb.gc_kv_restore_q8(b.pool.handle, img, _i32(ids, "cuda"), n, 0, w.L, None, None,
+                         gcb.GC_RESTORE_SRC_DEVICE)
+    assert db.check() == gcb.GC_OK and b.check() == gcb.GC_OK
+    ref = w.empty_pool()
+    oracle.kv_restore_q8(ref, oracle.kv_save_q8(oracle_pool(w), ids), ids)
+    assert np.array_equal(b.pool_bits(), ref)
+    bad = ids.copy()
+    bad[1] = w.num_pages
+    gcb.gc_kv_save_q8(db.pool.handle, img, _i32(bad, "cuda"), n, 0, w.L, None, None,
+                      gcb.GC_SAVE_DST_DEVICE)
+    assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
+    gcb.gc_kv_restore_q8(b.pool.handle, img, _i32(bad, "cuda"), n, 0, w.L, None, None,
+                         gcb.GC_RESTORE_SRC_DEVICE)
+    assert b.check() == gcb.GC_ERR_OUT_OF_RANGE
+    db.close()
+    b.close()
+
+
+def test_q8_subnormal_and_large_groups_match_oracle():
+    """Groups of tiny (subnormal) values, where 127/amax overflows, and of
+    large values take the general path and still match the oracle bit for bit."""
+    import torch
+    w = _layered(22)
+    src = wl.bf16_bits_to_f32(w.host_src())
+    src[0::3] *= 2.0 ** -130          # subnormal magnitudes in bf16
+    src[1::3] *= 2.0 ** 100
+    w._cache["src"] = wl.f32_to_bf16_bits(src)
+    db = DeviceBatch(w)
+    db.restore()
+    ids = w.prefix_blocks()
+    n = ids.size
+    img = torch.zeros(_q8_image_shape(w, n, False), dtype=torch.uint8, device="cuda")
+    gcb.gc_kv_save_q8(db.pool.handle, img, db.block_ids, n, 0, w.L, None, None,
+                      gcb.GC_SAVE_DST_DEVICE)
+    assert db.check() == gcb.GC_OK
+    want = oracle.kv_save_q8(oracle_pool(w, append=False), ids)
+    assert np.array_equal(img.cpu().numpy(), want)
+    b = DeviceBatch(w, with_restore=False)
+    gcb.gc_kv_restore_q8(b.pool.handle, img, db.block_ids, n, 0, w.L, None, None,
+                         gcb.GC_RESTORE_SRC_DEVICE)
+    assert b.check() == gcb.GC_OK
+    ref = w.empty_pool()
+    oracle.kv_restore_q8(ref, want, ids)
+    assert np.array_equal(b.pool_bits(), ref)
+    db.close()
+    b.close()

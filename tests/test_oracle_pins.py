@@ -346,3 +346,114 @@ def test_thread_count_does_not_change_results():
     pool = _fill_pool(w)
     args = (w.q(), pool, 0, w.block_table, w.prefix_lens, w.cu_new_lens, w.scale)
     assert np.array_equal(oracle.prefix_attn(*args, nthreads=1), oracle.prefix_attn(*args, nthreads=5))
+
+
+# ------------------------------------------------------ 8-bit cache tier
+def _q8_pool(groups, Hkv=1, ps=1):
+    """Pool [1][2][NP][Hkv][ps][d] holding `groups` (one per (plane, page, head))."""
+    g = np.asarray(groups, dtype=np.float32)
+    d = g.shape[-1] // ps
+    n = g.shape[0] // (2 * Hkv)
+    pool = wl.f32_to_bf16_bits(g).reshape(2, n, Hkv, ps, d)  # every value here is exact in bf16
+    return np.ascontiguousarray(pool.reshape(1, 2, n, Hkv, ps, d))
+
+
+def test_q8_codes_of_worked_groups():
+    """amax = 127/64 makes 127/amax = 64 and s = 1/64 exactly, so each code is
+    round_half_even(64 x) by hand, ties included (2.5 -> 2, 3.5 -> 4, -0.5 -> 0,
+    1.5 -> 2; half-away-from-zero would give 3, 4, -1, 2).  amax = 2 makes
+    127/amax = 63.5, so codes are round_half_even(63.5 x) (63.5 -> 64, -63.5 -> -64)."""
+    k = np.array([127, 2.5, 3.5, -0.5, 1.5, 0, -127, 64, -3, 10.5, 11.5, 100, -100.5, 1, -1, 0.5])
+    a = k / 64.0
+    want_a = [127, 2, 4, 0, 2, 0, -127, 64, -3, 10, 12, 100, -100, 1, -1, 0]
+    b = np.array([1.0, -0.5, 0.25, 0.125, 2.0, -2.0, 0.0, 1.5, -1.25, 0.75, 0.0625, -0.0625,
+                  0.296875, 0.5, -1.0, 0.109375])
+    want_b = [64, -32, 16, 8, 127, -127, 0, 95, -79, 48, 4, -4, 19, 32, -64, 7]
+    pool = _q8_pool([a, b])  # K plane: group a, V plane: group b
+    img = oracle.kv_save_q8(pool, [0])
+    scales, codes = oracle.q8_split(img, 1, 1, 16)
+    assert codes[0, 0, 0, 0, 0].tolist() == want_a
+    assert codes[0, 0, 1, 0, 0].tolist() == want_b
+    assert scales[0, 0, 0, 0] == np.float32(1 / 64)
+    assert abs(float(scales[0, 0, 1, 0]) * 127 - 2.0) <= 2.0 * 2.0 ** -23
+    out = np.zeros_like(pool)
+    oracle.kv_restore_q8(out, img, [0])
+    back = wl.bf16_bits_to_f32(out[0, 0, 0, 0, 0])
+    assert np.array_equal(back, np.asarray(want_a, np.float32) / 64)  # c/64 is exact in bf16
+
+
+def _random_q8_pool(seed, L=2, NP=5, Hkv=3, ps=4, d=16, scale=1.0):
+    rng = np.random.default_rng(seed)
+    x = (rng.standard_normal((L, 2, NP, Hkv, ps, d)) * scale).astype(np.float32)
+    return wl.f32_to_bf16_bits(x)
+
+
+def test_q8_round_trip_within_half_step():
+    """Every restored value is within half a quantisation step of the
+    original, plus the final bf16 rounding; each group's largest |x| maps to
+    +-127; every code is in [-127, 127]."""
+    pool = _random_q8_pool(1)
+    ids = np.array([4, 0, 2], np.int32)
+    img = oracle.kv_save_q8(pool, ids)
+    L, _, NP, Hkv, ps, d = pool.shape
+    scales, codes = oracle.q8_split(img, Hkv, ps, d)
+    assert codes.min() >= -127 and codes.max() <= 127
+    out = np.zeros_like(pool)
+    oracle.kv_restore_q8(out, img, ids)
+    x = wl.bf16_bits_to_f32(pool[:, :, ids]).astype(np.float64)      # [L][2][n][Hkv][ps][d]
+    y = wl.bf16_bits_to_f32(out[:, :, ids]).astype(np.float64)
+    s = scales.transpose(1, 2, 0, 3)[..., None, None].astype(np.float64)  # [L][2][n][Hkv]
+    assert np.all(np.abs(y - x) <= s / 2 * (1 + 2.0 ** -20) + np.abs(y) * 2.0 ** -8)
+    amax = np.abs(x).max(axis=(-1, -2))
+    cmax = np.abs(codes.transpose(1, 2, 0, 3, 4, 5).astype(np.int64)).max(axis=(-1, -2))
+    assert np.all(cmax == 127) and np.all(amax > 0)
+    untouched = np.setdiff1d(np.arange(NP), ids)
+    assert np.all(out[:, :, untouched] == 0)
+
+
+def test_q8_sign_and_power_of_two_scaling():
+    """Negating a page negates its codes; multiplying it by 4 (exact in bf16)
+    keeps the codes and multiplies the scales by 4."""
+    pool = _random_q8_pool(2)
+    ids = np.arange(pool.shape[2], dtype=np.int32)
+    img = oracle.kv_save_q8(pool, ids)
+    neg = pool ^ np.uint16(0x8000)
+    x4 = wl.f32_to_bf16_bits(wl.bf16_bits_to_f32(pool) * 4)
+    s0, c0 = oracle.q8_split(img, *pool.shape[3:])
+    s1, c1 = oracle.q8_split(oracle.kv_save_q8(neg, ids), *pool.shape[3:])
+    s4, c4 = oracle.q8_split(oracle.kv_save_q8(x4, ids), *pool.shape[3:])
+    assert np.array_equal(c1, -c0) and np.array_equal(s1, s0)
+    assert np.array_equal(c4, c0) and np.array_equal(s4, s0 * 4)
+
+
+def test_q8_zero_nan_and_infinite_values():
+    """An all-zero group has scale 0 and restores to +0; NaN codes to 0 and
+    infinities saturate, neither counting towards amax."""
+    zeros = np.zeros(16)
+    special = np.array([np.nan, np.inf, -np.inf, 1.0, -0.5] + [0.25] * 11)
+    pool = _q8_pool([zeros, special])
+    img = oracle.kv_save_q8(pool, [0])
+    scales, codes = oracle.q8_split(img, 1, 1, 16)
+    assert scales[0, 0, 0, 0] == 0 and np.all(codes[0, 0, 0] == 0)
+    assert scales[0, 0, 1, 0] == np.float32(1.0) / np.float32(127)
+    assert codes[0, 0, 1, 0, 0, :5].tolist() == [0, 127, -127, 127, -64]
+    out = np.full_like(pool, 0x7FC0)
+    oracle.kv_restore_q8(out, img, [0])
+    assert np.all(out[0, 0, 0] == 0)
+
+
+def test_q8_image_layout_and_layer_range():
+    """Hkv = 3: 12 scale bytes, 4 zero bytes, then the codes; a layer range
+    writes only its chunks and restores only its layers."""
+    pool = _random_q8_pool(3, L=4, NP=3, Hkv=3, ps=2, d=8)
+    assert oracle.q8_chunk_bytes(3, 2, 8) == 16 + 3 * 2 * 8
+    ids = np.array([2, 1], np.int32)
+    img = oracle.kv_save_q8(pool, ids, layer_begin=1, layer_count=2)
+    assert np.all(img[:, [0, 3]] == 0) and np.all(img[:, 1:3, :, 12:16] == 0)
+    full = oracle.kv_save_q8(pool, ids)
+    assert np.array_equal(img[:, 1:3], full[:, 1:3])
+    out = np.zeros_like(pool)
+    oracle.kv_restore_q8(out, full, ids, layer_begin=2, layer_count=1)
+    ref = np.zeros_like(pool)
+    oracle.kv_restore_q8(ref, full, ids)
+    assert np.array_equal(out[2], ref[2]) and np.all(out[[0, 1, 3]] == 0)
