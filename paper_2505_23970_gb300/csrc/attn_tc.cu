@@ -17,14 +17,14 @@
 //      warp 0        TMA producer: Q tiles (3-D map over [T_new][Hq][d]) and
 //                    K/V tiles page by page (2-D map over the pool rows);
 //                    zeroes V rows past the end of the sequence.
-//      warp 1        TMEM owner; lane 0 is the MMA issuer:
+//      warp 1        TMEM owner; lane 0 issues Q tile 0's MMAs, lane 0 of
+//      warp 2        issues Q tile 1's:
 //                      S_i = Q_i K^T   (SS, both operands K-major, fp32 in TMEM)
 //                      O_i += P_i V    (TS: P_i read from TMEM, V MN-major)
-//                    It polls the readiness of every pending MMA of both Q
-//                    tiles and issues each whole MMA as soon as its inputs
-//                    are ready, so the tensor pipe serialises the two tiles'
-//                    S -> softmax -> PV chains into a staggered schedule in
-//                    which one tile's softmax overlaps the other's MMAs.
+//                    Each issuer waits for its tile's inputs in chain order;
+//                    with one issuer per tile the tensor pipe interleaves the
+//                    two tiles' S -> softmax -> PV chains, so one tile's
+//                    softmax overlaps the other's MMAs.
 //      warps 4-7     softmax of Q tile 0; warps 8-11 softmax of Q tile 1.
 //    Warps 0-3 give registers to the softmax warpgroups (setmaxnreg).
 //                    One thread per row: S row from TMEM, causal mask, online
@@ -95,9 +95,9 @@ struct Barriers {
   int abort_flag;
 };
 
-// Consumers of the work-item ring: the MMA issuer thread and one elected
-// thread per softmax warp.
-constexpr int kItemConsumers = 1 + 2 * kTileM / 32;
+// Consumers of the work-item ring: the two MMA issuer threads and one
+// elected thread per softmax warp.
+constexpr int kItemConsumers = 2 + 2 * kTileM / 32;
 
 // A work item and the quantities every role derives from it.
 struct Item {
@@ -211,26 +211,28 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
     }
     armed_q = q_count & 1;
     ++q_count;
-    // ---- K/V tiles, page by page
+    // ---- K/V tiles, page by page.  The copies of a tile are issued by
+    // several lanes at once (lane = page * halves + half): one thread issuing
+    // every box of a 16-row-page tile could not keep up with the MMAs.
     const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
+    const int pg = lane / C::kHalves, hh = lane % C::kHalves;
     for (int j = 0; ok && j < w.nt; ++j) {
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
       const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
       const int blk0 = key0 >> geo.ps_shift;
-      int pages[kTileN / 16];
-      int good = 0;
-#pragma unroll
-      for (int pg = 0; pg < kTileN / 16; ++pg) {
-        int page = -1;
-        if (pg < npages && blk0 + pg < geo.max_blocks) page = __ldg(block_table + bt_row + blk0 + pg);
-        if (pg < npages && (page < 0 || page >= geo.num_pages)) {
-          if (lane == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
+      // lane p (< npages) looks up page p of the tile
+      int page = -1;
+      if (lane < npages) {
+        if (blk0 + lane < geo.max_blocks) page = __ldg(block_table + bt_row + blk0 + lane);
+        if (page < 0 || page >= geo.num_pages) {
+          record_error(status, GC_ERR_OUT_OF_RANGE);
           page = -1;
         }
-        pages[pg] = page;
-        good += page >= 0;
       }
+      const int good = __popc(__ballot_sync(0xffffffffu, page >= 0));
+      const int my_page = __shfl_sync(0xffffffffu, page, pg < 32 ? pg : 0);
+      const bool issues = pg < kTileN / 16 && my_page >= 0;
 #pragma unroll 1
       for (int kv = 0; kv < 2; ++kv) {
         const int slot = kv_count % C::kStages;
@@ -239,17 +241,13 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
         uint8_t* dst = smem_kv + slot * C::kTileBytes;
         const bool fix = kv == 1 && nkeys < kTileN;
         uint64_t* full = fix ? &bar.vfix : &bar.kv_full[slot];
-        if (lane == 0) {
+        if (lane == 0)
           mbar_arrive_expect_tx(full, static_cast<uint32_t>(good) * box_bytes * C::kHalves);
+        __syncwarp();
+        if (issues) {
           const int plane_row = (geo.layer * 2 + kv) * geo.num_pages;
-#pragma unroll
-          for (int pg = 0; pg < kTileN / 16; ++pg) {
-            if (pages[pg] < 0) continue;
-            const int row = (((plane_row + pages[pg]) * geo.Hkv + w.g) << geo.ps_shift);
-#pragma unroll
-            for (int h = 0; h < C::kHalves; ++h)
-              tma_load_2d(dst + h * C::kHalfBytes + pg * box_bytes, map_kv, full, h * 64, row);
-          }
+          const int row = (((plane_row + my_page) * geo.Hkv + w.g) << geo.ps_shift);
+          tma_load_2d(dst + hh * C::kHalfBytes + pg * box_bytes, map_kv, full, hh * 64, row);
         }
         if (fix) {
           // V rows past the end of the sequence must be zero, not stale or NaN:
@@ -287,18 +285,24 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
   }
 }
 
+// The MMA issuer of Q tile i (one thread).  Each tile's products are a
+// strict chain (P_i aliases S_i, so S_i(j+1) waits for PV_i(j) to complete),
+// so the issuer waits for each input in order; the two tiles have separate
+// issuer threads, so one tile's waits never delay the other tile's MMAs and
+// the tensor pipe interleaves the two chains.
 template <int D>
-__device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uint32_t tmem,
+__device__ void mma_issuer(int i, uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uint32_t tmem,
                            const int* item_start, int total_items, const Geom& geo,
                            const int32_t* __restrict__ prefix_lens,
                            const int32_t* __restrict__ new_lens,
                            const int32_t* __restrict__ cu_new_lens) {
   using C = Cfg<D>;
   volatile int* abortp = &bar.abort_flag;
-  uint32_t q_count = 0, kv_count = 0;
-  uint32_t p_cons[2] = {0, 0}, pv_issued[2] = {0, 0}, pv_acked[2] = {0, 0};
+  uint32_t q_count = 0, kv_count = 0, s_issued = 0, pv_issued = 0;
   bool ok = true;
-  const uint32_t q_base = smem_addr(smem_q), kv_smem = smem_addr(smem_kv);
+  const uint32_t q_addr = smem_addr(smem_q) + i * C::kTileBytes, kv_smem = smem_addr(smem_kv);
+  const uint32_t col_s = i ? C::kColS1 : C::kColS0;
+  const uint32_t col_o = i ? C::kColO1 : C::kColO0;
 
   for (uint32_t k = 0; ok; ++k) {
     const int it = read_item(bar, k, abortp, ok);
@@ -307,91 +311,46 @@ __device__ void mma_issuer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, uin
     if (it < 0) break;
     Item w;
     decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
-    ok = mbar_wait(&bar.q_full, q_count & 1, abortp);
-    ++q_count;
-    if (!ok) break;
-    tc_fence_after();
     // K_j sits in ring use kv_base + 2j, V_j in use kv_base + 2j + 1
     const uint32_t kv_base = kv_count;
-    int s_next[2] = {0, 0}, pv_next[2] = {0, 0};
-    int kfront = 0, vfront = 0;
-    bool q_released = false;
-    long long last = clock64();
-    while (true) {
-      bool progressed = false;
+    kv_count += 2 * w.nt;
+    const uint32_t q_par = q_count & 1;
+    ++q_count;
+    if (!w.valid[i]) continue;
+    ok = mbar_wait(&bar.q_full, q_par, abortp);
+    if (!ok) break;
+    tc_fence_after();
+    for (int j = 0; j < w.nt_i[i]; ++j) {
+      // S_i = Q_i K_j^T once K_j is in and PV_i(j-1) has finished reading P_i
+      const uint32_t ku = kv_base + 2 * j;
+      ok = mbar_wait(&bar.kv_full[ku % C::kStages], (ku / C::kStages) & 1, abortp);
+      if (ok && pv_issued > 0) ok = mbar_wait(&bar.pv_done[i], (pv_issued - 1) & 1, abortp);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t k_addr = kv_smem + (ku % C::kStages) * C::kTileBytes;
 #pragma unroll
-      for (int i = 0; i < 2; ++i) {
-        const uint32_t col_s = i ? C::kColS1 : C::kColS0;
-        const uint32_t col_o = i ? C::kColO1 : C::kColO0;
-        // O_i += P_i V_j once the softmax has written P_i(j)
-        int j = pv_next[i];
-        if (j < s_next[i]) {
-          const uint32_t use = kv_base + 2 * j + 1;
-          if (mbar_test(&bar.p_full[i], p_cons[i] & 1) &&
-              mbar_test(&bar.kv_full[use % C::kStages], (use / C::kStages) & 1)) {
-            tc_fence_after();
-            const uint32_t v_addr = kv_smem + (use % C::kStages) * C::kTileBytes;
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * C::kHalfBytes + (kk & 3) * 32;
+        mma_ss(tmem + col_s, sdesc_sw128(q_addr + off, 16, 1024),
+               sdesc_sw128(k_addr + off, 16, 1024), C::kIdescQK, kk > 0);
+      }
+      mma_commit(&bar.s_full[i]);
+      ++s_issued;
+      // O_i += P_i V_j once the softmax has written P_i(j) and V_j is in
+      const uint32_t vu = ku + 1;
+      ok = mbar_wait(&bar.p_full[i], (s_issued - 1) & 1, abortp);
+      if (ok) ok = mbar_wait(&bar.kv_full[vu % C::kStages], (vu / C::kStages) & 1, abortp);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t v_addr = kv_smem + (vu % C::kStages) * C::kTileBytes;
 #pragma unroll
-            for (int kk = 0; kk < kTileN / 16; ++kk)
-              mma_ts(tmem + col_o, tmem + col_s + kk * 8,
-                     sdesc_sw128(v_addr + kk * 16 * 128, C::kHalfBytes, 1024), C::kIdescPV,
-                     (j > 0 || kk > 0) ? 1u : 0u);
-            mma_commit(&bar.pv_done[i]);
-            ++pv_issued[i];
-            ++p_cons[i];
-            ++pv_next[i];
-            progressed = true;
-          }
-        }
-        // S_i = Q_i K_j^T once PV_i(j-1) has finished reading P_i (it aliases S_i)
-        j = s_next[i];
-        if (j < w.nt_i[i] && pv_next[i] == j) {
-          const uint32_t use = kv_base + 2 * j;
-          const bool alias_free = pv_acked[i] == pv_issued[i] ||
-                                  mbar_test(&bar.pv_done[i], (pv_issued[i] - 1) & 1);
-          if (alias_free && mbar_test(&bar.kv_full[use % C::kStages], (use / C::kStages) & 1)) {
-            pv_acked[i] = pv_issued[i];
-            tc_fence_after();
-            const uint32_t k_addr = kv_smem + (use % C::kStages) * C::kTileBytes;
-            const uint32_t q_addr = q_base + i * C::kTileBytes;
-#pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * C::kHalfBytes + (kk & 3) * 32;
-              mma_ss(tmem + col_s, sdesc_sw128(q_addr + off, 16, 1024),
-                     sdesc_sw128(k_addr + off, 16, 1024), C::kIdescQK, kk > 0);
-            }
-            mma_commit(&bar.s_full[i]);
-            ++s_next[i];
-            progressed = true;
-          }
-        }
-      }
-      // release ring slots whose last reader has been issued (the commit
-      // arrives once those MMAs complete), and the Q tiles after their last S
-      while (kfront < w.nt && (s_next[0] > kfront || kfront >= w.nt_i[0]) &&
-             (s_next[1] > kfront || kfront >= w.nt_i[1])) {
-        mma_commit(&bar.kv_empty[(kv_base + 2 * kfront) % C::kStages]);
-        ++kfront;
-      }
-      while (vfront < w.nt && (pv_next[0] > vfront || vfront >= w.nt_i[0]) &&
-             (pv_next[1] > vfront || vfront >= w.nt_i[1])) {
-        mma_commit(&bar.kv_empty[(kv_base + 2 * vfront + 1) % C::kStages]);
-        ++vfront;
-      }
-      if (!q_released && s_next[0] == w.nt_i[0] && s_next[1] == w.nt_i[1]) {
-        mma_commit(&bar.q_empty);
-        q_released = true;
-      }
-      if (kfront == w.nt && vfront == w.nt) break;
-      if (progressed) {
-        last = clock64();
-      } else if (*abortp || clock64() - last > kWaitCycles) {
-        *abortp = 1;
-        ok = false;
-        break;
-      }
+      for (int kk = 0; kk < kTileN / 16; ++kk)
+        mma_ts(tmem + col_o, tmem + col_s + kk * 8,
+               sdesc_sw128(v_addr + kk * 16 * 128, C::kHalfBytes, 1024), C::kIdescPV,
+               (j > 0 || kk > 0) ? 1u : 0u);
+      mma_commit(&bar.pv_done[i]);
+      ++pv_issued;
     }
-    kv_count = kv_base + 2 * w.nt;
   }
   // wait for every MMA this thread issued before TMEM is released
   mma_commit(&bar.drain);
@@ -456,11 +415,15 @@ __device__ __forceinline__ void rescale_o(uint32_t tO, float alpha) {
   }
 }
 
-// Make this thread's P writes visible to the MMA issuer and arrive.
+// Make this warp's P writes visible to the MMA issuer: every thread waits
+// for its TMEM stores and fences, then one elected thread arrives for the
+// warp (one arrival per warp: per-thread arrivals on a single barrier are
+// serialised and cost more than the softmax itself).
 __device__ __forceinline__ void publish_p(uint64_t* bar) {
   tmem_wait_st();
   tc_fence_before();
-  mbar_arrive(bar);
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
 }
 
 template <int D, int i>
@@ -477,7 +440,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
   const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
   const uint32_t tS = lane_addr + (i ? C::kColS1 : C::kColS0);
   const uint32_t tO = lane_addr + (i ? C::kColO1 : C::kColO0);
-  uint32_t s_count = 0, pv_total = 0;
+  uint32_t s_count = 0, pv_total = 0, kv_count = 0;
   bool ok = true;
 
   for (uint32_t k = 0; ok; ++k) {
@@ -488,7 +451,19 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
     if (it < 0) break;
     Item w;
     decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
+    // K_j sits in ring use kv_base + 2j, V_j in use kv_base + 2j + 1
+    const uint32_t kv_base = kv_count;
+    kv_count += 2 * w.nt;
     if (!w.valid[i]) continue;
+    // This tile releases the ring slots (and the Q tiles) once the MMAs that
+    // read them are known complete; for K/V tiles (or Q) the other tile does
+    // not use, it arrives on that tile's behalf too.
+    const bool rel = threadIdx.x == kTileM * (1 + i);
+    const int nt_o = w.valid[1 - i] ? w.nt_i[1 - i] : 0;
+    auto release = [&](int j, int kv) {
+      const uint32_t use = kv_base + 2 * j + kv;
+      mbar_arrive_cnt(&bar.kv_empty[use % C::kStages], j < nt_o ? 1u : 2u);
+    };
     const int tok = w.tok0[i] + r / geo.G;
     const bool row_valid = tok < w.n;
     const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
@@ -497,6 +472,13 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
       ok = mbar_wait(&bar.s_full[i], s_count & 1, abortp);
       ++s_count;
       if (!ok) break;
+      if (rel) {
+        // S_i(j) is complete: K_j is done with for this tile; and S_i(j) was
+        // issued after PV_i(j-1) completed, so V_{j-1} is too
+        release(j, 0);
+        if (j > 0) release(j - 1, 1);
+        if (j == w.nt_i[i] - 1) mbar_arrive_cnt(&bar.q_empty, w.valid[1 - i] ? 1u : 2u);
+      }
       tc_fence_after();
       uint32_t sr[4][32];
 #pragma unroll
@@ -538,6 +520,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
     pv_total += w.nt_i[i];
     ok = mbar_wait(&bar.pv_done[i], (pv_total - 1) & 1, abortp);
     if (!ok) break;
+    if (rel) release(w.nt_i[i] - 1, 1);
     tc_fence_after();
     const float inv_l = 1.f / l;
     const int h = w.g * geo.G + r % geo.G;
@@ -585,16 +568,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(&bar.q_full, 1);
-    mbar_init(&bar.q_empty, 1);
+    mbar_init(&bar.q_empty, 2);
     mbar_init(&bar.vfix, 1);
-    mbar_init(&bar.drain, 1);
+    mbar_init(&bar.drain, 2);
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(&bar.kv_full[s], 1);
-      mbar_init(&bar.kv_empty[s], 1);
+      mbar_init(&bar.kv_empty[s], 2);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bar.s_full[i], 1);
-      mbar_init(&bar.p_full[i], kTileM);
+      mbar_init(&bar.p_full[i], kTileM / 32);
       mbar_init(&bar.pv_done[i], 1);
     }
     for (int s = 0; s < 2; ++s) {
@@ -661,10 +644,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
       producer<D>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv,
                   block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
-    } else if (warp == 1) {
+    } else if (warp == 1 || warp == 2) {
       if (lane == 0)
-        mma_issuer<D>(smem_q, smem_kv, bar, tmem, item_start, total_items, geo, prefix_lens,
-                      new_lens, cu_new_lens);
+        mma_issuer<D>(warp - 1, smem_q, smem_kv, bar, tmem, item_start, total_items, geo,
+                      prefix_lens, new_lens, cu_new_lens);
       __syncwarp();
     }
   } else {
