@@ -93,6 +93,7 @@ struct Barriers {
   int item_slot[2];
   uint32_t tmem_base;
   int abort_flag;
+  int p0_steps;  // P tiles tile 0's softmax has published so far (pacing hint)
 };
 
 // Consumers of the work-item ring: the two MMA issuer threads and one
@@ -216,20 +217,29 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
     // every box of a 16-row-page tile could not keep up with the MMAs.
     const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
     const int pg = lane / C::kHalves, hh = lane % C::kHalves;
-    for (int j = 0; ok && j < w.nt; ++j) {
+    // lane p (< pages of the tile) looks up page p of a tile; tile j+1's
+    // lookup is issued before tile j's copies so its latency is hidden
+    auto lookup = [&](int j) -> int {
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
       const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
       const int blk0 = key0 >> geo.ps_shift;
-      // lane p (< npages) looks up page p of the tile
-      int page = -1;
-      if (lane < npages) {
-        if (blk0 + lane < geo.max_blocks) page = __ldg(block_table + bt_row + blk0 + lane);
-        if (page < 0 || page >= geo.num_pages) {
-          record_error(status, GC_ERR_OUT_OF_RANGE);
-          page = -1;
-        }
+      int pg_id = -2;  // -2: no page in this lane
+      if (j < w.nt && lane < npages)
+        pg_id = blk0 + lane < geo.max_blocks ? __ldg(block_table + bt_row + blk0 + lane) : -1;
+      return pg_id;
+    };
+    int page_next = lookup(0);
+    for (int j = 0; ok && j < w.nt; ++j) {
+      const int key0 = j * kTileN;
+      const int nkeys = min(kTileN, w.T - key0);
+      int page = page_next;
+      page_next = lookup(j + 1);
+      if (page != -2 && (page < 0 || page >= geo.num_pages)) {
+        record_error(status, GC_ERR_OUT_OF_RANGE);
+        page = -1;
       }
+      if (page == -2) page = -1;
       const int good = __popc(__ballot_sync(0xffffffffu, page >= 0));
       const int my_page = __shfl_sync(0xffffffffu, page, pg < 32 ? pg : 0);
       const bool issues = pg < kTileN / 16 && my_page >= 0;
@@ -304,6 +314,7 @@ __device__ void mma_issuer(int i, uint8_t* smem_q, uint8_t* smem_kv, Barriers& b
   const uint32_t col_s = i ? C::kColS1 : C::kColS0;
   const uint32_t col_o = i ? C::kColO1 : C::kColO0;
 
+  int p0_base = 0;  // tile-0 steps of earlier items
   for (uint32_t k = 0; ok; ++k) {
     const int it = read_item(bar, k, abortp, ok);
     if (!ok) break;
@@ -314,6 +325,8 @@ __device__ void mma_issuer(int i, uint8_t* smem_q, uint8_t* smem_kv, Barriers& b
     // K_j sits in ring use kv_base + 2j, V_j in use kv_base + 2j + 1
     const uint32_t kv_base = kv_count;
     kv_count += 2 * w.nt;
+    const int p0_item = p0_base;
+    p0_base += w.nt_i[0];
     const uint32_t q_par = q_count & 1;
     ++q_count;
     if (!w.valid[i]) continue;
@@ -325,6 +338,20 @@ __device__ void mma_issuer(int i, uint8_t* smem_q, uint8_t* smem_kv, Barriers& b
       const uint32_t ku = kv_base + 2 * j;
       ok = mbar_wait(&bar.kv_full[ku % C::kStages], (ku / C::kStages) & 1, abortp);
       if (ok && pv_issued > 0) ok = mbar_wait(&bar.pv_done[i], (pv_issued - 1) & 1, abortp);
+      if (ok && i == 1 && j < w.nt_i[0]) {
+        // pacing: tile 1's S(j) follows tile 0's softmax of step j, so the two
+        // tiles' softmax phases alternate instead of sharing the MUFU and
+        // their MMAs fill each other's softmax time
+        const volatile int* p0 = &bar.p0_steps;
+        const long long t0 = clock64();
+        while (*p0 < p0_item + j + 1) {
+          if (*abortp || clock64() - t0 > kWaitCycles) {
+            *abortp = 1;
+            ok = false;
+            break;
+          }
+        }
+      }
       if (!ok) break;
       tc_fence_after();
       const uint32_t k_addr = kv_smem + (ku % C::kStages) * C::kTileBytes;
@@ -441,6 +468,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
   const uint32_t tS = lane_addr + (i ? C::kColS1 : C::kColS0);
   const uint32_t tO = lane_addr + (i ? C::kColO1 : C::kColO0);
   uint32_t s_count = 0, pv_total = 0, kv_count = 0;
+  int p0_published = 0;
   bool ok = true;
 
   for (uint32_t k = 0; ok; ++k) {
@@ -514,6 +542,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
       }
       l += lt;
       publish_p(&bar.p_full[i]);
+      if (i == 0 && rel) *reinterpret_cast<volatile int*>(&bar.p0_steps) = ++p0_published;
     }
     if (!ok) break;
     // ---- epilogue: O / l -> bf16
@@ -585,6 +614,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.item_empty[s], kItemConsumers);
     }
     bar.abort_flag = 0;
+    bar.p0_steps = 0;
     fence_barrier_init();
   }
   if (warp == 0 && lane == 0) {
