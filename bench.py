@@ -362,7 +362,9 @@ def run_ours(args):
             raise RuntimeError("device status after the end-to-end loop")
 
     # ---- restore of the full 80-layer KV of one 8192-token prefix
-    restore80 = ttft80 = None
+    restore80 = ttft80 = decode = None
+    if not args.no_decode and rank == 0:
+        decode = bench_decode(args, pk)
     if not args.no_restore80 and rank == 0:
         image, restore80 = bench_restore80(args, pk)
         ttft80 = bench_ttft80(args, image)
@@ -395,7 +397,8 @@ def run_ours(args):
                              "bytes_per_launch": 2 * restore_payload, "ms_per_launch": restore_ms},
         "breakdown_ms": {"restore": restore_ms, "append": append_ms, "attention": attn_ms},
         "attn_tflops": attn_tflops, "restore_gbs": restore_gbs,
-        "e2e": e2e, "restore_80layer": restore80, "prefill_80layer": ttft80, "clocks": clocks,
+        "e2e": e2e, "restore_80layer": restore80, "prefill_80layer": ttft80, "decode": decode,
+        "clocks": clocks,
         "gpu_launches": 3 * args.steps,
     }
     if world == 1 and rank == 0 and not args.no_cpu_baseline:
@@ -513,6 +516,49 @@ def bench_restore80(args, pk):
     }
 
 
+def bench_decode(args, pk):
+    """Paged decode attention (one new token per request) on two contexts
+    mixes: 8 x 9216 tokens (the 70B prefill config, continued) and the 64
+    conversation-mix contexts.  HBM-bound: algorithmic bytes = every context
+    key's K and V row once + q + out."""
+    import torch
+
+    from paper_2505_23970_gb300 import binding as gcb
+    from paper_2505_23970_gb300 import workloads as wl
+    from paper_2505_23970_gb300.harness import DeviceBatch
+
+    res = {}
+    stream = torch.cuda.current_stream()
+    for w in (wl.llama3_70b_decode(seed=args.seed), wl.decode_mix(seed=args.seed)):
+        db = DeviceBatch(w)
+        db.restore()
+        db.append()
+        db.decode()
+        torch.cuda.synchronize()
+        reps = 20
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        for _ in range(3):
+            db.decode(stream)
+        a.record(stream)
+        for _ in range(reps):
+            db.decode(stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / reps
+        ok = db.check(stream) == gcb.GC_OK
+        kv = int(w.total_lens.sum()) * w.Hkv * w.d * 2 * 2
+        qo = 2 * w.B * w.Hq * w.d * 2
+        gbs = (kv + qo) / (ms / 1e3) / 1e9
+        splits = gcb.gc_paged_decode_workspace_bytes(db.pool.handle, w.B, w.max_blocks, w.Hq)
+        res[w.name] = {"batch": w.B, "context_tokens": int(w.total_lens.sum()),
+                       "us_per_step": ms * 1e3, "bytes_per_step": kv + qo, "gbs": gbs,
+                       "frac_hbm": gbs / pk["hbm_gbs"], "tok_per_s": w.B / (ms / 1e3),
+                       "split": splits > 0, "device_status_ok": ok}
+        db.close()
+    return res
+
+
 def bench_ttft80(args, image=None):
     """All 80 layers of one request with an 8192-token cached prefix and
     1024 new tokens: restore of each layer's cached pages (pinned host ->
@@ -593,6 +639,7 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-restore80", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--ref-step-seconds", type=float, default=None,

@@ -22,6 +22,8 @@
  *                           request's cached prefix                (stitch)
  *   gc_prefix_prefill_attn  causal GQA attention of the new tokens over
  *                           the pool through a block table         (prefill)
+ *   gc_paged_decode_attn    the same for one new token per request,
+ *                           split over key ranges                  (decode)
  *
  * Conventions for every call
  *  - All device work is ordered on the caller's stream; no call synchronises
@@ -349,6 +351,39 @@ GC_API gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* po
                                       int32_t layer, const int32_t* cu_new_lens, int32_t batch,
                                       int32_t max_blocks_per_seq, int32_t num_q_heads,
                                       float softmax_scale, int32_t total_new_tokens);
+
+/* Paged decode attention: one new token per request (Sec. 2.1: the decode
+ * phase generates output tokens one at a time, and with the KV cache it is
+ * bound by memory).  For request b, q head h and g = h / (Hq/Hkv):
+ *     out[b][h] = sum_{j < seq_lens[b]} softmax_j(softmax_scale *
+ *                                         q[b][h] . k_j) v_j
+ * with k_j, v_j read from pool[layer] through block_table[b]; the new
+ * token's own K/V must already be in the pool at position seq_lens[b] - 1
+ * (gc_kv_append with one new token).  Equals gc_prefix_prefill_attn with
+ * prefix_lens = seq_lens - 1 and one new token per request.
+ *   q, out      [batch][Hq][d] bf16, device.  fp32 arithmetic, out rounded
+ *               to nearest even.
+ *   seq_lens    int32 [batch], device: context length T_b >= 1 including
+ *               the new token; a length outside [1, max_blocks_per_seq*ps]
+ *               is recorded as GC_ERR_OUT_OF_RANGE (and clamped).
+ *   block_table int32 [batch][max_blocks_per_seq], device; a bad page is
+ *               skipped (its keys left out) and recorded.
+ *   workspace   device scratch for requests split over several key ranges:
+ *               gc_paged_decode_workspace_bytes(pool, batch,
+ *               max_blocks_per_seq, num_q_heads) bytes (0: NULL is fine),
+ *               owned by the caller, not used after the stream passes the
+ *               call.  Calls sharing a workspace must not overlap on the GPU.
+ * Errors: GC_ERR_INVALID_ARG (null, unaligned, workspace too small),
+ * GC_ERR_OUT_OF_RANGE (layer), GC_ERR_UNSUPPORTED (head grouping),
+ * GC_ERR_CUDA. */
+GC_API size_t gc_paged_decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch,
+                                              int32_t max_blocks_per_seq, int32_t num_q_heads);
+GC_API gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool,
+                                      const int32_t* block_table, const int32_t* seq_lens,
+                                      void* out, cudaStream_t stream, int32_t layer,
+                                      int32_t batch, int32_t max_blocks_per_seq,
+                                      int32_t num_q_heads, float softmax_scale, void* workspace,
+                                      size_t workspace_bytes);
 
 /* Message of the last failing call on this thread ("" if none). */
 GC_API const char* gc_last_error(void);

@@ -38,7 +38,8 @@ EXPORTED = (
     "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
     "gc_kv_save_layers", "gc_kv_q8_chunk_bytes", "gc_kv_save_q8", "gc_kv_restore_q8",
     "gc_kv_append", "gc_prefix_prefill_attn",
-    "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc", "gc_last_error",
+    "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc",
+    "gc_paged_decode_workspace_bytes", "gc_paged_decode_attn", "gc_last_error",
     "gc_status_string",
 )
 
@@ -90,11 +91,15 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_prefix_prefill_attn.argtypes = attn
         lib.gc_prefix_prefill_attn_simt.argtypes = attn
         lib.gc_prefix_prefill_attn_noalloc.argtypes = attn
+        lib.gc_paged_decode_workspace_bytes.argtypes = [vp, i32, i32, i32]
+        lib.gc_paged_decode_workspace_bytes.restype = ctypes.c_size_t
+        lib.gc_paged_decode_attn.argtypes = [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32,
+                                             ctypes.c_float, vp, ctypes.c_size_t]
         for f in ("gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
                   "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
                   "gc_kv_save_layers", "gc_kv_save_q8", "gc_kv_restore_q8", "gc_kv_append",
                   "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt",
-                  "gc_prefix_prefill_attn_noalloc"):
+                  "gc_prefix_prefill_attn_noalloc", "gc_paged_decode_attn"):
             getattr(lib, f).restype = ctypes.c_int
         lib.gc_last_error.argtypes = []
         lib.gc_last_error.restype = ctypes.c_char_p
@@ -305,3 +310,19 @@ class KVPool:
             self.close()
         except Exception:
             pass
+
+
+def gc_paged_decode_workspace_bytes(pool, batch: int, max_blocks_per_seq: int,
+                                    num_q_heads: int) -> int:
+    return int(load().gc_paged_decode_workspace_bytes(pool, batch, max_blocks_per_seq,
+                                                      num_q_heads))
+
+
+def gc_paged_decode_attn(q, pool, block_table, seq_lens, out, stream, layer: int, batch: int,
+                         max_blocks_per_seq: int, num_q_heads: int, softmax_scale: float,
+                         workspace=None, workspace_bytes: int = 0) -> None:
+    _check(load().gc_paged_decode_attn(_addr(q), pool, _addr(block_table), _addr(seq_lens),
+                                       _addr(out), _stream(stream), layer, batch,
+                                       max_blocks_per_seq, num_q_heads, softmax_scale,
+                                       _addr(workspace), workspace_bytes),
+           "gc_paged_decode_attn")

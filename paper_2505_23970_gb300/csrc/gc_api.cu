@@ -108,7 +108,8 @@ gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, size_t dev
   p->data = static_cast<uint8_t*>(mem);
   p->data_bytes = need - kTrailer;
   p->status = reinterpret_cast<int32_t*>(p->data + p->data_bytes);
-  p->work_counter = p->status + 32;  // 128 bytes into the 256-byte control block
+  p->work_counter = p->status + 32;    // 128 bytes into the 256-byte control block
+  p->decode_counter = p->status + 48;  // 192 bytes in
   p->owned = owned;
   p->device = dev;
   p->num_sms = sms;
@@ -536,6 +537,45 @@ gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* pool,
                             num_q_heads, softmax_scale, total_new_tokens, &a, &noop);
   if (s != GC_OK || noop) return s;
   return gc::launch_attn_simt(pool, a, stream);
+}
+
+size_t gc_paged_decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch,
+                                       int32_t max_blocks_per_seq, int32_t num_q_heads) {
+  if (!pool || batch <= 0 || max_blocks_per_seq <= 0 || num_q_heads <= 0) return 0;
+  return gc::decode_split(pool, batch, max_blocks_per_seq, num_q_heads).workspace_bytes;
+}
+
+gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool, const int32_t* block_table,
+                               const int32_t* seq_lens, void* out, cudaStream_t stream,
+                               int32_t layer, int32_t batch, int32_t max_blocks_per_seq,
+                               int32_t num_q_heads, float softmax_scale, void* workspace,
+                               size_t workspace_bytes) {
+  g_msg[0] = 0;
+  const char* who = "gc_paged_decode_attn";
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (batch < 0 || max_blocks_per_seq < 0) return fail(GC_ERR_INVALID_ARG, "%s: negative size", who);
+  if (layer < 0 || layer >= pool->cfg.num_layers)
+    return fail(GC_ERR_OUT_OF_RANGE, "%s: layer %d outside [0, %d)", who, layer,
+                pool->cfg.num_layers);
+  const int hkv = pool->cfg.num_kv_heads;
+  if (num_q_heads <= 0 || num_q_heads % hkv)
+    return fail(GC_ERR_INVALID_ARG, "%s: num_q_heads %d not a multiple of num_kv_heads %d", who,
+                num_q_heads, hkv);
+  const int G = num_q_heads / hkv;
+  if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16)
+    return fail(GC_ERR_UNSUPPORTED, "%s: q heads per kv head %d not in {1,2,4,8,16}", who, G);
+  if (!(softmax_scale > 0.0f) || softmax_scale == __builtin_inff())
+    return fail(GC_ERR_INVALID_ARG, "%s: softmax_scale must be positive and finite", who);
+  if (batch == 0) return GC_OK;
+  if (!q || !out || !block_table || !seq_lens)
+    return fail(GC_ERR_INVALID_ARG, "%s: NULL array argument", who);
+  if (max_blocks_per_seq == 0) return fail(GC_ERR_INVALID_ARG, "%s: max_blocks_per_seq is 0", who);
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out) |
+       reinterpret_cast<uintptr_t>(workspace)) % 16)
+    return fail(GC_ERR_INVALID_ARG, "%s: q / out / workspace not 16-byte aligned", who);
+  const gc::DecodeArgs a{q, out, block_table, seq_lens, batch, max_blocks_per_seq, layer,
+                         num_q_heads, softmax_scale, workspace, workspace_bytes};
+  return gc::launch_decode(pool, a, stream);
 }
 
 }  // extern "C"

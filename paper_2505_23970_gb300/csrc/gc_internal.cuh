@@ -15,6 +15,7 @@ struct gc_kv_pool {
   size_t data_bytes;
   int32_t* status;        // device status word (first error recorded by a kernel)
   int32_t* work_counter;  // attention work-item counter (control block, zeroed per launch)
+  int32_t* decode_counter;  // decode work-unit counter (control block, zeroed per launch)
   void* owned;            // cudaMalloc'd block, or nullptr if caller-owned
   int device;
   int num_sms;
@@ -77,5 +78,24 @@ struct AttnArgs {
 gc_status launch_attn_simt(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
+
+// Paged decode attention (one new token per request), split-KV.
+struct DecodeArgs {
+  const void* q;
+  void* out;
+  const int32_t* block_table;
+  const int32_t* seq_lens;
+  int32_t batch, max_blocks, layer, num_q_heads;
+  float softmax_scale;
+  void* workspace;
+  size_t workspace_bytes;
+};
+struct DecodeSplit {
+  int32_t splits, split_len;  // key ranges per request and their length
+  size_t workspace_bytes;     // 0 when requests are not split
+};
+DecodeSplit decode_split(const gc_kv_pool* pool, int32_t batch, int32_t max_blocks,
+                         int32_t num_q_heads);
+gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream);
 
 }  // namespace gc

@@ -124,6 +124,25 @@ class DeviceBatch:
            self.out if out is None else out, stream, layer, self.cu_new_lens, w.B, w.max_blocks,
            w.Hq, w.scale, w.T_new)
 
+    def decode(self, stream=None, layer: int = 0, out=None, workspace=None):
+        """gc_paged_decode_attn of the batch's one new token per request over
+        its whole context (seq_lens = prefix + 1); allocates the workspace the
+        library asks for unless one is given."""
+        import torch
+        w = self.w
+        assert np.all(w.new_lens == 1), "decode takes one new token per request"
+        if not hasattr(self, "seq_lens"):
+            self.seq_lens = _i32(w.total_lens, self.device)
+        need = gcb.gc_paged_decode_workspace_bytes(self.pool.handle, w.B, w.max_blocks, w.Hq)
+        if workspace is None and need:
+            if getattr(self, "_dec_ws", None) is None or self._dec_ws.numel() < need:
+                self._dec_ws = torch.empty(need, dtype=torch.uint8, device=self.device)
+            workspace = self._dec_ws
+        gcb.gc_paged_decode_attn(self.q, self.pool.handle, self.block_table, self.seq_lens,
+                                 self.out if out is None else out, stream, layer, w.B,
+                                 w.max_blocks, w.Hq, w.scale, workspace,
+                                 0 if workspace is None else workspace.numel())
+
     def run(self, stream=None, restore_mode: str = "staged", impl: str = "tc"):
         self.restore(stream, restore_mode)
         self.append(stream)

@@ -238,6 +238,22 @@ def llama3_70b_80layer_prefill(seed: int = 0, prefix: int = 8192, new: int = 102
     return w
 
 
+def llama3_70b_decode(seed: int = 0, B: int = 8, context: int = 9216) -> Workload:
+    """Decode step on the 70B-shaped layer: B requests whose context of
+    `context` tokens (the 8192 + 1024 of the 70B prefill config) ends with the
+    new token: cached prefix context - 1, one new token each."""
+    return _mk("llama3-70b-decode", B, 64, 8, 128, 16, [context - 1] * B, [1] * B, seed)
+
+
+def decode_mix(seed: int = 0, B: int = 64) -> Workload:
+    """Decode step after the multi-turn mix: contexts = prefix + suffix of
+    the conversation mix (p = 1), one new token each."""
+    rng = np.random.default_rng([seed, _S_LENS])
+    P = np.clip(np.rint(rng.lognormal(math.log(2048), 1.0, size=B)), 0, 32768).astype(np.int64)
+    S = np.clip(np.rint(rng.lognormal(math.log(200), 0.8, size=B)), 16, 4096).astype(np.int64)
+    return _mk("decode-mix", B, 64, 8, 128, 16, P + S - 1, [1] * B, seed)
+
+
 def conversation_mix(seed: int = 0, hit_p: float = 1.0, B: int = 64) -> Workload:
     """Multi-turn mix on the 70B-shaped layer: prefix ~ LogNormal(ln 2048, 1.0)
     clipped to [0, 32768], new ~ LogNormal(ln 200, 0.8) clipped to
@@ -274,4 +290,6 @@ CONFIGS = {
     "70b": llama3_70b_layer,
     "mix": conversation_mix,
     "long": long_document,
+    "decode": llama3_70b_decode,
+    "decode-mix": decode_mix,
 }
