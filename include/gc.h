@@ -364,8 +364,9 @@ GC_API gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* po
  *   q, out      [batch][Hq][d] bf16, device.  fp32 arithmetic, out rounded
  *               to nearest even.
  *   seq_lens    int32 [batch], device: context length T_b >= 1 including
- *               the new token; a length outside [1, max_blocks_per_seq*ps]
- *               is recorded as GC_ERR_OUT_OF_RANGE (and clamped).
+ *               the new token; a request whose length is outside
+ *               [1, max_blocks_per_seq*ps] is skipped (its out rows are not
+ *               written) and recorded as GC_ERR_OUT_OF_RANGE.
  *   block_table int32 [batch][max_blocks_per_seq], device; a bad page is
  *               skipped (its keys left out) and recorded.
  *   workspace   device scratch for requests split over several key ranges:
@@ -373,9 +374,12 @@ GC_API gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* po
  *               max_blocks_per_seq, num_q_heads) bytes (0: NULL is fine),
  *               owned by the caller, not used after the stream passes the
  *               call.  Calls sharing a workspace must not overlap on the GPU.
+ * Runs on the prefill kernel's tensor-core path in a decode mode; calls on
+ * one pool must not overlap on the GPU with each other or with
+ * gc_prefix_prefill_attn (they share the pool's work counter).
  * Errors: GC_ERR_INVALID_ARG (null, unaligned, workspace too small),
- * GC_ERR_OUT_OF_RANGE (layer), GC_ERR_UNSUPPORTED (head grouping),
- * GC_ERR_CUDA. */
+ * GC_ERR_OUT_OF_RANGE (layer), GC_ERR_UNSUPPORTED (head grouping,
+ * batch > 8192), GC_ERR_CUDA. */
 GC_API size_t gc_paged_decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch,
                                               int32_t max_blocks_per_seq, int32_t num_q_heads);
 GC_API gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool,

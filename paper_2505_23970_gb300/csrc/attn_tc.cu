@@ -83,6 +83,12 @@ struct Cfg {
 struct Geom {
   int32_t batch, Hq, Hkv, G, ps, ps_shift, num_pages, max_blocks, layer, total_new;
   float scale_log2;
+  // decode mode: one new token per request, context lengths in seq_lens,
+  // each request's keys cut into ranges of split_tiles K/V tiles; a request
+  // with several ranges writes fp32 partials (O, max, sum) to ws
+  int32_t decode, split_tiles, max_splits;
+  const int32_t* seq_lens;
+  float* ws;
 };
 
 struct Barriers {
@@ -105,6 +111,8 @@ struct Item {
   int b, g, P, n, cu, T;
   int tok0[2], nt_i[2], nt;
   bool valid[2];
+  int j0;             // first K/V tile (key range start / kTileN)
+  int split, nsplit;  // key range of the item and ranges of its request
 };
 
 // item_start[p] = first item of the p-th request in work order; the request
@@ -123,6 +131,28 @@ __device__ __forceinline__ bool decode_item(int it, const int* item_start, const
                                        : lo;
   w.b = b;
   const int local = it - item_start[lo];
+  if (geo.decode) {
+    // (request, kv head, key range): one Q tile of G rows, tiles [j0, end)
+    w.g = local % geo.Hkv;
+    w.split = local / geo.Hkv;
+    w.T = __ldg(geo.seq_lens + b);
+    w.P = w.T - 1;
+    w.n = 1;
+    w.cu = b;
+    const int nt_full = (w.T + kTileN - 1) / kTileN;
+    w.nsplit = (nt_full + geo.split_tiles - 1) / geo.split_tiles;
+    w.j0 = w.split * geo.split_tiles;
+    w.valid[0] = true;
+    w.valid[1] = false;
+    w.tok0[0] = w.tok0[1] = 0;
+    w.nt_i[0] = min(w.j0 + geo.split_tiles, nt_full);
+    w.nt_i[1] = 0;
+    w.nt = w.nt_i[0];
+    return true;
+  }
+  w.j0 = 0;
+  w.split = 0;
+  w.nsplit = 1;
   const int pairs = (item_start[lo + 1] - item_start[lo]) / geo.Hkv;
   const int pair = pairs - 1 - local / geo.Hkv;  // later rows (more keys) first
   w.g = local % geo.Hkv;
@@ -229,8 +259,8 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
         pg_id = blk0 + lane < geo.max_blocks ? __ldg(block_table + bt_row + blk0 + lane) : -1;
       return pg_id;
     };
-    int page_next = lookup(0);
-    for (int j = 0; ok && j < w.nt; ++j) {
+    int page_next = lookup(w.j0);
+    for (int j = w.j0; ok && j < w.nt; ++j) {
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
       int page = page_next;
@@ -324,18 +354,18 @@ __device__ void mma_issuer(int i, uint8_t* smem_q, uint8_t* smem_kv, Barriers& b
     decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
     // K_j sits in ring use kv_base + 2j, V_j in use kv_base + 2j + 1
     const uint32_t kv_base = kv_count;
-    kv_count += 2 * w.nt;
+    kv_count += 2 * (w.nt - w.j0);
     const int p0_item = p0_base;
-    p0_base += w.nt_i[0];
+    p0_base += w.nt_i[0] - w.j0;
     const uint32_t q_par = q_count & 1;
     ++q_count;
     if (!w.valid[i]) continue;
     ok = mbar_wait(&bar.q_full, q_par, abortp);
     if (!ok) break;
     tc_fence_after();
-    for (int j = 0; j < w.nt_i[i]; ++j) {
+    for (int j = w.j0; j < w.nt_i[i]; ++j) {
       // S_i = Q_i K_j^T once K_j is in and PV_i(j-1) has finished reading P_i
-      const uint32_t ku = kv_base + 2 * j;
+      const uint32_t ku = kv_base + 2 * (j - w.j0);
       ok = mbar_wait(&bar.kv_full[ku % C::kStages], (ku / C::kStages) & 1, abortp);
       if (ok && pv_issued > 0) ok = mbar_wait(&bar.pv_done[i], (pv_issued - 1) & 1, abortp);
       if (ok && i == 1 && j < w.nt_i[0]) {
@@ -344,7 +374,7 @@ __device__ void mma_issuer(int i, uint8_t* smem_q, uint8_t* smem_kv, Barriers& b
         // their MMAs fill each other's softmax time
         const volatile int* p0 = &bar.p0_steps;
         const long long t0 = clock64();
-        while (*p0 < p0_item + j + 1) {
+        while (*p0 < p0_item + (j - w.j0) + 1) {
           if (*abortp || clock64() - t0 > kWaitCycles) {
             *abortp = 1;
             ok = false;
@@ -374,7 +404,7 @@ __device__ void mma_issuer(int i, uint8_t* smem_q, uint8_t* smem_kv, Barriers& b
       for (int kk = 0; kk < kTileN / 16; ++kk)
         mma_ts(tmem + col_o, tmem + col_s + kk * 8,
                sdesc_sw128(v_addr + kk * 16 * 128, C::kHalfBytes, 1024), C::kIdescPV,
-               (j > 0 || kk > 0) ? 1u : 0u);
+               (j > w.j0 || kk > 0) ? 1u : 0u);
       mma_commit(&bar.pv_done[i]);
       ++pv_issued;
     }
@@ -481,7 +511,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
     decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
     // K_j sits in ring use kv_base + 2j, V_j in use kv_base + 2j + 1
     const uint32_t kv_base = kv_count;
-    kv_count += 2 * w.nt;
+    kv_count += 2 * (w.nt - w.j0);
     if (!w.valid[i]) continue;
     // This tile releases the ring slots (and the Q tiles) once the MMAs that
     // read them are known complete; for K/V tiles (or Q) the other tile does
@@ -489,14 +519,14 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
     const bool rel = threadIdx.x == kTileM * (1 + i);
     const int nt_o = w.valid[1 - i] ? w.nt_i[1 - i] : 0;
     auto release = [&](int j, int kv) {
-      const uint32_t use = kv_base + 2 * j + kv;
+      const uint32_t use = kv_base + 2 * (j - w.j0) + kv;
       mbar_arrive_cnt(&bar.kv_empty[use % C::kStages], j < nt_o ? 1u : 2u);
     };
     const int tok = w.tok0[i] + r / geo.G;
     const bool row_valid = tok < w.n;
     const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
     float m_run = -INFINITY, l = 0.f;
-    for (int j = 0; j < w.nt_i[i]; ++j) {
+    for (int j = w.j0; j < w.nt_i[i]; ++j) {
       ok = mbar_wait(&bar.s_full[i], s_count & 1, abortp);
       ++s_count;
       if (!ok) break;
@@ -504,7 +534,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
         // S_i(j) is complete: K_j is done with for this tile; and S_i(j) was
         // issued after PV_i(j-1) completed, so V_{j-1} is too
         release(j, 0);
-        if (j > 0) release(j - 1, 1);
+        if (j > w.j0) release(j - 1, 1);
         if (j == w.nt_i[i] - 1) mbar_arrive_cnt(&bar.q_empty, w.valid[1 - i] ? 1u : 2u);
       }
       tc_fence_after();
@@ -546,13 +576,39 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
     }
     if (!ok) break;
     // ---- epilogue: O / l -> bf16
-    pv_total += w.nt_i[i];
+    pv_total += w.nt_i[i] - w.j0;
     ok = mbar_wait(&bar.pv_done[i], (pv_total - 1) & 1, abortp);
     if (!ok) break;
     if (rel) release(w.nt_i[i] - 1, 1);
     tc_fence_after();
-    const float inv_l = 1.f / l;
     const int h = w.g * geo.G + r % geo.G;
+    if (w.nsplit > 1) {
+      // one key range of a split request: fp32 partials O (unnormalised),
+      // reference max (log2 units) and sum, merged by a second kernel
+      const int64_t head = static_cast<int64_t>(w.b) * geo.Hq + h;
+      float* o_ws = geo.ws + (head * geo.max_splits + w.split) * D;
+#pragma unroll 1
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t o[32];
+        tmem_ld32(tO + c * 32, o);
+        tmem_wait_ld();
+        if (row_valid) {
+#pragma unroll
+          for (int v = 0; v < 8; ++v)
+            reinterpret_cast<uint4*>(o_ws + c * 32)[v] =
+                make_uint4(o[4 * v], o[4 * v + 1], o[4 * v + 2], o[4 * v + 3]);
+        }
+      }
+      if (row_valid) {
+        float* ml = geo.ws + static_cast<int64_t>(geo.batch) * geo.Hq * geo.max_splits * D +
+                    (head * geo.max_splits + w.split) * 2;
+        ml[0] = m_run;
+        ml[1] = l;
+      }
+      tc_fence_before();
+      continue;
+    }
+    const float inv_l = 1.f / l;
     uint4* orow = reinterpret_cast<uint4*>(
         out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * D);
 #pragma unroll 1
@@ -627,11 +683,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (geo.batch <= kSortMax) {
     // rank requests by total length, longest first (ties by index)
+    auto total_len = [&](int b) {
+      return geo.decode ? __ldg(geo.seq_lens + b) : __ldg(prefix_lens + b) + __ldg(new_lens + b);
+    };
     for (int b = threadIdx.x; b < geo.batch; b += kThreads) {
-      const int tb = __ldg(prefix_lens + b) + __ldg(new_lens + b);
+      const int tb = total_len(b);
       int rank = 0;
       for (int o = 0; o < geo.batch; ++o) {
-        const int to = __ldg(prefix_lens + o) + __ldg(new_lens + o);
+        const int to = total_len(o);
         rank += (to > tb) || (to == tb && o < b);
       }
       order[rank] = static_cast<int16_t>(b);
@@ -645,7 +704,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int p = b0 + lane;
       const int b = p < geo.batch ? (geo.batch <= kSortMax ? order[p] : p) : p;
       int cnt = 0;
-      if (p < geo.batch) {
+      if (p < geo.batch && geo.decode) {
+        // a context of T keys, cut into ranges of split_tiles K/V tiles
+        const int T = __ldg(geo.seq_lens + b);
+        if (T < 1 || T > (geo.max_blocks << geo.ps_shift)) {
+          record_error(status, GC_ERR_OUT_OF_RANGE);
+        } else {
+          const int nt_full = (T + kTileN - 1) / kTileN;
+          cnt = geo.Hkv * ((nt_full + geo.split_tiles - 1) / geo.split_tiles);
+        }
+      } else if (p < geo.batch) {
         const int n = __ldg(new_lens + b), P = __ldg(prefix_lens + b);
         const int cu = __ldg(cu_new_lens + b);
         const bool sane = n >= 0 && P >= 0 && cu >= 0 && cu + n <= geo.total_new;
@@ -713,7 +781,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 template <int D>
 gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
-                 int* work_counter) {
+                 int* work_counter, const DecodeMode* dm = nullptr) {
   using C = Cfg<D>;
   auto enc = encode_fn();
   if (!enc) return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: cuTensorMapEncodeTiled unavailable");
@@ -732,6 +800,11 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   geo.layer = a.layer;
   geo.total_new = a.total_new_tokens;
   geo.scale_log2 = a.softmax_scale * 1.4426950408889634f;
+  geo.decode = dm != nullptr;
+  geo.split_tiles = dm ? dm->split_tiles : 0;
+  geo.max_splits = dm ? dm->max_splits : 0;
+  geo.seq_lens = dm ? dm->seq_lens : nullptr;
+  geo.ws = dm ? dm->ws : nullptr;
 
   const uint64_t pool_rows = static_cast<uint64_t>(cfg.num_layers) * 2 * cfg.num_pages *
                              cfg.num_kv_heads * cfg.page_size;
@@ -786,6 +859,12 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
   if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter);
   return launch<64>(pool, a, stream, pool->work_counter);
+}
+
+gc_status launch_attn_tc_decode(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode& dm,
+                                cudaStream_t stream) {
+  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter, &dm);
+  return launch<64>(pool, a, stream, pool->work_counter, &dm);
 }
 
 }  // namespace gc

@@ -108,8 +108,7 @@ gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, size_t dev
   p->data = static_cast<uint8_t*>(mem);
   p->data_bytes = need - kTrailer;
   p->status = reinterpret_cast<int32_t*>(p->data + p->data_bytes);
-  p->work_counter = p->status + 32;    // 128 bytes into the 256-byte control block
-  p->decode_counter = p->status + 48;  // 192 bytes in
+  p->work_counter = p->status + 32;  // 128 bytes into the 256-byte control block
   p->owned = owned;
   p->device = dev;
   p->num_sms = sms;

@@ -15,7 +15,6 @@ struct gc_kv_pool {
   size_t data_bytes;
   int32_t* status;        // device status word (first error recorded by a kernel)
   int32_t* work_counter;  // attention work-item counter (control block, zeroed per launch)
-  int32_t* decode_counter;  // decode work-unit counter (control block, zeroed per launch)
   void* owned;            // cudaMalloc'd block, or nullptr if caller-owned
   int device;
   int num_sms;
@@ -78,6 +77,15 @@ struct AttnArgs {
 gc_status launch_attn_simt(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
+// The same kernel in decode mode: one new token per request (AttnArgs'
+// prefix_lens / new_lens / cu_new_lens unused), keys cut into ranges.
+struct DecodeMode {
+  int32_t split_tiles, max_splits;
+  const int32_t* seq_lens;
+  float* ws;
+};
+gc_status launch_attn_tc_decode(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode& dm,
+                                cudaStream_t stream);
 
 // Paged decode attention (one new token per request), split-KV.
 struct DecodeArgs {
