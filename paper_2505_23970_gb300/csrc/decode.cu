@@ -12,8 +12,9 @@
 // pages through a TMA ring with bulk copies several tiles ahead, and the
 // tensor cores do the G-row products (a Q tile of G real rows: the padding
 // rows cost tensor time that the memory bound leaves idle anyway).  To fill
-// every SM, each request is cut into key ranges of kSplitTiles K/V tiles
-// (work items = requests x kv heads x ranges); a request with several ranges
+// every SM, each request is cut into key ranges of 4 to 16 K/V tiles, chosen
+// per call from the batch and the block table's capacity (work items =
+// requests x kv heads x ranges); a request with several ranges
 // writes fp32 partials (O unnormalised, reference max in log2 units, sum)
 // and the merge kernel below combines them:
 //     out = sum_s O_s 2^(m_s - M) / sum_s l_s 2^(m_s - M),  M = max_s m_s.
@@ -23,13 +24,14 @@
 namespace gc {
 namespace {
 
-constexpr int kTileKeys = 128;  // keys per K/V tile of the attention kernel
-constexpr int kSplitTiles = 4;  // K/V tiles per key range (512 keys)
+constexpr int kTileKeys = 128;     // keys per K/V tile of the attention kernel
+constexpr int kMinSplitTiles = 4;  // key ranges of 4..16 K/V tiles (512..2048 keys)
+constexpr int kMaxSplitTiles = 16;
 
-__device__ __forceinline__ int request_splits(int T, int cap) {
+__device__ __forceinline__ int request_splits(int T, int cap, int split_tiles) {
   if (T < 1 || T > cap) return 0;  // recorded as an error by the attention kernel
   const int tiles = (T + kTileKeys - 1) / kTileKeys;
-  return (tiles + kSplitTiles - 1) / kSplitTiles;
+  return (tiles + split_tiles - 1) / split_tiles;
 }
 
 template <int D>
@@ -37,10 +39,11 @@ __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict
                                                          const int32_t* __restrict__ seq_lens,
                                                          int32_t batch, int32_t Hq,
                                                          int32_t max_splits, int32_t cap,
+                                                         int32_t split_tiles,
                                                          __nv_bfloat16* __restrict__ out) {
   const int64_t head = blockIdx.x;
   const int b = static_cast<int>(head / Hq);
-  const int nsplit = request_splits(__ldg(seq_lens + b), cap);
+  const int nsplit = request_splits(__ldg(seq_lens + b), cap, split_tiles);
   if (nsplit <= 1) return;  // written by the attention kernel itself (or invalid)
   const int d = threadIdx.x;
   const float* ml = ws + static_cast<int64_t>(batch) * Hq * max_splits * D + head * max_splits * 2;
@@ -62,9 +65,18 @@ DecodeSplit decode_split(const gc_kv_pool* pool, int32_t batch, int32_t max_bloc
   DecodeSplit d;
   const int64_t cap = static_cast<int64_t>(max_blocks) * pool->cfg.page_size;
   const int64_t tiles = (cap + kTileKeys - 1) / kTileKeys;
-  const int64_t splits = tiles > 0 ? (tiles + kSplitTiles - 1) / kSplitTiles : 1;
+  // Longer ranges cost less per tile (each work item has a fixed start-up and
+  // epilogue); shorter ones spread a small batch over more SMs.  Aim for about
+  // two items per CTA when every request had the longest context.
+  const int64_t tile_units = static_cast<int64_t>(batch) * pool->cfg.num_kv_heads * tiles;
+  int split_tiles = kMinSplitTiles;
+  while (split_tiles < kMaxSplitTiles &&
+         tile_units > static_cast<int64_t>(split_tiles) * 2 * pool->num_sms)
+    split_tiles *= 2;
+  const int64_t splits = tiles > 0 ? (tiles + split_tiles - 1) / split_tiles : 1;
   d.splits = static_cast<int32_t>(splits);
-  d.split_len = kSplitTiles * kTileKeys;
+  d.split_tiles = split_tiles;
+  d.split_len = split_tiles * kTileKeys;
   d.workspace_bytes = splits > 1 ? static_cast<size_t>(batch) * num_q_heads * splits *
                                        (pool->cfg.head_dim + 2) * sizeof(float)
                                  : 0;
@@ -87,18 +99,18 @@ gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_
     return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: %lld-token block table", (long long)cap);
   AttnArgs args{a.q, a.out, a.block_table, nullptr, nullptr, nullptr, a.batch, a.max_blocks,
                 a.layer, a.num_q_heads, a.batch, a.softmax_scale};
-  const DecodeMode dm{kSplitTiles, sp.splits, a.seq_lens, static_cast<float*>(a.workspace)};
+  const DecodeMode dm{sp.split_tiles, sp.splits, a.seq_lens, static_cast<float*>(a.workspace)};
   gc_status st = launch_attn_tc_decode(pool, args, dm, stream);
   if (st != GC_OK || sp.splits <= 1) return st;
   const unsigned heads = static_cast<unsigned>(a.batch) * static_cast<unsigned>(a.num_q_heads);
   if (pool->cfg.head_dim == 128)
     decode_merge_kernel<128><<<heads, 128, 0, stream>>>(
         static_cast<const float*>(a.workspace), a.seq_lens, a.batch, a.num_q_heads, sp.splits,
-        static_cast<int32_t>(cap), static_cast<__nv_bfloat16*>(a.out));
+        static_cast<int32_t>(cap), sp.split_tiles, static_cast<__nv_bfloat16*>(a.out));
   else
     decode_merge_kernel<64><<<heads, 64, 0, stream>>>(
         static_cast<const float*>(a.workspace), a.seq_lens, a.batch, a.num_q_heads, sp.splits,
-        static_cast<int32_t>(cap), static_cast<__nv_bfloat16*>(a.out));
+        static_cast<int32_t>(cap), sp.split_tiles, static_cast<__nv_bfloat16*>(a.out));
   const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "gc_paged_decode_attn: merge kernel launch");
   return GC_OK;

@@ -99,7 +99,7 @@ struct DecodeArgs {
   size_t workspace_bytes;
 };
 struct DecodeSplit {
-  int32_t splits, split_len;  // key ranges per request and their length
+  int32_t splits, split_tiles, split_len;  // key ranges per request (at most), their length
   size_t workspace_bytes;     // 0 when requests are not split
 };
 DecodeSplit decode_split(const gc_kv_pool* pool, int32_t batch, int32_t max_blocks,

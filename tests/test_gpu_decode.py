@@ -104,7 +104,7 @@ def test_decode_matches_prefill_kernel_with_one_new_token():
 
 def test_decode_errors():
     import torch
-    w = wl.llama3_70b_decode(seed=2, B=2, context=1000)
+    w = wl.llama3_70b_decode(seed=2, B=2, context=5000)
     db = DeviceBatch(w)
     db.restore()
     db.append()
@@ -115,7 +115,7 @@ def test_decode_errors():
         db.decode(workspace=small)
     assert e.value.status == gcb.GC_ERR_INVALID_ARG
     # a context longer than the block table allows, and a bad page
-    db.seq_lens = _i32(np.array([w.max_blocks * w.ps + 5, 1000]), "cuda")
+    db.seq_lens = _i32(np.array([w.max_blocks * w.ps + 5, 5000]), "cuda")
     db.decode()
     assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
     bt = w.block_table.copy()
@@ -129,3 +129,10 @@ def test_decode_errors():
                              0, w.max_blocks, w.Hq, w.scale)
     assert db.check() == gcb.GC_OK
     db.close()
+
+
+@pytest.mark.parametrize("B,ctx", [(1, 9216), (2, 700), (40, 3000)])
+def test_decode_range_lengths_chosen_per_batch(B, ctx):
+    """Small and large batches get different key-range lengths (more ranges
+    for few requests); every choice matches the oracle."""
+    decode_parity(wl.llama3_70b_decode(seed=B, B=B, context=ctx))
