@@ -659,6 +659,8 @@ def main():
     ap.add_argument("--ref-step-seconds", type=float, default=None,
                     help="oracle seconds per step of --impl reference (default: sized so "
                          "the whole run takes about 2.5 minutes)")
+    ap.add_argument("--only", choices=["decode", "restore80", "prefill80"], default=None,
+                    help="run one secondary measurement alone and print it (for profilers)")
     ap.add_argument("--profile", action="store_true",
                     help="timed loop only (for ncu launch lists): no e2e, clocks or baselines")
     args = ap.parse_args()
@@ -668,6 +670,17 @@ def main():
     WORKLOAD = {"70b": "llama3-70b-layer", "8b": "llama3-8b-layer", "tiny": "tiny",
                 "long": "long-document", "long-recompute": "long-document-recompute"}.get(
                     args.config, f"conversation-{args.config}")
+    if args.only:
+        import torch
+        torch.cuda.set_device(0)
+        pk = peaks()
+        if args.only == "decode":
+            print(json.dumps({"decode": bench_decode(args, pk)}), flush=True)
+        elif args.only == "restore80":
+            print(json.dumps({"restore_80layer": bench_restore80(args, pk)[1]}), flush=True)
+        else:
+            print(json.dumps({"prefill_80layer": bench_ttft80(args)}), flush=True)
+        return
     if args.impl == "reference":
         run_reference(args)
     else:
