@@ -254,3 +254,14 @@ def test_layer_pipelined_schedule_matches_serial_and_oracle():
         assert_attn_close(piped.outs[l].to(torch.float64).cpu().numpy(), ref, f"layer {l}")
     serial.close()
     piped.close()
+
+
+def test_batch_beyond_sorted_ranking():
+    """More requests than the kernel ranks by length (512): work items keep
+    the given request order; outputs still match the oracle."""
+    rng = np.random.default_rng(21)
+    B = 700
+    P = rng.integers(0, 300, size=B)
+    n = rng.integers(0, 40, size=B)
+    w = wl.custom("big-batch", B, 16, 4, 64, 16, P, n, seed=21)
+    full_parity(w)

@@ -136,3 +136,10 @@ def test_decode_range_lengths_chosen_per_batch(B, ctx):
     """Small and large batches get different key-range lengths (more ranges
     for few requests); every choice matches the oracle."""
     decode_parity(wl.llama3_70b_decode(seed=B, B=B, context=ctx))
+
+
+def test_decode_batch_beyond_sorted_ranking():
+    """1000 requests (more than the 512 the kernel ranks by length)."""
+    ctx = np.random.default_rng(22).integers(1, 600, size=1000)
+    w = wl.custom("dec-big-batch", 1000, 16, 4, 64, 16, ctx - 1, np.ones(1000, int), seed=22)
+    decode_parity(w)
