@@ -8,39 +8,47 @@
 //
 // Design
 //  * Work item = (request b, kv head g, pair of 128-row Q tiles), handed out
-//    dynamically (an atomic counter in the pool's control block; items of a
-//    request are numbered later rows first, so long items start early).  A Q tile
-//    packs 128/G new tokens x the G q heads of one kv group (row = token*G +
-//    head), so every K/V tile fetched from the pool feeds all G heads, and
-//    the two Q tiles of a CTA share each K/V tile as well.
+//    dynamically (an atomic counter in the pool's control block; requests are
+//    numbered longest first and a request's items later rows first, so long
+//    items start early).  A Q tile packs 128/G new tokens x the G q heads of
+//    one kv group (row = token*G + head), so every K/V tile fetched from the
+//    pool feeds all G heads, and the two Q tiles of a CTA share each K/V tile.
 //  * One persistent CTA per SM, 12 warps:
 //      warp 0        TMA producer: Q tiles (3-D map over [T_new][Hq][d]) and
-//                    K/V tiles page by page (2-D map over the pool rows);
-//                    zeroes V rows past the end of the sequence.
+//                    K/V tiles page by page (2-D map over the pool rows) into
+//                    a 4-slot ring; the page copies of a tile are issued by
+//                    16 lanes, the next tile's pages looked up one tile
+//                    ahead; zeroes V rows past the end of the sequence.
 //      warp 1        TMEM owner; lane 0 issues Q tile 0's MMAs, lane 0 of
 //      warp 2        issues Q tile 1's:
 //                      S_i = Q_i K^T   (SS, both operands K-major, fp32 in TMEM)
 //                      O_i += P_i V    (TS: P_i read from TMEM, V MN-major)
-//                    Each issuer waits for its tile's inputs in chain order;
-//                    with one issuer per tile the tensor pipe interleaves the
-//                    two tiles' S -> softmax -> PV chains, so one tile's
-//                    softmax overlaps the other's MMAs.
+//                    Each issuer waits for its tile's inputs in chain order,
+//                    and tile 1's S(j) also waits until tile 0 has published
+//                    P(j), so the two softmax phases alternate and each
+//                    tile's MMAs fill the other's softmax time.
 //      warps 4-7     softmax of Q tile 0; warps 8-11 softmax of Q tile 1.
-//    Warps 0-3 give registers to the softmax warpgroups (setmaxnreg).
 //                    One thread per row: S row from TMEM, causal mask, online
 //                    softmax in the log2 domain against a running reference
 //                    max (the exact max of the row's first tile; recomputed,
 //                    with O and l rescaled, only if a later tile's terms
 //                    would approach fp32 overflow), P as bf16 written back
-//                    over S in TMEM, final 1/l normalisation and the bf16
-//                    store of O.
+//                    over S in TMEM (one arrival per warp), final 1/l
+//                    normalisation and the bf16 store of O.  They also
+//                    release the ring slots and Q tiles once they have seen
+//                    the MMAs that read them complete.
+//    Warps 0-3 give registers to the softmax warpgroups (setmaxnreg).
 //  * TMEM (512 columns): S0 [0,128) S1 [128,256) O0 [256,256+d) O1 [.., +d).
 //    P_i overwrites the first 64 columns of S_i.  Because P_i aliases S_i,
 //    S_i(j+1) is issued only after PV_i(j) has completed; the other Q
 //    tile's MMAs keep the tensor pipe fed meanwhile.
-//  * Every mbarrier wait is bounded; a timeout raises the CTA's abort flag,
-//    all roles leave their loops, in-flight copies and MMAs are drained, TMEM
-//    is freed and GC_ERR_TIMEOUT is recorded in the pool status word.
+//  * Decode mode (one new token per request): items are (request, kv head,
+//    range of K/V tiles); a request cut into several ranges writes fp32
+//    partials that a separate kernel merges.
+//  * Every mbarrier wait and spin is bounded; a timeout raises the CTA's
+//    abort flag, all roles leave their loops, in-flight copies and MMAs are
+//    drained, TMEM is freed and GC_ERR_TIMEOUT is recorded in the pool
+//    status word.
 #include <cmath>
 #include <mutex>
 
