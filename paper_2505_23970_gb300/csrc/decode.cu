@@ -41,19 +41,40 @@ __global__ void __launch_bounds__(D) decode_merge_kernel(const float* __restrict
                                                          int32_t max_splits, int32_t cap,
                                                          int32_t split_tiles,
                                                          __nv_bfloat16* __restrict__ out) {
+  // launched as a programmatic dependent of the attention kernel: the
+  // blocks may be resident before it ends, so wait for its results here
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int64_t head = blockIdx.x;
   const int b = static_cast<int>(head / Hq);
   const int nsplit = request_splits(__ldg(seq_lens + b), cap, split_tiles);
   if (nsplit <= 1) return;  // written by the attention kernel itself (or invalid)
   const int d = threadIdx.x;
-  const float* ml = ws + static_cast<int64_t>(batch) * Hq * max_splits * D + head * max_splits * 2;
+  const float2* ml = reinterpret_cast<const float2*>(
+      ws + static_cast<int64_t>(batch) * Hq * max_splits * D + head * max_splits * 2);
+  const float* o = ws + head * max_splits * D + d;
+  // independent loads, 8 ranges at a time
   float M = -INFINITY;
-  for (int s = 0; s < nsplit; ++s) M = fmaxf(M, ml[2 * s]);
+  for (int s0 = 0; s0 < nsplit; s0 += 8) {
+#pragma unroll
+    for (int t = 0; t < 8; ++t)
+      if (s0 + t < nsplit) M = fmaxf(M, __ldg(ml + s0 + t).x);
+  }
   float acc = 0.f, L = 0.f;
-  for (int s = 0; s < nsplit; ++s) {
-    const float f = ptx::ex2_approx(ml[2 * s] - M);
-    acc = fmaf(ws[(head * max_splits + s) * D + d], f, acc);
-    L = fmaf(ml[2 * s + 1], f, L);
+  for (int s0 = 0; s0 < nsplit; s0 += 8) {
+    float2 mls[8];
+    float os[8];
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      const bool in = s0 + t < nsplit;
+      mls[t] = in ? __ldg(ml + s0 + t) : make_float2(-INFINITY, 0.f);
+      os[t] = in ? __ldg(o + static_cast<int64_t>(s0 + t) * D) : 0.f;
+    }
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      const float f = ptx::ex2_approx(mls[t].x - M);
+      acc = fmaf(os[t], f, acc);
+      L = fmaf(mls[t].y, f, L);
+    }
   }
   out[head * D + d] = __float2bfloat16_rn(acc / L);
 }
@@ -103,15 +124,27 @@ gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_
   gc_status st = launch_attn_tc_decode(pool, args, dm, stream);
   if (st != GC_OK || sp.splits <= 1) return st;
   const unsigned heads = static_cast<unsigned>(a.batch) * static_cast<unsigned>(a.num_q_heads);
-  if (pool->cfg.head_dim == 128)
-    decode_merge_kernel<128><<<heads, 128, 0, stream>>>(
-        static_cast<const float*>(a.workspace), a.seq_lens, a.batch, a.num_q_heads, sp.splits,
-        static_cast<int32_t>(cap), sp.split_tiles, static_cast<__nv_bfloat16*>(a.out));
-  else
-    decode_merge_kernel<64><<<heads, 64, 0, stream>>>(
-        static_cast<const float*>(a.workspace), a.seq_lens, a.batch, a.num_q_heads, sp.splits,
-        static_cast<int32_t>(cap), sp.split_tiles, static_cast<__nv_bfloat16*>(a.out));
-  const cudaError_t e = cudaGetLastError();
+  // programmatic dependent launch: the merge grid is set up while the
+  // attention kernel drains, and waits for it with griddepcontrol.wait
+  cudaLaunchConfig_t lc = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.gridDim = dim3(heads);
+  lc.blockDim = dim3(pool->cfg.head_dim);
+  lc.dynamicSmemBytes = 0;
+  lc.stream = stream;
+  lc.attrs = attr;
+  lc.numAttrs = 1;
+  const float* wsp = static_cast<const float*>(a.workspace);
+  __nv_bfloat16* outp = static_cast<__nv_bfloat16*>(a.out);
+  const int32_t cap32 = static_cast<int32_t>(cap);
+  const cudaError_t e =
+      pool->cfg.head_dim == 128
+          ? cudaLaunchKernelEx(&lc, decode_merge_kernel<128>, wsp, a.seq_lens, a.batch,
+                               a.num_q_heads, sp.splits, cap32, sp.split_tiles, outp)
+          : cudaLaunchKernelEx(&lc, decode_merge_kernel<64>, wsp, a.seq_lens, a.batch,
+                               a.num_q_heads, sp.splits, cap32, sp.split_tiles, outp);
   if (e != cudaSuccess) return cuda_fail(e, "gc_paged_decode_attn: merge kernel launch");
   return GC_OK;
 }
