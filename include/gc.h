@@ -390,6 +390,14 @@ GC_API gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool,
                                       size_t workspace_bytes);
 
 /* Message of the last failing call on this thread ("" if none). */
+/* Test hook, not part of the method (the paper has no counterpart): launches
+ * one thread that waits on a device barrier nobody arrives at, with the same
+ * bounded wait every libgc kernel uses.  After its limit (about 1.5 s) the
+ * wait gives up, GC_ERR_TIMEOUT is recorded in the pool's status word (read
+ * with gc_kv_pool_check) and the kernel returns, so the timeout path can be
+ * exercised without hanging the GPU.  Errors: GC_ERR_INVALID_ARG, GC_ERR_CUDA. */
+GC_API gc_status gc_selftest_wait_timeout(gc_kv_pool* pool, cudaStream_t stream);
+
 GC_API const char* gc_last_error(void);
 
 /* Static name of a status code. */

@@ -39,7 +39,8 @@ EXPORTED = (
     "gc_kv_save_layers", "gc_kv_q8_chunk_bytes", "gc_kv_save_q8", "gc_kv_restore_q8",
     "gc_kv_append", "gc_prefix_prefill_attn",
     "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc",
-    "gc_paged_decode_workspace_bytes", "gc_paged_decode_attn", "gc_last_error",
+    "gc_paged_decode_workspace_bytes", "gc_paged_decode_attn", "gc_selftest_wait_timeout",
+    "gc_last_error",
     "gc_status_string",
 )
 
@@ -91,6 +92,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_prefix_prefill_attn.argtypes = attn
         lib.gc_prefix_prefill_attn_simt.argtypes = attn
         lib.gc_prefix_prefill_attn_noalloc.argtypes = attn
+        lib.gc_selftest_wait_timeout.argtypes = [vp, vp]
+        lib.gc_selftest_wait_timeout.restype = ctypes.c_int
         lib.gc_paged_decode_workspace_bytes.argtypes = [vp, i32, i32, i32]
         lib.gc_paged_decode_workspace_bytes.restype = ctypes.c_size_t
         lib.gc_paged_decode_attn.argtypes = [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32,
@@ -326,3 +329,7 @@ def gc_paged_decode_attn(q, pool, block_table, seq_lens, out, stream, layer: int
                                        max_blocks_per_seq, num_q_heads, softmax_scale,
                                        _addr(workspace), workspace_bytes),
            "gc_paged_decode_attn")
+
+
+def gc_selftest_wait_timeout(pool, stream=None) -> None:
+    _check(load().gc_selftest_wait_timeout(pool, _stream(stream)), "gc_selftest_wait_timeout")

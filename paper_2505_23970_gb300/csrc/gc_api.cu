@@ -6,6 +6,8 @@
 #include <cstring>
 #include <new>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "gc_internal.cuh"
 
 namespace {
@@ -31,6 +33,15 @@ gc_status cuda_fail(cudaError_t e, const char* what) {
 }  // namespace gc
 
 using gc::fail;
+
+// An NVTX range around every data-path call, so that profiler timelines show
+// which libgc call each kernel belongs to (no cost without a profiler).
+namespace {
+struct Range {
+  explicit Range(const char* name) { nvtxRangePushA(name); }
+  ~Range() { nvtxRangePop(); }
+};
+}  // namespace
 
 static bool pool_config_ok(const gc_pool_config* c) {
   return c && c->num_layers >= 1 && c->num_kv_heads >= 1 && c->head_dim >= 1 &&
@@ -96,6 +107,10 @@ gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, size_t dev
   void* owned = nullptr;
   if (!mem) {
     e = cudaMalloc(&mem, need);
+    if (e == cudaErrorMemoryAllocation) {
+      cudaGetLastError();  // not sticky: clear it so later calls are unaffected
+      return fail(GC_ERR_OOM, "gc_kv_pool_create: cudaMalloc of %zu bytes failed", need);
+    }
     if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_pool_create: cudaMalloc");
     owned = mem;
   }
@@ -387,6 +402,7 @@ gc_status save_q8_impl(const char* who, gc_kv_pool* pool, void* dst_img, const i
 
 gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
                         int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  Range range_("gc_kv_restore");
   return restore_impl("gc_kv_restore", pool, host_src, block_ids, n_blocks, 0,
                       pool ? pool->cfg.num_layers : 0, stream, dev_staging, flags);
 }
@@ -394,12 +410,14 @@ gc_status gc_kv_restore(gc_kv_pool* pool, const void* host_src, const int32_t* b
 gc_status gc_kv_restore_layers(gc_kv_pool* pool, const void* host_src, const int32_t* block_ids,
                                int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
                                cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  Range range_("gc_kv_restore_layers");
   return restore_impl("gc_kv_restore_layers", pool, host_src, block_ids, n_blocks, layer_begin,
                       layer_count, stream, dev_staging, flags);
 }
 
 gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
                      int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  Range range_("gc_kv_save");
   return save_impl("gc_kv_save", pool, host_dst, block_ids, n_blocks, 0,
                    pool ? pool->cfg.num_layers : 0, stream, dev_staging, flags);
 }
@@ -407,6 +425,7 @@ gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
 gc_status gc_kv_save_layers(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
                             int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
                             cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  Range range_("gc_kv_save_layers");
   return save_impl("gc_kv_save_layers", pool, host_dst, block_ids, n_blocks, layer_begin,
                    layer_count, stream, dev_staging, flags);
 }
@@ -419,6 +438,7 @@ size_t gc_kv_q8_chunk_bytes(const gc_pool_config* cfg) {
 gc_status gc_kv_save_q8(gc_kv_pool* pool, void* dst, const int32_t* block_ids, int32_t n_blocks,
                         int32_t layer_begin, int32_t layer_count, cudaStream_t stream,
                         void* dev_staging, uint32_t flags) {
+  Range range_("gc_kv_save_q8");
   return save_q8_impl("gc_kv_save_q8", pool, dst, block_ids, n_blocks, layer_begin, layer_count,
                       stream, dev_staging, flags);
 }
@@ -426,6 +446,7 @@ gc_status gc_kv_save_q8(gc_kv_pool* pool, void* dst, const int32_t* block_ids, i
 gc_status gc_kv_restore_q8(gc_kv_pool* pool, const void* src, const int32_t* block_ids,
                            int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
                            cudaStream_t stream, void* dev_staging, uint32_t flags) {
+  Range range_("gc_kv_restore_q8");
   return restore_q8_impl("gc_kv_restore_q8", pool, src, block_ids, n_blocks, layer_begin,
                          layer_count, stream, dev_staging, flags);
 }
@@ -434,6 +455,7 @@ gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v_new,
                        const int32_t* block_table, const int32_t* seq_lens, cudaStream_t stream,
                        int32_t layer, const int32_t* cu_new_lens, int32_t batch,
                        int32_t max_blocks_per_seq, int32_t total_new_tokens) {
+  Range range_("gc_kv_append");
   g_msg[0] = 0;
   if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_kv_append: pool is NULL");
   if (batch < 0 || total_new_tokens < 0 || max_blocks_per_seq < 0)
@@ -496,6 +518,7 @@ gc_status gc_prefix_prefill_attn(const void* q, const gc_kv_pool* pool, const in
                                  cudaStream_t stream, int32_t layer, const int32_t* cu_new_lens,
                                  int32_t batch, int32_t max_blocks_per_seq, int32_t num_q_heads,
                                  float softmax_scale, int32_t total_new_tokens) {
+  Range range_("gc_prefix_prefill_attn");
   g_msg[0] = 0;
   gc::AttnArgs a;
   bool noop;
@@ -512,6 +535,7 @@ gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool* pool,
                                          int32_t layer, const int32_t* cu_new_lens, int32_t batch,
                                          int32_t max_blocks_per_seq, int32_t num_q_heads,
                                          float softmax_scale, int32_t total_new_tokens) {
+  Range range_("gc_prefix_prefill_attn_noalloc");
   g_msg[0] = 0;
   gc::AttnArgs a;
   bool noop;
@@ -528,6 +552,7 @@ gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* pool,
                                       int32_t layer, const int32_t* cu_new_lens, int32_t batch,
                                       int32_t max_blocks_per_seq, int32_t num_q_heads,
                                       float softmax_scale, int32_t total_new_tokens) {
+  Range range_("gc_prefix_prefill_attn_simt");
   g_msg[0] = 0;
   gc::AttnArgs a;
   bool noop;
@@ -549,6 +574,7 @@ gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool, const int3
                                int32_t layer, int32_t batch, int32_t max_blocks_per_seq,
                                int32_t num_q_heads, float softmax_scale, void* workspace,
                                size_t workspace_bytes) {
+  Range range_("gc_paged_decode_attn");
   g_msg[0] = 0;
   const char* who = "gc_paged_decode_attn";
   if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
@@ -575,6 +601,12 @@ gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool, const int3
   const gc::DecodeArgs a{q, out, block_table, seq_lens, batch, max_blocks_per_seq, layer,
                          num_q_heads, softmax_scale, workspace, workspace_bytes};
   return gc::launch_decode(pool, a, stream);
+}
+
+gc_status gc_selftest_wait_timeout(gc_kv_pool* pool, cudaStream_t stream) {
+  g_msg[0] = 0;
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_selftest_wait_timeout: pool is NULL");
+  return gc::launch_selftest_timeout(pool, stream);
 }
 
 }  // extern "C"

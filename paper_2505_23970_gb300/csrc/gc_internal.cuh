@@ -58,6 +58,7 @@ gc_status launch_save_q8(const gc_kv_pool* pool, uint8_t* image, const int32_t* 
 gc_status launch_restore_q8(const gc_kv_pool* pool, const uint8_t* image,
                             const int32_t* block_ids, int32_t n_blocks, int32_t layer0,
                             int32_t layers, bool layer_major, cudaStream_t stream);
+gc_status launch_selftest_timeout(const gc_kv_pool* pool, cudaStream_t stream);
 gc_status launch_append(const gc_kv_pool* pool, const void* k_new, const void* v_new,
                         const int32_t* block_table, const int32_t* prefix_lens,
                         const int32_t* cu_new_lens, int32_t batch, int32_t max_blocks,

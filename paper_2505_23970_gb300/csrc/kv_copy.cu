@@ -233,6 +233,19 @@ __global__ void __launch_bounds__(256) append_kernel(const uint4* __restrict__ k
   }
 }
 
+// Self-test of the bounded device wait every libgc kernel uses: one thread
+// waits on a barrier nobody arrives at; the wait gives up after its cycle
+// limit and the kernel records GC_ERR_TIMEOUT and returns.
+__global__ void __launch_bounds__(32) selftest_timeout_kernel(int32_t* status) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  ptx::mbar_init(&bar, 1);
+  abort_flag = 0;
+  ptx::fence_barrier_init();
+  if (!ptx::mbar_wait(&bar, 0, &abort_flag)) record_error(status, GC_ERR_TIMEOUT);
+}
+
 int ilog2(int x) {
   int s = 0;
   while ((1 << s) < x) ++s;
@@ -240,6 +253,13 @@ int ilog2(int x) {
 }
 
 }  // namespace
+
+gc_status launch_selftest_timeout(const gc_kv_pool* pool, cudaStream_t stream) {
+  selftest_timeout_kernel<<<1, 32, 0, stream>>>(pool->status);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "gc_selftest_wait_timeout: launch");
+  return GC_OK;
+}
 
 gc_status launch_restore_bulk(const gc_kv_pool* pool, uint8_t* staging,
                               const int32_t* block_ids, int32_t n_blocks, int32_t layer0,

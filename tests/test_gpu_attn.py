@@ -265,3 +265,30 @@ def test_batch_beyond_sorted_ranking():
     n = rng.integers(0, 40, size=B)
     w = wl.custom("big-batch", B, 16, 4, 64, 16, P, n, seed=21)
     full_parity(w)
+
+
+def test_output_canaries_untouched():
+    """Prefill and decode write exactly their output rows: a canary after the
+    end of the output buffer keeps its bytes."""
+    import torch
+    w = wl.custom("canary", 3, 16, 2, 128, 16, [100, 0, 37], [20, 5, 1], seed=23)
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    rows = w.T_new * w.Hq * w.d
+    buf = torch.full((rows + 4096,), -7.0, dtype=torch.bfloat16, device="cuda")
+    out = buf[:rows].view(w.T_new, w.Hq, w.d)
+    db.attn(out=out)
+    assert db.check() == gcb.GC_OK
+    assert torch.all(buf[rows:] == -7.0)
+    wd = wl.custom("canary-dec", 3, 16, 2, 128, 16, [100, 0, 37], [1, 1, 1], seed=24)
+    dd = DeviceBatch(wd)
+    dd.restore()
+    dd.append()
+    rows = wd.B * wd.Hq * wd.d
+    buf = torch.full((rows + 4096,), -7.0, dtype=torch.bfloat16, device="cuda")
+    dd.decode(out=buf[:rows].view(wd.B, wd.Hq, wd.d))
+    assert dd.check() == gcb.GC_OK
+    assert torch.all(buf[rows:] == -7.0)
+    db.close()
+    dd.close()

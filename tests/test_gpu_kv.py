@@ -436,3 +436,34 @@ def test_q8_subnormal_and_large_groups_match_oracle():
     assert np.array_equal(b.pool_bits(), ref)
     db.close()
     b.close()
+
+
+# --------------------------------------------------------- failure handling
+def test_bounded_wait_times_out_and_reports():
+    """A device wait nobody satisfies gives up after its limit (~1.5 s), is
+    reported as GC_ERR_TIMEOUT, and leaves the context usable."""
+    import time
+    pool = gcb.KVPool.create(1, 1, 64, 16, 4)
+    t0 = time.time()
+    gcb.gc_selftest_wait_timeout(pool.handle)
+    assert pool.check() == gcb.GC_ERR_TIMEOUT
+    assert 0.5 < time.time() - t0 < 30
+    assert pool.check() == gcb.GC_OK  # read and cleared
+    pool.close()
+    w = wl.tiny()
+    db = DeviceBatch(w)
+    db.restore()
+    assert db.check() == gcb.GC_OK
+    assert np.array_equal(db.pool_bits(), oracle_pool(w, append=False))
+    db.close()
+
+
+def test_pool_create_out_of_memory_is_reported():
+    """A library-owned pool larger than the GPU fails with GC_ERR_OOM and
+    later allocations still succeed."""
+    cfg = gcb.make_config(1, 8, 128, 16, 2**24)  # 1 TiB of pages
+    with pytest.raises(gcb.GcError) as e:
+        gcb.gc_kv_pool_create(cfg)
+    assert e.value.status == gcb.GC_ERR_OOM
+    h = gcb.gc_kv_pool_create(gcb.make_config(1, 1, 64, 16, 4))
+    gcb.gc_kv_pool_destroy(h)
