@@ -99,8 +99,9 @@ typedef struct gc_pool_config {
 } gc_pool_config;
 
 /* Device bytes a pool of this shape needs: the KV planes
- * (L*2*num_pages*Hkv*ps*d*2 bytes) plus a 256-byte control block (device
- * status word, attention work counter).
+ * (L*2*num_pages*Hkv*ps*d*2 bytes, rounded up to 256) plus a 2048-byte
+ * control block (device status word, attention work counter, decode merge
+ * counters).
  * Returns 0 for an invalid configuration. */
 GC_API size_t gc_kv_pool_bytes(const gc_pool_config* cfg);
 
@@ -110,7 +111,7 @@ GC_API size_t gc_kv_pool_bytes(const gc_pool_config* cfg);
  *   dev_mem != NULL: caller-owned device memory of dev_bytes >=
  *                    gc_kv_pool_bytes(cfg) bytes, 256-byte aligned; the
  *                    library never frees it.
- * The KV planes are not initialised; the status word is cleared.
+ * The KV planes are not initialised; the control block is cleared.
  * Errors: GC_ERR_INVALID_ARG, GC_ERR_UNSUPPORTED (d or ps), GC_ERR_OOM,
  * GC_ERR_CUDA. */
 GC_API gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, size_t dev_bytes,
@@ -126,8 +127,9 @@ GC_API gc_status gc_kv_pool_data(const gc_kv_pool* pool, void** dev_ptr, size_t*
 /* Synchronise `stream`, then read and clear the pool's device status word:
  * *device_status receives GC_OK or the first error a kernel recorded since
  * the last check (GC_ERR_OUT_OF_RANGE for a bad device-side index,
- * GC_ERR_TIMEOUT for a device wait that gave up).  The return value reports
- * failures of the check itself (GC_ERR_CUDA). */
+ * GC_ERR_TIMEOUT for a device wait that gave up); after an error the
+ * control block's decode merge counters are cleared too.  The return value
+ * reports failures of the check itself (GC_ERR_CUDA). */
 GC_API gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t* device_status);
 
 /* gc_kv_restore flags */
@@ -369,14 +371,19 @@ GC_API gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* po
  *               written) and recorded as GC_ERR_OUT_OF_RANGE.
  *   block_table int32 [batch][max_blocks_per_seq], device; a bad page is
  *               skipped (its keys left out) and recorded.
- *   workspace   device scratch for requests split over several key ranges:
- *               gc_paged_decode_workspace_bytes(pool, batch,
- *               max_blocks_per_seq, num_q_heads) bytes (0: NULL is fine),
- *               owned by the caller, not used after the stream passes the
- *               call.  Calls sharing a workspace must not overlap on the GPU.
- * Runs on the prefill kernel's tensor-core path in a decode mode; calls on
- * one pool must not overlap on the GPU with each other or with
- * gc_prefix_prefill_attn (they share the pool's work counter).
+ *   workspace   device scratch for the partial results of requests split
+ *               over several CTAs: gc_paged_decode_workspace_bytes(pool,
+ *               batch, max_blocks_per_seq, num_q_heads) bytes (0: NULL is
+ *               fine), owned by the caller, not used after the stream passes
+ *               the call; no initial contents needed.  Calls sharing a
+ *               workspace must not overlap on the GPU.
+ * d = 128 with Hq/Hkv <= 16 runs on a transposed tensor-core kernel (keys on
+ * the 128-row side of the MMA) that gives every SM an equal share of the K/V
+ * tiles; a request cut between shares is combined by the last CTA to finish
+ * it.  Other shapes run on the prefill kernel's tensor-core path in a decode
+ * mode.  Calls on one pool must not overlap on the GPU with each other or
+ * with gc_prefix_prefill_attn (they share counters in the pool's control
+ * block).
  * Errors: GC_ERR_INVALID_ARG (null, unaligned, workspace too small),
  * GC_ERR_OUT_OF_RANGE (layer), GC_ERR_UNSUPPORTED (head grouping,
  * batch > 8192), GC_ERR_CUDA. */

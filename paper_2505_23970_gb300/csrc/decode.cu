@@ -7,16 +7,19 @@
 // with k_j, v_j read from the paged pool through block_table[b].
 //
 // Decode streams every cached K/V row once (2*Hkv*d*2 bytes per key) for
-// 4*G*d FLOP per key and kv head, so the bound is HBM.  The work runs on the
-// prefill kernel in decode mode (attn_tc.cu): its persistent CTAs stream the
-// pages through a TMA ring with bulk copies several tiles ahead, and the
-// tensor cores do the G-row products (a Q tile of G real rows: the padding
-// rows cost tensor time that the memory bound leaves idle anyway).  To fill
-// every SM, each request is cut into key ranges of 4 to 16 K/V tiles, chosen
-// per call from the batch and the block table's capacity (work items =
-// requests x kv heads x ranges); a request with several ranges
-// writes fp32 partials (O unnormalised, reference max in log2 units, sum)
-// and the merge kernel below combines them:
+// 4*G*d FLOP per key and kv head, so the bound is HBM.  Two kernels do it:
+//  - head_dim 128 with G <= 16 (the 70B-shaped layer): decode_tc.cu, the
+//    transposed tensor-core kernel (keys on the TMEM lanes), each CTA an equal
+//    share of all K/V tiles;
+//  - otherwise: the prefill kernel in decode mode (attn_tc.cu).  Its
+//    persistent CTAs stream the pages through a TMA ring, and the tensor cores
+//    do the G-row products (a Q tile of G real rows: the padding rows cost
+//    tensor time that the memory bound leaves idle).  To fill every SM, each
+//    request is cut into key ranges of 4 to 16 K/V tiles, chosen per call
+//    from the batch and the block table's capacity (work items = requests x
+//    kv heads x ranges); a request with several ranges writes fp32 partials
+//    (O unnormalised, reference max in log2 units, sum) and the merge kernel
+//    below combines them:
 //     out = sum_s O_s 2^(m_s - M) / sum_s l_s 2^(m_s - M),  M = max_s m_s.
 #include "gc_internal.cuh"
 #include "sm103_ptx.cuh"
@@ -104,20 +107,28 @@ DecodeSplit decode_split(const gc_kv_pool* pool, int32_t batch, int32_t max_bloc
   return d;
 }
 
+size_t decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch, int32_t max_blocks,
+                              int32_t num_q_heads) {
+  if (decode_tc_supported(pool, num_q_heads)) return decode_tc_workspace_bytes(pool, batch);
+  return decode_split(pool, batch, max_blocks, num_q_heads).workspace_bytes;
+}
+
 gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream) {
+  if (a.batch > 8192) return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: batch %d > 8192", a.batch);
+  if (static_cast<int64_t>(a.max_blocks) * pool->cfg.page_size > 2147483647LL)
+    return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: %lld-token block table",
+                static_cast<long long>(a.max_blocks) * pool->cfg.page_size);
+  if (decode_tc_supported(pool, a.num_q_heads)) return launch_decode_tc(pool, a, stream);
   const DecodeSplit sp = decode_split(pool, a.batch, a.max_blocks, a.num_q_heads);
   if (sp.workspace_bytes > 0 && (a.workspace == nullptr || a.workspace_bytes < sp.workspace_bytes))
     return fail(GC_ERR_INVALID_ARG,
                 "gc_paged_decode_attn: workspace of %zu bytes needed "
                 "(gc_paged_decode_workspace_bytes), got %zu",
                 sp.workspace_bytes, a.workspace_bytes);
-  if (a.batch > 8192) return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: batch %d > 8192", a.batch);
   const long long items = static_cast<long long>(a.batch) * pool->cfg.num_kv_heads * sp.splits;
   if (items > 2147483647LL)
     return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: %lld work items", items);
   const int64_t cap = static_cast<int64_t>(a.max_blocks) * pool->cfg.page_size;
-  if (cap > 2147483647LL)
-    return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: %lld-token block table", (long long)cap);
   AttnArgs args{a.q, a.out, a.block_table, nullptr, nullptr, nullptr, a.batch, a.max_blocks,
                 a.layer, a.num_q_heads, a.batch, a.softmax_scale};
   const DecodeMode dm{sp.split_tiles, sp.splits, a.seq_lens, static_cast<float*>(a.workspace)};

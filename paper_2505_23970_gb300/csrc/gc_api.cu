@@ -12,7 +12,9 @@
 
 namespace {
 thread_local char g_msg[512] = "";
-constexpr size_t kTrailer = 256;  // control block after the KV planes: status word, work counter
+// control block after the KV planes: status word, work counter (at 128 bytes),
+// the decode merge counters (from 256 bytes)
+constexpr size_t kTrailer = 2048;
 }  // namespace
 
 namespace gc {
@@ -123,7 +125,9 @@ gc_status gc_kv_pool_create(const gc_pool_config* cfg, void* dev_mem, size_t dev
   p->data = static_cast<uint8_t*>(mem);
   p->data_bytes = need - kTrailer;
   p->status = reinterpret_cast<int32_t*>(p->data + p->data_bytes);
-  p->work_counter = p->status + 32;  // 128 bytes into the 256-byte control block
+  p->work_counter = p->status + 32;    // 128 bytes into the control block
+  p->merge_counters = p->status + 64;  // 256 bytes in, kMergeCounters ints
+  static_assert(256 + gc::kMergeCounters * 4 <= kTrailer, "control block too small");
   p->owned = owned;
   p->device = dev;
   p->num_sms = sms;
@@ -168,6 +172,10 @@ gc_status gc_kv_pool_check(gc_kv_pool* pool, cudaStream_t stream, int32_t* devic
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e == cudaSuccess) e = cudaMemcpy(&host, pool->status, sizeof host, cudaMemcpyDeviceToHost);
   if (e == cudaSuccess) e = cudaMemset(pool->status, 0, sizeof host);
+  // a kernel that gave up on a wait may have left decode merge counters
+  // raised: after any error, clear them (nothing runs on the pool now)
+  if (e == cudaSuccess && host != GC_OK)
+    e = cudaMemset(pool->merge_counters, 0, gc::kMergeCounters * sizeof(int32_t));
   if (e == cudaSuccess) e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return gc::cuda_fail(e, "gc_kv_pool_check");
   *device_status = host;
@@ -566,7 +574,7 @@ gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* pool,
 size_t gc_paged_decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch,
                                        int32_t max_blocks_per_seq, int32_t num_q_heads) {
   if (!pool || batch <= 0 || max_blocks_per_seq <= 0 || num_q_heads <= 0) return 0;
-  return gc::decode_split(pool, batch, max_blocks_per_seq, num_q_heads).workspace_bytes;
+  return gc::decode_workspace_bytes(pool, batch, max_blocks_per_seq, num_q_heads);
 }
 
 gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool, const int32_t* block_table,

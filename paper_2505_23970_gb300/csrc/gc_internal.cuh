@@ -15,12 +15,15 @@ struct gc_kv_pool {
   size_t data_bytes;
   int32_t* status;        // device status word (first error recorded by a kernel)
   int32_t* work_counter;  // attention work-item counter (control block, zeroed per launch)
+  int32_t* merge_counters;  // [kMergeCounters] decode merge counters (control block, kept at 0)
   void* owned;            // cudaMalloc'd block, or nullptr if caller-owned
   int device;
   int num_sms;
 };
 
 namespace gc {
+
+constexpr int kMergeCounters = 448;  // ints after the first 256 bytes of the control block
 
 // Thread-local error message; returns `s` for convenient `return fail(...)`.
 gc_status fail(gc_status s, const char* fmt, ...);
@@ -106,5 +109,13 @@ struct DecodeSplit {
 DecodeSplit decode_split(const gc_kv_pool* pool, int32_t batch, int32_t max_blocks,
                          int32_t num_q_heads);
 gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream);
+// The transposed tensor-core decode kernel (decode_tc.cu): head_dim 128 and
+// at most 16 q heads per kv head.
+bool decode_tc_supported(const gc_kv_pool* pool, int32_t num_q_heads);
+size_t decode_tc_workspace_bytes(const gc_kv_pool* pool, int32_t batch);
+gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream);
+// Workspace bytes of a decode call on either path.
+size_t decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch, int32_t max_blocks,
+                              int32_t num_q_heads);
 
 }  // namespace gc

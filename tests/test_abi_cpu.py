@@ -39,7 +39,7 @@ def test_every_declared_symbol_is_exported(lib):
 def test_pool_bytes_arithmetic(lib):
     cfg = gcb.make_config(80, 8, 128, 16, 640)
     planes = 80 * 2 * 640 * 8 * 16 * 128 * 2
-    assert gcb.gc_kv_pool_bytes(cfg) == planes + 256
+    assert gcb.gc_kv_pool_bytes(cfg) == planes + 2048
     assert gcb.gc_kv_pool_bytes(gcb.make_config(0, 8, 128, 16, 10)) == 0
 
 

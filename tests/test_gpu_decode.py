@@ -53,12 +53,46 @@ def test_decode_mix_full():
     decode_parity(wl.decode_mix(seed=1))
 
 
-def test_unsplit_path_matches_oracle():
-    """Enough requests x kv heads to fill the GPU: no split, no workspace."""
+def test_wide_batch_of_short_contexts():
+    """160 requests of 2..161 keys (d 128): most (request, kv head) pairs lie
+    whole inside one CTA's share of the K/V tiles."""
     w = wl.custom("dec-wide", 160, 32, 8, 128, 16, list(range(1, 161)), [1] * 160, seed=3)
+    decode_parity(w)
+
+
+def test_unsplit_path_d64_needs_no_workspace():
+    """d 64 runs on the prefill kernel's decode mode: with enough requests x
+    kv heads to fill the GPU no request is split and no workspace is needed."""
+    w = wl.custom("dec-wide64", 160, 32, 8, 64, 16, list(range(1, 161)), [1] * 160, seed=3)
     assert gcb.gc_paged_decode_workspace_bytes(DeviceBatch(w).pool.handle, w.B, w.max_blocks,
                                                w.Hq) == 0
     assert decode_parity(w) == 0
+
+
+def test_decode_reference_max_raised_inside_a_piece():
+    """Keys aligned with q heads 0 and 1 (k = 12 q: scores ~190 in log2
+    units against ~4 elsewhere) in later tiles of a CTA's piece: each head's
+    reference max is raised once (O and the sums rescaled).  Without the
+    raise the probabilities (2^190) would overflow bf16; with a wrong rescale
+    of the sums the output would be off by the old keys' weight."""
+    w = wl.custom("dec-rescale", 8, 16, 2, 128, 16, [8999] * 8, [1] * 8, seed=31)
+    src = w.host_src()  # cached: the device batch and the oracle see the edit
+    q = wl.bf16_bits_to_f32(w.q())
+    # 8 x 2 pairs of 71 tiles over 152 CTAs: shares of 8 tiles, so the tiles
+    # 13 and 14 of request 0, kv head 0 are the 6th and 7th of one piece
+    for tile, h in ((13, 0), (14, 1)):
+        for j in range(tile * 128 + 3, tile * 128 + 9):
+            blk, row = divmod(j, w.ps)
+            src[blk, 0, 0, 0, row] = wl.f32_to_bf16_bits(12.0 * q[0, h])
+    decode_parity(w)
+
+
+def test_decode_batch_with_five_slot_ring():
+    """4600 requests: the unit table leaves room for five K/V ring slots
+    instead of six."""
+    ctx = np.random.default_rng(23).integers(1, 200, size=4600)
+    w = wl.custom("dec-5slot", 4600, 16, 2, 128, 16, ctx - 1, np.ones(4600, int), seed=23)
+    decode_parity(w)
 
 
 @pytest.mark.parametrize("G,d,ps", [(1, 128, 16), (2, 64, 32), (4, 64, 16), (8, 128, 64),
