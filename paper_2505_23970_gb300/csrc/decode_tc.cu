@@ -45,7 +45,12 @@ constexpr int kKeys = 128;                  // keys per K/V tile
 constexpr int kD = 128;                     // head dim
 constexpr int kN = 16;                      // q-head columns of S^T, O^T (G padded)
 constexpr int kTileBytes = kKeys * kD * 2;  // 32 KB
-constexpr int kHalfBytes = kKeys * 128;     // one 64-column block of a K/V tile
+// A K/V tile in shared memory: groups of 8 keys (2 KB), each the 8 rows of
+// columns 0-63 then the 8 rows of columns 64-127 (1 KB each, 128-byte
+// swizzled): key n, column half h at (n / 8) * 2048 + h * 1024 + (n % 8) * 128.
+// One 4-D TMA box per page lays a page's rows out this way.
+constexpr int kGroupBytes = 2048;
+constexpr int kAtomBytes = 1024;
 constexpr int kSmallHalf = kN * 128;        // one 64-element block of Q^T or P^T
 constexpr int kSmallBytes = 2 * kSmallHalf;
 constexpr uint32_t kIdescS = idesc_bf16_f32(128, kN, false, false);
@@ -131,8 +136,7 @@ __device__ void d_producer(uint8_t* smem_q, uint8_t* smem_kv, DBar& bar, const i
   uint32_t q_count = 0, kv_count = 0;
   uint32_t armed = 0, armed_par = 0, armed_q = 0, armed_q_par = 0;
   bool ok = true;
-  const uint32_t box_bytes = static_cast<uint32_t>(geo.ps) * 128;
-  const int pg = lane >> 1, hh = lane & 1;
+  const uint32_t box_bytes = static_cast<uint32_t>(geo.ps) * kD * 2;  // one page
 
   // lane p looks up page p of tile jt of piece pc (-2: no such page).  The
   // next tile's lookup (the next piece's first, at a piece's end) is issued
@@ -185,8 +189,7 @@ __device__ void d_producer(uint8_t* smem_q, uint8_t* smem_kv, DBar& bar, const i
       }
       if (page == -2) page = -1;
       const int good = __popc(__ballot_sync(0xffffffffu, page >= 0));
-      const int my_page = __shfl_sync(0xffffffffu, page, pg);
-      const bool issues = pg < kKeys / 16 && my_page >= 0;
+      const bool issues = page >= 0;  // lane p copies page p of the tile
 #pragma unroll 1
       for (int kv = 0; kv < 2; ++kv) {
         const int slot = kv_count % kStages;
@@ -194,13 +197,12 @@ __device__ void d_producer(uint8_t* smem_q, uint8_t* smem_kv, DBar& bar, const i
         if (!ok) break;
         uint8_t* dst = smem_kv + slot * kTileBytes;
         if (lane == 0)
-          mbar_arrive_expect_tx(&bar.kv_full[slot], static_cast<uint32_t>(good) * box_bytes * 2);
+          mbar_arrive_expect_tx(&bar.kv_full[slot], static_cast<uint32_t>(good) * box_bytes);
         __syncwarp();
         if (issues) {
           const int plane_row = (geo.layer * 2 + kv) * geo.num_pages;
-          const int row = (((plane_row + my_page) * geo.Hkv + w.g) << geo.ps_shift);
-          tma_load_2d(dst + hh * kHalfBytes + pg * box_bytes, map_kv, &bar.kv_full[slot],
-                      hh * 64, row);
+          const int row = (((plane_row + page) * geo.Hkv + w.g) << geo.ps_shift);
+          tma_load_4d(dst + lane * box_bytes, map_kv, &bar.kv_full[slot], 0, 0, 0, row >> 3);
         }
         armed |= 1u << slot;
         armed_par = (armed_par & ~(1u << slot)) | (((kv_count / kStages) & 1u) << slot);
@@ -250,9 +252,9 @@ __device__ void d_issuer(uint8_t* smem_q, uint8_t* smem_p, uint8_t* smem_kv, DBa
       const uint32_t k_addr = kv_smem + (ku % kStages) * kTileBytes;
 #pragma unroll
       for (int kk = 0; kk < kD / 16; ++kk) {
-        const uint32_t ka = k_addr + (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+        const uint32_t ka = k_addr + (kk >> 2) * kAtomBytes + (kk & 3) * 32;
         const uint32_t qa = q_addr + (kk >> 2) * kSmallHalf + (kk & 3) * 32;
-        mma_ss(tmem + kColS + (t & 1) * kN, sdesc_sw128(ka, 16, 1024), sdesc_sw128(qa, 16, 1024),
+        mma_ss(tmem + kColS + (t & 1) * kN, sdesc_sw128(ka, 16, kGroupBytes), sdesc_sw128(qa, 16, 1024),
                kIdescS, kk > 0 ? 1u : 0u);
       }
       mma_commit(&bar.s_full[t & 1]);
@@ -276,7 +278,7 @@ __device__ void d_issuer(uint8_t* smem_q, uint8_t* smem_p, uint8_t* smem_kv, DBa
 #pragma unroll
       for (int kk = 0; kk < kKeys / 16; ++kk) {
         const uint32_t pa = pt + (kk >> 2) * kSmallHalf + (kk & 3) * 32;
-        mma_ss(tmem + kColO, sdesc_sw128(v_addr + kk * 16 * 128, kHalfBytes, 1024),
+        mma_ss(tmem + kColO, sdesc_sw128(v_addr + kk * 2 * kGroupBytes, kAtomBytes, kGroupBytes),
                sdesc_sw128(pa, 16, 1024), kIdescPV, (t > 0 || kk > 0) ? 1u : 0u);
       }
       mma_commit(&bar.pv_done[pb]);
@@ -487,12 +489,13 @@ __device__ void d_softmax(uint8_t* smem_p, uint8_t* smem_kv, DBar& bar, float* x
         ok = mbar_wait(&bar.kv_full[vu % kStages], (vu / kStages) & 1, abortp);
         if (!ok) break;
         if (!key_valid) {
-          uint8_t* vrow = smem_kv + (vu % kStages) * kTileBytes + t_id * 128;
+          uint8_t* vrow = smem_kv + (vu % kStages) * kTileBytes + (t_id >> 3) * kGroupBytes +
+                          (t_id & 7) * 128;
 #pragma unroll
           for (int h = 0; h < 2; ++h)
 #pragma unroll
             for (int c = 0; c < 8; ++c)
-              reinterpret_cast<uint4*>(vrow + h * kHalfBytes)[c] = make_uint4(0, 0, 0, 0);
+              reinterpret_cast<uint4*>(vrow + h * kAtomBytes)[c] = make_uint4(0, 0, 0, 0);
         }
       }
       // this key's probabilities for the 16 head columns: column t_id of P^T
@@ -768,11 +771,14 @@ gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStre
       return fail(GC_ERR_CUDA, "gc_paged_decode_attn: q tensor map (CUresult %d)", (int)r);
   }
   {
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(kD), pool_rows};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(kD) * 2};
-    cuuint32_t box[2] = {64, static_cast<cuuint32_t>(geo.ps)};
-    cuuint32_t es[2] = {1, 1};
-    CUresult r = enc(&map_kv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool->data, dims, strides, box,
+    // pool rows of 128 columns seen as (column in half, row in group of 8,
+    // half, group): one box of (64, 8, 2, ps/8) is a page, laid out in
+    // shared memory group by group, half by half
+    cuuint64_t dims[4] = {64, 8, 2, pool_rows / 8};
+    cuuint64_t strides[3] = {static_cast<cuuint64_t>(kD) * 2, 128, 8 * static_cast<cuuint64_t>(kD) * 2};
+    cuuint32_t box[4] = {64, 8, 2, static_cast<cuuint32_t>(geo.ps / 8)};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    CUresult r = enc(&map_kv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, pool->data, dims, strides, box,
                      es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS)
