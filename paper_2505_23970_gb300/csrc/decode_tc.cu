@@ -25,7 +25,8 @@
 // order, are cut into one equal share per CTA, so every SM streams the same
 // number of bytes whatever the mix of context lengths.  A pair that a share
 // boundary cuts is done in pieces: each writes fp32 partials (O^T unscaled,
-// its reference max, its sum) and a small merge kernel combines them.
+// its reference max, its sum) and the last CTA to finish one of the pair's
+// pieces combines them (a counter per cut pair in the pool's control block).
 //
 // Roles: warp 0 TMA producer (Q^T rows, K/V pages into the ring), warp 1 TMEM
 // owner and MMA issuer (its commits also free the ring slots and Q^T), warp 2
