@@ -614,6 +614,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(&bar.tmem_base, kTmemCols);
     tmem_relinquish();
   }
+  // Launched as a programmatic dependent of the previous kernel on the
+  // stream: the set-up above touches only this CTA's shared memory and TMEM;
+  // inputs are read, and outputs written, once the previous grid is complete.
+  // The next kernel may in turn be set up on the SMs this grid frees.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   if (warp == 2) {
     // units per request (kv heads x K/V tiles), exclusive scan; a context
     // length outside [1, block table capacity] gets none and is recorded
@@ -702,10 +708,19 @@ gc_status launch_stages(const gc_kv_pool* pool, const DecodeArgs& a, const DGeom
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return cuda_fail(e, "gc_paged_decode_attn: smem attribute");
-  decode_tc_kernel<kStages><<<decode_grid(pool), kThreads, smem, stream>>>(
-      map_q, map_kv, a.block_table, a.seq_lens, static_cast<__nv_bfloat16*>(a.out), a.workspace,
-      geo, pool->status, pool->merge_counters);
-  e = cudaGetLastError();
+  cudaLaunchConfig_t lc = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.gridDim = dim3(decode_grid(pool));
+  lc.blockDim = dim3(kThreads);
+  lc.dynamicSmemBytes = smem;
+  lc.stream = stream;
+  lc.attrs = attr;
+  lc.numAttrs = 1;
+  e = cudaLaunchKernelEx(&lc, decode_tc_kernel<kStages>, map_q, map_kv, a.block_table, a.seq_lens,
+                         static_cast<__nv_bfloat16*>(a.out), a.workspace, geo, pool->status,
+                         pool->merge_counters);
   if (e != cudaSuccess) return cuda_fail(e, "gc_paged_decode_attn: launch");
   return GC_OK;
 }
