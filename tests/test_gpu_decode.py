@@ -177,3 +177,33 @@ def test_decode_batch_beyond_sorted_ranking():
     ctx = np.random.default_rng(22).integers(1, 600, size=1000)
     w = wl.custom("dec-big-batch", 1000, 16, 4, 64, 16, ctx - 1, np.ones(1000, int), seed=22)
     decode_parity(w)
+
+
+def test_merge_counters_cleared_after_an_error():
+    """A (request, kv head) pair cut between two SMs' shares is merged by the
+    last CTA to finish one of its pieces, counted in the pool's control block.
+    After any recorded error gc_kv_pool_check clears those counters: raise
+    them by hand, record an error (a bad page), check, and the next decode
+    matches the oracle again (with raised counters the merges would be
+    skipped or early)."""
+    import torch
+    w = wl.llama3_70b_decode(seed=4, B=2, context=3000)
+    db = DeviceBatch(w)
+    db.restore()
+    db.append()
+    control = db.pool.buffer[-2048:]
+    control[256:256 + 448 * 4].view(torch.int32).fill_(5)
+    bt = w.block_table.copy()
+    bt[1, 3] = -7
+    db.block_table = _i32(bt, "cuda")
+    db.decode()
+    assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
+    assert int(control[256:256 + 448 * 4].view(torch.int32).abs().sum()) == 0
+    db.block_table = _i32(w.block_table, "cuda")
+    db.decode()
+    assert db.check() == gcb.GC_OK
+    got = db.out_f64()
+    db.close()
+    ref = oracle.prefix_attn(w.q(), oracle_pool(w), 0, w.block_table, w.prefix_lens,
+                             w.cu_new_lens, w.scale)
+    assert_attn_close(got, ref, "decode after counters were cleared")
