@@ -96,7 +96,8 @@ def test_decode_batch_with_five_slot_ring():
 
 
 @pytest.mark.parametrize("G,d,ps", [(1, 128, 16), (2, 64, 32), (4, 64, 16), (8, 128, 64),
-                                    (16, 128, 128), (16, 64, 16), (8, 64, 128)])
+                                    (16, 128, 128), (16, 64, 16), (8, 64, 128), (2, 128, 16),
+                                    (4, 128, 32)])
 def test_decode_head_grouping_dims_and_page_sizes(G, d, ps):
     Hkv = 2
     ctx = [1, 17, 300, 1000, 64, 129]
