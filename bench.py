@@ -655,11 +655,11 @@ def bench_decode(args, pk):
         kv = int(w.total_lens.sum()) * w.Hkv * w.d * 2 * 2
         qo = 2 * w.B * w.Hq * w.d * 2
         gbs = (kv + qo) / (ms / 1e3) / 1e9
-        splits = gcb.gc_paged_decode_workspace_bytes(db.pool.handle, w.B, w.max_blocks, w.Hq)
+        ws = gcb.gc_paged_decode_workspace_bytes(db.pool.handle, w.B, w.max_blocks, w.Hq)
         res[w.name] = {"batch": w.B, "context_tokens": int(w.total_lens.sum()),
                        "us_per_step": ms * 1e3, "bytes_per_step": kv + qo, "gbs": gbs,
                        "frac_hbm": gbs / pk["hbm_gbs"], "tok_per_s": w.B / (ms / 1e3),
-                       "split": splits > 0, "device_status_ok": ok}
+                       "workspace_bytes": ws, "device_status_ok": ok}
         db.close()
     return res
 
