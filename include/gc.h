@@ -189,6 +189,36 @@ GC_API gc_status gc_kv_restore_layers(gc_kv_pool* pool, const void* host_src,
                                       int32_t layer_begin, int32_t layer_count,
                                       cudaStream_t stream, void* dev_staging, uint32_t flags);
 
+/* gc_kv_stage_layers flag: the images are the 8-bit cache tier's
+ * (chunks of gc_kv_q8_chunk_bytes instead of Hkv*ps*d*2 bytes) */
+#define GC_STAGE_Q8 8u
+
+/* The host -> device leg of a staged restore on its own (Sec. 2.2: the
+ * cached context KV is loaded from the cache tier before the prefill uses
+ * it): copies layers [layer_begin, layer_begin + layer_count) of a pinned
+ * host image into the same offsets of a device image of the same layout.
+ * The scatter into the pool is then gc_kv_restore_layers (or
+ * gc_kv_restore_q8) with GC_RESTORE_SRC_DEVICE on that device image.  With
+ * the two legs apart, a serving loop can issue every layer's copy on a copy
+ * stream, back to back so the host link never waits for a scatter, and run
+ * each layer's scatter on the compute stream right before that layer's
+ * append and attention, once the layer's copy has landed (an event).
+ *   host_src   the whole image, pinned host memory: bf16
+ *              [n_blocks][L][2][Hkv][ps][d], or with GC_STAGE_Q8 the 8-bit
+ *              image [n_blocks][L][2][gc_kv_q8_chunk_bytes]; with
+ *              GC_RESTORE_LAYER_MAJOR the layer-major layouts [L][n_blocks]...
+ *   dev_image  device memory of the whole image's size (16-byte aligned);
+ *              only the chosen layers' slices are written.
+ *   Nothing is launched: the copies are cudaMemcpyAsync (one per call for a
+ *   layer-major image or all layers; one cudaMemcpy2DAsync of the strided
+ *   slices otherwise).  The pool is only read for its geometry.
+ * Errors: GC_ERR_INVALID_ARG (null/negative, unknown flags, host_src not
+ * pinned, dev_image misaligned), GC_ERR_OUT_OF_RANGE (layer range outside
+ * [0, L)), GC_ERR_CUDA. */
+GC_API gc_status gc_kv_stage_layers(const gc_kv_pool* pool, const void* host_src,
+                                    void* dev_image, int32_t n_blocks, int32_t layer_begin,
+                                    int32_t layer_count, cudaStream_t stream, uint32_t flags);
+
 /* gc_kv_save flags */
 #define GC_SAVE_DST_DEVICE 1u /* host_dst is device memory (gather only) */
 #define GC_SAVE_VECTOR 2u     /* 16-byte vector-copy kernel instead of bulk copies */
@@ -307,8 +337,13 @@ GC_API gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v
  *   total_new_tokens  T_new = cu_new_lens[batch], passed from the host; it
  *               bounds every q / out row access.  A request whose rows would
  *               pass it is skipped and recorded as GC_ERR_OUT_OF_RANGE.
+ *   Size limit: the kernel numbers its work items (a kv head of a request
+ *   and 256 of its q rows) with 32-bit ints, so T_new * (Hq/Hkv) + 256 and
+ *   Hkv * (T_new * (Hq/Hkv) / 256 + batch) + 2 * (SM count) must both stay
+ *   at or below 2^31 - 1; a larger call fails with GC_ERR_UNSUPPORTED before
+ *   anything is launched.
  * Errors: GC_ERR_INVALID_ARG, GC_ERR_OUT_OF_RANGE (layer),
- * GC_ERR_UNSUPPORTED (head grouping), GC_ERR_CUDA. */
+ * GC_ERR_UNSUPPORTED (head grouping, size limit), GC_ERR_CUDA. */
 GC_API gc_status gc_prefix_prefill_attn(const void* q, const gc_kv_pool* pool, const int32_t* block_table,
                                  const int32_t* prefix_lens, const int32_t* new_lens, void* out,
                                  cudaStream_t stream, int32_t layer, const int32_t* cu_new_lens,
@@ -327,11 +362,15 @@ GC_API gc_status gc_prefix_prefill_attn(const void* q, const gc_kv_pool* pool, c
  *   that loads the library holds until the process exits.  The first call on
  *   a device looks up the array's device address (cudaGetSymbolAddress) with
  *   that device current; make that first call before any stream capture.
+ *   The address is kept per device and CUDA context: after a device reset
+ *   (cudaDeviceReset) the next call finds a new context and looks it up
+ *   again, so that call too should come before any stream capture.
  *   Each call clears the counter with a stream-ordered memset.
  *   All calls share the array, on every pool: two calls that overlap on the
  *   GPU race on it and give wrong results.  Serialise them.
- *   Limit: at most 2^31 - 1 work items per call, i.e.
- *   Hkv * (total_new_tokens * (Hq/Hkv) / 256 + batch) <= 2^31 - 1; larger
+ *   Limit: the size limit of gc_prefix_prefill_attn, i.e. at most
+ *   2^31 - 1 - 2 * (SM count) work items,
+ *   Hkv * (total_new_tokens * (Hq/Hkv) / 256 + batch), per call; larger
  *   calls fail with GC_ERR_UNSUPPORTED before anything is launched.
  *   The current device must be the pool's device (GC_ERR_INVALID_ARG).
  * Other errors as gc_prefix_prefill_attn. */

@@ -505,14 +505,17 @@ int oracle_full_causal_attn(const uint16_t *q, const uint16_t *k, const uint16_t
     pthread_t th[256];
     dense_arg a[256];
     if (nthreads > 256) nthreads = 256;
+    int started = 0, st = OR_OK;
     for (int t = 0; t < nthreads; ++t) {
         a[t] = (dense_arg){q, k, v, T, Hq, Hkv, d, scale, out, Hq * t / nthreads,
                            Hq * (t + 1) / nthreads, OR_OK};
-        if (nthreads == 1) dense_worker(&a[t]);
-        else pthread_create(&th[t], NULL, dense_worker, &a[t]);
+        if (nthreads == 1) { dense_worker(&a[t]); continue; }
+        /* only threads that were created are joined */
+        if (pthread_create(&th[t], NULL, dense_worker, &a[t]) != 0) { st = OR_ERR_OOM; break; }
+        started++;
     }
-    if (nthreads > 1)
-        for (int t = 0; t < nthreads; ++t) pthread_join(th[t], NULL);
+    for (int t = 0; t < started; ++t) pthread_join(th[t], NULL);
+    if (st != OR_OK) return st;
     for (int t = 0; t < nthreads; ++t)
         if (a[t].status) return a[t].status;
     return OR_OK;

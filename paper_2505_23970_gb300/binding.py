@@ -32,11 +32,13 @@ GC_SAVE_DST_DEVICE = 1
 GC_SAVE_VECTOR = 2
 GC_RESTORE_LAYER_MAJOR = 4
 GC_SAVE_LAYER_MAJOR = 4
+GC_STAGE_Q8 = 8
 
 EXPORTED = (
     "gc_kv_pool_bytes", "gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
     "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
-    "gc_kv_save_layers", "gc_kv_q8_chunk_bytes", "gc_kv_save_q8", "gc_kv_restore_q8",
+    "gc_kv_save_layers", "gc_kv_stage_layers", "gc_kv_q8_chunk_bytes", "gc_kv_save_q8",
+    "gc_kv_restore_q8",
     "gc_kv_append", "gc_prefix_prefill_attn",
     "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc",
     "gc_paged_decode_workspace_bytes", "gc_paged_decode_attn", "gc_selftest_wait_timeout",
@@ -83,6 +85,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_kv_save.argtypes = [vp, vp, vp, i32, vp, vp, u32]
         lib.gc_kv_restore_layers.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
         lib.gc_kv_save_layers.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
+        lib.gc_kv_stage_layers.argtypes = [vp, vp, vp, i32, i32, i32, vp, u32]
         lib.gc_kv_q8_chunk_bytes.argtypes = [ctypes.POINTER(gc_pool_config)]
         lib.gc_kv_q8_chunk_bytes.restype = ctypes.c_size_t
         lib.gc_kv_save_q8.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, u32]
@@ -100,7 +103,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                                              ctypes.c_float, vp, ctypes.c_size_t]
         for f in ("gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
                   "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
-                  "gc_kv_save_layers", "gc_kv_save_q8", "gc_kv_restore_q8", "gc_kv_append",
+                  "gc_kv_save_layers", "gc_kv_stage_layers", "gc_kv_save_q8", "gc_kv_restore_q8",
+                  "gc_kv_append",
                   "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt",
                   "gc_prefix_prefill_attn_noalloc", "gc_paged_decode_attn"):
             getattr(lib, f).restype = ctypes.c_int
@@ -206,6 +210,13 @@ def gc_kv_save_layers(pool, host_dst, block_ids, n_blocks: int, layer_begin: int
     _check(load().gc_kv_save_layers(pool, _addr(host_dst), _addr(block_ids), n_blocks,
                                     layer_begin, layer_count, _stream(stream), _addr(dev_staging),
                                     flags), "gc_kv_save_layers")
+
+
+def gc_kv_stage_layers(pool, host_src, dev_image, n_blocks: int, layer_begin: int,
+                       layer_count: int, stream=None, flags: int = 0) -> None:
+    _check(load().gc_kv_stage_layers(pool, _addr(host_src), _addr(dev_image), n_blocks,
+                                     layer_begin, layer_count, _stream(stream), flags),
+           "gc_kv_stage_layers")
 
 
 def gc_kv_q8_chunk_bytes(cfg: gc_pool_config) -> int:

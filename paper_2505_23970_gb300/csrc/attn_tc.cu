@@ -774,6 +774,41 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0 && bar.abort_flag) record_error(status, GC_ERR_TIMEOUT);
 }
 
+}  // namespace
+
+// The work items of one call are numbered with 32-bit ints and handed out by
+// a 32-bit counter that every CTA (or CTA pair) raises once more after the
+// last item: the items, plus two claims per CTA of margin, must stay below
+// 2^31, and so must the q rows of the batch (T_new * G), from which the
+// kernel derives each request's item count.  Host-side bound, checked
+// before anything is launched.
+gc_status check_item_bound(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode* dm,
+                           int grid) {
+  const long long hkv = pool->cfg.num_kv_heads;
+  const long long G = a.num_q_heads / hkv;
+  const long long rows = static_cast<long long>(a.total_new_tokens) * G;
+  long long items;
+  if (dm) {
+    // a request's keys (at most max_blocks * ps) cut into ranges of split_tiles tiles
+    const long long tiles =
+        (static_cast<long long>(a.max_blocks) * pool->cfg.page_size + kTileN - 1) / kTileN;
+    const long long per_req = (tiles + dm->split_tiles - 1) / dm->split_tiles;
+    items = hkv * a.batch * per_req;
+  } else {
+    // sum_b ceil(n_b * G / 256) <= T_new * G / 256 + batch
+    items = hkv * (rows / (2 * kTileM) + a.batch);
+  }
+  const long long limit = 2147483647LL - 2LL * grid;
+  if (rows + 2 * kTileM > 2147483647LL || items > limit)
+    return fail(GC_ERR_UNSUPPORTED,
+                "attention: up to %lld work items (%lld q rows) exceed what the 32-bit work "
+                "counter can hand out (%lld)",
+                items, rows, limit);
+  return GC_OK;
+}
+
+namespace {
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (!fn) {
@@ -791,6 +826,8 @@ template <int D>
 gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
                  int* work_counter, const DecodeMode* dm = nullptr) {
   using C = Cfg<D>;
+  gc_status bound = check_item_bound(pool, a, dm, pool->num_sms);
+  if (bound != GC_OK) return bound;
   auto enc = encode_fn();
   if (!enc) return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: cuTensorMapEncodeTiled unavailable");
   const auto& cfg = pool->cfg;
@@ -890,21 +927,55 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 
-// Device address of the static scratch on `device`, looked up once per device
-// with that device current (host code cannot use the symbol itself: it only
-// names a host-side stand-in).
+// Unique id of the calling thread's current CUDA context, 0 if there is none
+// or the driver cannot say (the lookup below is then repeated on every call).
+unsigned long long current_context_id() {
+  static PFN_cuCtxGetCurrent_v4000 get_cur = nullptr;
+  static PFN_cuCtxGetId_v12000 get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_cur = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_cur || !get_id || get_cur(&ctx) != CUDA_SUCCESS || !ctx) return 0;
+  if (get_id(ctx, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// Device address of the static scratch on `device`, with that device
+// current.  Host code cannot use the symbol itself (it only names a
+// host-side stand-in), so the address is looked up with
+// cudaGetSymbolAddress: once per device and context.  A device reset
+// (cudaDeviceReset) makes a new context with the library's module loaded
+// again, so the next call looks the address up again instead of using a
+// stale one.
 gc_status noalloc_scratch(int device, int** out) {
   static std::mutex mu;
   static int* addr[kMaxDevices] = {};
+  static unsigned long long ctx_of[kMaxDevices] = {};
   if (device < 0 || device >= kMaxDevices)
     return fail(GC_ERR_UNSUPPORTED, "gc_prefix_prefill_attn_noalloc: device %d >= %d", device,
                 kMaxDevices);
   std::lock_guard<std::mutex> lock(mu);
-  if (!addr[device]) {
+  const unsigned long long ctx = current_context_id();
+  if (!addr[device] || ctx == 0 || ctx != ctx_of[device]) {
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_attn_noalloc_scratch);
     if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn_noalloc: cudaGetSymbolAddress");
     addr[device] = static_cast<int*>(p);
+    // the lookup made the context current if it was not yet
+    ctx_of[device] = ctx ? ctx : current_context_id();
   }
   *out = addr[device];
   return GC_OK;
@@ -914,16 +985,6 @@ gc_status noalloc_scratch(int device, int** out) {
 
 gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a,
                                  cudaStream_t stream) {
-  // the items of a call must fit the 32-bit counter: Hkv * sum ceil(n_b*G/256)
-  const long long G = a.num_q_heads / pool->cfg.num_kv_heads;
-  const long long items_max =
-      static_cast<long long>(pool->cfg.num_kv_heads) *
-      (static_cast<long long>(a.total_new_tokens) * G / (2 * kTileM) + a.batch);
-  if (items_max > 2147483647LL)
-    return fail(GC_ERR_UNSUPPORTED,
-                "gc_prefix_prefill_attn_noalloc: up to %lld work items exceed the 2^31-1 the "
-                "static work counter can hand out",
-                items_max);
   int device = -1;
   cudaError_t e = cudaGetDevice(&device);
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn_noalloc: cudaGetDevice");
@@ -931,8 +992,12 @@ gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a,
     return fail(GC_ERR_INVALID_ARG,
                 "gc_prefix_prefill_attn_noalloc: current device %d is not the pool's device %d",
                 device, pool->device);
+  // the item bound is checked again by the launch; checking it first keeps a
+  // refused call from touching the device at all
+  gc_status st = check_item_bound(pool, a, nullptr, pool->num_sms);
+  if (st != GC_OK) return st;
   int* counter = nullptr;
-  const gc_status st = noalloc_scratch(device, &counter);
+  st = noalloc_scratch(device, &counter);
   if (st != GC_OK) return st;
   if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, counter);
   return launch<64>(pool, a, stream, counter);

@@ -423,6 +423,35 @@ gc_status gc_kv_restore_layers(gc_kv_pool* pool, const void* host_src, const int
                       layer_count, stream, dev_staging, flags);
 }
 
+gc_status gc_kv_stage_layers(const gc_kv_pool* pool, const void* host_src, void* dev_image,
+                             int32_t n_blocks, int32_t layer_begin, int32_t layer_count,
+                             cudaStream_t stream, uint32_t flags) {
+  Range range_("gc_kv_stage_layers");
+  g_msg[0] = 0;
+  const char* who = "gc_kv_stage_layers";
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (n_blocks < 0) return fail(GC_ERR_INVALID_ARG, "%s: n_blocks < 0", who);
+  if (flags & ~(GC_RESTORE_LAYER_MAJOR | GC_STAGE_Q8))
+    return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
+  gc_status st = check_layers(who, pool, layer_begin, layer_count);
+  if (st != GC_OK) return st;
+  if (n_blocks == 0 || layer_count == 0) return GC_OK;
+  if (!host_src || !dev_image) return fail(GC_ERR_INVALID_ARG, "%s: image is NULL", who);
+  if (reinterpret_cast<uintptr_t>(dev_image) % 16)
+    return fail(GC_ERR_INVALID_ARG, "%s: dev_image not 16-byte aligned", who);
+  cudaPointerAttributes attr;
+  cudaError_t e = cudaPointerGetAttributes(&attr, host_src);
+  if (e != cudaSuccess || attr.type != cudaMemoryTypeHost) {
+    cudaGetLastError();
+    return fail(GC_ERR_INVALID_ARG, "%s: host_src must be pinned host memory", who);
+  }
+  const size_t layer_bytes =
+      2 * ((flags & GC_STAGE_Q8) ? gc::q8_chunk_bytes(pool->cfg) : gc::page_bytes(pool->cfg));
+  return copy_layers(who, dev_image, host_src, n_blocks, pool->cfg.num_layers, layer_begin,
+                     layer_count, layer_bytes, (flags & GC_RESTORE_LAYER_MAJOR) != 0,
+                     cudaMemcpyHostToDevice, stream);
+}
+
 gc_status gc_kv_save(gc_kv_pool* pool, void* host_dst, const int32_t* block_ids,
                      int32_t n_blocks, cudaStream_t stream, void* dev_staging, uint32_t flags) {
   Range range_("gc_kv_save");

@@ -90,6 +90,11 @@ struct DecodeMode {
 };
 gc_status launch_attn_tc_decode(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode& dm,
                                 cudaStream_t stream);
+// Host-side bound of the attention kernels' 32-bit work numbering (items and
+// q rows of one call, with a margin of two claims per CTA of `grid`):
+// GC_ERR_UNSUPPORTED before anything is launched when a call could pass it.
+gc_status check_item_bound(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode* dm,
+                           int grid);
 
 // Paged decode attention (one new token per request), split-KV.
 struct DecodeArgs {

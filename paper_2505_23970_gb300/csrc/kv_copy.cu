@@ -106,12 +106,14 @@ __global__ void __launch_bounds__(32) restore_bulk_kernel(uint8_t* __restrict__ 
   int issued = 0;
   while (issued < kStages && issue(issued)) ++issued;
   bool ok = true;
+  int consumed = 0;  // loads [0, consumed) have landed
   for (int k = 0; k < issued; ++k) {
     const int slot = k % kStages;
     if (!ptx::mbar_wait(&full[slot], (k / kStages) & 1, &abort_flag)) {
       ok = false;
       break;
     }
+    consumed = k + 1;
     ptx::bulk_store(dst_of[slot], smem + slot * kPiece, bytes_of[slot]);
     ptx::bulk_commit();
     if (k >= 1) {
@@ -123,8 +125,9 @@ __global__ void __launch_bounds__(32) restore_bulk_kernel(uint8_t* __restrict__ 
   ptx::bulk_wait_all();
   if (!ok) {
     record_error(status, GC_ERR_TIMEOUT);
-    // let loads still in flight land before the CTA exits (bounded)
-    for (int k = 0; k < issued; ++k) {
+    // let the loads still in flight land before the CTA exits (bounded):
+    // only loads [consumed, issued), at most kStages, one per slot
+    for (int k = consumed; k < issued; ++k) {
       int dummy = 0;
       ptx::mbar_wait(&full[k % kStages], (k / kStages) & 1, &dummy);
     }

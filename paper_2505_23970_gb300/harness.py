@@ -168,13 +168,20 @@ class LayerStack:
     of that layer are restored, the layer's new K/V appended and its
     attention run.
 
-    ``run(pipelined=True)`` issues every layer's restore
-    (gc_kv_restore_layers, one layer per call) on a side stream with one
-    CUDA event per layer; the main stream waits for layer l's event before
-    layer l's append and attention, so the restore of later layers overlaps
-    the attention of earlier ones.  ``run(pipelined=False)`` restores all
-    layers first (one gc_kv_restore) and then computes layer by layer on one
-    stream.  Q and the new tokens' K/V are the same tensors for every layer
+    ``run(pipelined=True)`` splits each layer's restore into its two legs:
+    every layer's host -> device copy (gc_kv_stage_layers) is issued up front
+    on a copy stream, back to back, each followed by a CUDA event, so the
+    host link never waits for a kernel; the main stream waits for layer l's
+    event, then runs layer l's scatter (gc_kv_restore_layers from the device
+    image), append and attention.  The copies of later layers overlap the
+    compute of earlier ones, and the scatter, which needs the SMs the
+    attention of the previous layer holds, sits where it is needed anyway.
+    ``run(pipelined=True, schedule="side-restore")`` is the simpler schedule
+    it replaced: one staged gc_kv_restore_layers per layer (copy + scatter)
+    on a side stream, so each copy waits behind the previous layer's
+    scatter, which waits for the attention holding the SMs.
+    ``run(pipelined=False)`` restores all layers first (one gc_kv_restore)
+    and then computes layer by layer on one stream.  Q and the new tokens' K/V are the same tensors for every layer
     (inputs of the attention step, not produced here); the cached pages
     differ per layer.  Only streams, events and buffers are handled here:
     every byte is moved or computed by libgc."""
@@ -209,6 +216,7 @@ class LayerStack:
         self.outs = [torch.empty((w.T_new, w.Hq, w.d), dtype=torch.bfloat16, device=device)
                      for _ in range(n_out)]
         self.side = torch.cuda.Stream(device=device)
+        self.copy = torch.cuda.Stream(device=device)
         self.events = [torch.cuda.Event() for _ in range(w.L)]
 
     def use_q8(self):
@@ -236,6 +244,30 @@ class LayerStack:
             gcb.gc_kv_restore_layers(self.pool.handle, self.host_src, self.block_ids,
                                      self.n_blocks, l, 1, stream, self.staging, self.flags)
 
+    def stage_layer(self, l, stream):
+        """Host -> device copy of layer l's slice of the cached image."""
+        if not self.n_blocks:
+            return
+        if self.q8:
+            gcb.gc_kv_stage_layers(self.pool.handle, self.q8_host, self.q8_staging, self.n_blocks,
+                                   l, 1, stream, gcb.GC_RESTORE_LAYER_MAJOR | gcb.GC_STAGE_Q8)
+        else:
+            gcb.gc_kv_stage_layers(self.pool.handle, self.host_src, self.staging, self.n_blocks,
+                                   l, 1, stream, self.flags)
+
+    def scatter_layer(self, l, stream):
+        """Layer l's pages from the device image into the pool."""
+        if not self.n_blocks:
+            return
+        if self.q8:
+            gcb.gc_kv_restore_q8(self.pool.handle, self.q8_staging, self.block_ids, self.n_blocks,
+                                 l, 1, stream, None,
+                                 gcb.GC_RESTORE_SRC_DEVICE | gcb.GC_RESTORE_LAYER_MAJOR)
+        else:
+            gcb.gc_kv_restore_layers(self.pool.handle, self.staging, self.block_ids,
+                                     self.n_blocks, l, 1, stream, None,
+                                     gcb.GC_RESTORE_SRC_DEVICE | self.flags)
+
     def restore_all(self, stream):
         if self.n_blocks and self.q8:
             gcb.gc_kv_restore_q8(self.pool.handle, self.q8_host, self.block_ids, self.n_blocks,
@@ -253,23 +285,48 @@ class LayerStack:
                                    self.outs[l % len(self.outs)], stream, l, self.cu_new_lens,
                                    w.B, w.max_blocks, w.Hq, w.scale, w.T_new)
 
-    def run(self, pipelined: bool = True):
+    def run(self, pipelined: bool = True, schedule: str = "copy-stream", trace=None):
         """Restore + append + attention of every layer, issued on the current
-        stream (and, when pipelined, the side stream for the restores)."""
+        stream (and, when pipelined, the copy or side stream).  `trace`, a
+        dict, receives per-layer timing events of the copy-stream schedule:
+        'copied' (copy stream, after layer l's copy), 'scattered' (main, after
+        layer l's scatter) and 'computed' (main, after layer l's attention)."""
         import torch
         main = torch.cuda.current_stream(self.device)
+        L = self.w.L
         if not pipelined:
             self.restore_all(main)
-            for l in range(self.w.L):
+            for l in range(L):
                 self.prefill_layer(l, main)
             return
-        self.side.wait_stream(main)  # the restores may not pass earlier work on main
-        for l in range(self.w.L):
-            self.restore_layer(l, self.side)
-            self.events[l].record(self.side)
-        for l in range(self.w.L):
+        if schedule == "side-restore":
+            self.side.wait_stream(main)  # the restores may not pass earlier work on main
+            for l in range(L):
+                self.restore_layer(l, self.side)
+                self.events[l].record(self.side)
+            for l in range(L):
+                main.wait_event(self.events[l])
+                self.prefill_layer(l, main)
+            return
+        if schedule != "copy-stream":
+            raise ValueError(schedule)
+        if trace is not None:
+            for k in ("copied", "scattered", "computed"):
+                trace[k] = [torch.cuda.Event(enable_timing=True) for _ in range(L)]
+        self.copy.wait_stream(main)  # the copies may not pass earlier work on main
+        for l in range(L):
+            self.stage_layer(l, self.copy)
+            self.events[l].record(self.copy)
+            if trace is not None:
+                trace["copied"][l].record(self.copy)
+        for l in range(L):
             main.wait_event(self.events[l])
+            self.scatter_layer(l, main)
+            if trace is not None:
+                trace["scattered"][l].record(main)
             self.prefill_layer(l, main)
+            if trace is not None:
+                trace["computed"][l].record(main)
 
     def prefill_only(self):
         """Append + attention of every layer (the compute half alone)."""

@@ -225,11 +225,14 @@ def test_large_score_jumps_take_the_exact_path():
     full_parity(w)
 
 
-def test_layer_pipelined_schedule_matches_serial_and_oracle():
-    """Restoring layer l on a side stream (one gc_kv_restore_layers call per
-    layer, event-chained to the layer's append and attention) leaves the
-    pool and every layer's output bit-identical to restoring all layers
-    first; the pool equals the oracle's and the outputs match its attention."""
+@pytest.mark.parametrize("schedule", ["copy-stream", "side-restore"])
+def test_layer_pipelined_schedule_matches_serial_and_oracle(schedule):
+    """Restoring layer l in a pipeline with the layers' compute — each layer's
+    copy on a copy stream (gc_kv_stage_layers) and its scatter right before
+    its append and attention, or one staged gc_kv_restore_layers call per
+    layer on a side stream — leaves the pool and every layer's output
+    bit-identical to restoring all layers first; the pool equals the
+    oracle's and the outputs match its attention."""
     import torch
     from paper_2505_23970_gb300.harness import LayerStack
     w = wl.custom("layers", 2, 16, 2, 128, 16, [700, 33], [64, 130], seed=14)
@@ -237,7 +240,7 @@ def test_layer_pipelined_schedule_matches_serial_and_oracle():
     serial = LayerStack(w, keep_outputs=True)
     serial.run(pipelined=False)
     piped = LayerStack(w, keep_outputs=True)
-    piped.run(pipelined=True)
+    piped.run(pipelined=True, schedule=schedule)
     assert serial.check() == gcb.GC_OK and piped.check() == gcb.GC_OK
     for a, b in zip(serial.outs, piped.outs):
         assert torch.equal(a.view(torch.int16), b.view(torch.int16))
@@ -254,6 +257,32 @@ def test_layer_pipelined_schedule_matches_serial_and_oracle():
         assert_attn_close(piped.outs[l].to(torch.float64).cpu().numpy(), ref, f"layer {l}")
     serial.close()
     piped.close()
+
+
+def test_layer_pipeline_from_the_8bit_tier_matches_whole_restore():
+    """With the cache tier holding the 8-bit image, the copy-stream pipeline
+    (gc_kv_stage_layers with GC_STAGE_Q8, then gc_kv_restore_q8 of one layer
+    from the device image) leaves the same pool and outputs, bit for bit, as
+    dequantising every layer at once before the compute."""
+    import torch
+    from paper_2505_23970_gb300.harness import LayerStack
+    w = wl.custom("layers-q8", 2, 16, 2, 128, 16, [520, 47], [40, 129], seed=15)
+    w.L = 3
+    stacks = []
+    for pipelined in (False, True):
+        st = LayerStack(w, keep_outputs=True)
+        st.restore_all(None)
+        st.use_q8()
+        st.pool.planes().view(torch.int16).fill_(0x7FC0)
+        st.run(pipelined=pipelined)
+        assert st.check() == gcb.GC_OK
+        stacks.append(st)
+    serial, piped = stacks
+    assert np.array_equal(serial.pool_bits(), piped.pool_bits())
+    for a, b in zip(serial.outs, piped.outs):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    for st in stacks:
+        st.close()
 
 
 def test_batch_beyond_sorted_ranking():
@@ -292,3 +321,30 @@ def test_output_canaries_untouched():
     assert torch.all(buf[rows:] == -7.0)
     db.close()
     dd.close()
+
+
+def test_work_item_bound_refused_before_launch():
+    """A call whose 32-bit work numbering could overflow (q rows or work items
+    near 2^31) is refused on the host with GC_ERR_UNSUPPORTED: the dummy
+    arrays below are far too small and are never touched."""
+    import torch
+    dummy = torch.zeros(1024, dtype=torch.int32, device="cuda")
+    # 16 q heads per kv head x 2^27 new tokens = 2^31 q rows
+    pool = gcb.KVPool.create(1, 64, 64, 16, 1)
+    with pytest.raises(gcb.GcError) as e:
+        gcb.gc_prefix_prefill_attn(dummy, pool.handle, dummy, dummy, dummy, dummy, None, 0, dummy,
+                                   1, 1, 64 * 16, 0.125, 2**27)
+    assert e.value.status == gcb.GC_ERR_UNSUPPORTED
+    assert "work items" in gcb.gc_last_error()
+    assert pool.check() == gcb.GC_OK
+    pool.close()
+    # q rows within bounds, but 512 kv heads x (2^31 - 512) / 256 row groups
+    # give more work items than the counter can hand out
+    pool = gcb.KVPool.create(1, 512, 64, 16, 1)
+    with pytest.raises(gcb.GcError) as e:
+        gcb.gc_prefix_prefill_attn(dummy, pool.handle, dummy, dummy, dummy, dummy, None, 0, dummy,
+                                   1, 1, 512, 0.125, 2**31 - 512)
+    assert e.value.status == gcb.GC_ERR_UNSUPPORTED
+    assert "work items" in gcb.gc_last_error()
+    assert pool.check() == gcb.GC_OK
+    pool.close()

@@ -50,6 +50,31 @@ def test_noalloc_matches_regular_entry_point_on_two_calls():
     db.close()
 
 
+def test_noalloc_allocates_no_device_memory():
+    """The pool here lives in memory the caller owns (KVPool.create passes a
+    torch buffer as dev_mem).  After the first call, which looks up the static
+    scratch's address once, further calls leave the device's free memory
+    unchanged: nothing is allocated, not even by the CUDA runtime."""
+    import torch
+    w = wl.custom("noalloc-mem", 3, 16, 2, 128, 16, [260, 0, 31], [70, 129, 2], seed=22)
+    db = DeviceBatch(w)
+    db.run()
+    assert db.check() == gcb.GC_OK
+    ref = db.out_f64()
+    out = torch.full_like(db.out, float("nan"))
+    _call_noalloc(db, out)                      # first call: symbol lookup
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    for _ in range(3):
+        _call_noalloc(db, out)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0, f"free device memory changed by {free0 - free1} bytes"
+    assert db.check() == gcb.GC_OK
+    assert_attn_close(out.to(torch.float64).cpu().numpy(), ref, "noalloc, caller-owned pool")
+    db.close()
+
+
 def test_noalloc_rejects_calls_beyond_its_limit():
     """Up to 2^31 - 1 work items per call fit the static work counter; a call
     that could need more is refused before anything is launched."""
