@@ -902,7 +902,7 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
 }  // namespace
 
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
-  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter);
+  if (pool->cfg.head_dim == 128) return launch_attn_tc2(pool, a, stream, pool->work_counter);
   return launch<64>(pool, a, stream, pool->work_counter);
 }
 
@@ -999,7 +999,7 @@ gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a,
   int* counter = nullptr;
   st = noalloc_scratch(device, &counter);
   if (st != GC_OK) return st;
-  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, counter);
+  if (pool->cfg.head_dim == 128) return launch_attn_tc2(pool, a, stream, counter);
   return launch<64>(pool, a, stream, counter);
 }
 

@@ -1,0 +1,851 @@
+// Prefix-reuse causal GQA attention, head_dim 128, on pairs of SMs
+// (tcgen05 cta_group::2).
+//
+// Operation (Sec. 2.2: the cached context KV and the new tokens' KV are
+// processed together; Sec. 2.1: prefill): for request b, q head h, new row
+// i < n_b and kv head g = h / G,
+//     O[b,i,h] = sum_{j <= P_b + i} softmax_j(scale * q . k_j) v_j
+// with keys read from the paged pool through block_table[b].
+//
+// Design
+//  * A work item is (request b, kv head g, 256 q rows); a q row is
+//    (token, head) with row = token*G + head, so one item covers 256/G new
+//    tokens x the G q heads of kv group g and every K/V tile fetched from
+//    the pool feeds all of them.  Items are handed out by a counter, longest
+//    request first, later rows first within a request.
+//  * Each item runs on a CTA pair (a cluster of two, one CTA per SM).  The
+//    MMAs are M = 256 products issued by one thread of the even CTA: each
+//    SM holds 128 of the q rows (its half of A and of every product) and
+//    half of every K/V tile (B is split by columns between the two SMs), so
+//    each SM fetches 32 KB of K/V per 128-key step for 128 rows x 128 keys
+//    of work.
+//      S = Q K^T    M 256, N 128 keys, K 128 (both operands K-major, smem)
+//      O += P V     M 256, N 128 (d), K 128 keys (P from tensor memory,
+//                   V MN-major in smem)
+//  * Tensor memory per SM: S double-buffered [0,128) [128,256), O [256,384),
+//    P double-buffered [384,448) [448,512) (bf16 pairs).  P has its own
+//    columns, so S(t+1) is computed while the softmax works on S(t); the
+//    issuer's order S(t+1), PV(t) keeps the tensor pipe fed from one chain.
+//  * Warps per CTA:
+//      0     TMA producer: this SM's Q half, then per 128-key step its K
+//            half (64 keys x 128 d) and V half (128 keys x 64 d) into a ring
+//            of 16 KB slots; page boxes issued by several lanes at once.
+//      1     tensor-memory owner (both CTAs allocate together); lane 0 of
+//            the even CTA issues every MMA of the pair.
+//      2     item table at start-up.
+//      3     forwarder: waits for this SM's copies to land, zeroes V rows
+//            past the end of the sequence (their P is 0 but 0 * NaN is
+//            NaN), and reports the slot as full to the even CTA.
+//      4-7   softmax, one thread per q row (= tensor-memory lane): S row from
+//            tensor memory, causal mask, p = 2^(s*scale*log2 e - m) against a
+//            reference max (the exact max of the row's first tile; raised,
+//            with O and l rescaled, only if a later tile would approach fp32
+//            overflow), P as bf16 into tensor memory, final 1/l and the bf16
+//            store of O.  Thread 0 also frees ring slots once the products
+//            that read them are complete.
+//  * Every wait and spin is bounded; a CTA that gives up raises its own and
+//    its peer's abort flag, every role leaves its loop, copies and MMAs in
+//    flight are drained, both CTAs meet at a cluster barrier, tensor memory
+//    is freed and GC_ERR_TIMEOUT is recorded.
+#include <cmath>
+
+#include "gc_internal.cuh"
+#include "sm103_ptx.cuh"
+
+namespace gc {
+namespace {
+
+using namespace ptx;
+
+constexpr int kD = 128;
+constexpr int kThreads = 256;
+constexpr int kRows = 128;            // q rows per SM
+constexpr int kKeys = 128;            // keys per K/V step
+constexpr int kStages = 8;            // ring slots of 16 KB (K and V halves alternate)
+constexpr int kSlotBytes = 16384;
+constexpr int kQBytes = kRows * kD * 2;  // 32 KB: two 64-column blocks of 128 rows
+constexpr int kSortMax = 512;
+constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
+constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
+constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
+constexpr float kSpecLimit = 9.223372036854775808e18f;  // 2^63, as in the single-SM kernel
+// consumers of the work-item ring per CTA: forwarder + 4 softmax warps +
+// (even CTA) the MMA issuer or (odd CTA) the producer
+constexpr int kItemConsumers = 2 * 6;
+
+struct Geom2 {
+  int32_t batch, Hq, Hkv, G, ps, ps_shift, num_pages, max_blocks, layer, total_new;
+  int32_t box_rows, box_shift;  // TMA box height min(ps, 64) and its log2
+  float scale_log2;
+};
+
+struct Bars2 {
+  uint64_t q_landed[2];       // this CTA's Q half copied (tx)
+  uint64_t q_full[2];         // even CTA: both Q halves landed (2 forwards)
+  uint64_t q_empty[2];        // the item's last S product done (commit, both CTAs)
+  uint64_t landed[kStages];   // this CTA's ring slot copied (tx)
+  uint64_t full[kStages];     // even CTA: both halves of the slot ready (2 forwards)
+  uint64_t empty[kStages];    // this CTA's slot read by its products (softmax thread 0)
+  uint64_t s_full[2];         // S buffer computed (commit, both CTAs)
+  uint64_t s_free[2];         // even CTA: S buffer read by all 8 softmax warps
+  uint64_t p_full[2];         // even CTA: P buffer written by all 8 softmax warps
+  uint64_t pv_done[2];        // PV product from a P buffer done (commit, both CTAs)
+  uint64_t o_free;            // even CTA: O read by the epilogue (8 warps)
+  uint64_t item_full[2];      // work-item ring, written by the even CTA's producer
+  uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
+  uint64_t drain;             // even CTA: the issuer's last commit
+  int item_slot[2];
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+// Shared::cluster addresses of the barriers that live in the even CTA, and
+// of the peer's abort flag and item slots.
+struct Remote {
+  uint32_t q_full, full, s_free, p_full, o_free, item_empty, item_full, item_slot, abort_peer;
+};
+
+struct Item2 {
+  int b, g, P, n, cu, T;
+  int tok0;      // first token of this CTA's 128 rows
+  int nt;        // K/V steps of the item (both CTAs)
+  bool rows_ok;  // this CTA has at least one valid row
+};
+
+__device__ __forceinline__ void decode_item2(int it, const int* item_start, const Geom2& geo,
+                                             uint32_t rank, const int32_t* __restrict__ prefix_lens,
+                                             const int32_t* __restrict__ new_lens,
+                                             const int32_t* __restrict__ cu_new_lens, Item2& w) {
+  int lo = 0, hi = geo.batch;  // last p with item_start[p] <= it
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (item_start[mid] <= it) lo = mid; else hi = mid;
+  }
+  const int b = geo.batch <= kSortMax ? static_cast<int>(
+                    reinterpret_cast<const int16_t*>(item_start + geo.batch + 1)[lo])
+                                       : lo;
+  const int local = it - item_start[lo];
+  const int tiles = (item_start[lo + 1] - item_start[lo]) / geo.Hkv;
+  const int tile = tiles - 1 - local / geo.Hkv;  // later rows (more keys) first
+  w.b = b;
+  w.g = local % geo.Hkv;
+  w.P = __ldg(prefix_lens + b);
+  w.n = __ldg(new_lens + b);
+  w.cu = __ldg(cu_new_lens + b);
+  w.T = w.P + w.n;
+  const int rows = w.n * geo.G;
+  const int r0 = tile * 2 * kRows;
+  w.tok0 = (r0 + static_cast<int>(rank) * kRows) / geo.G;
+  w.rows_ok = r0 + static_cast<int>(rank) * kRows < rows;
+  const int r_last = min(r0 + 2 * kRows - 1, rows - 1);  // last valid row of the item
+  const int kend = w.P + r_last / geo.G + 1;              // keys [0, kend) reach some row
+  w.nt = (kend + kKeys - 1) / kKeys;
+}
+
+// Read item k of the ring (every consumer thread); the caller releases the
+// slot with one arrival per consumer warp on the even CTA's item_empty.
+__device__ __forceinline__ int read_item2(Bars2& bar, uint32_t k, volatile int* abortp,
+                                          bool& ok) {
+  ok = mbar_wait_cluster(&bar.item_full[k & 1], (k >> 1) & 1, abortp);
+  return ok ? *reinterpret_cast<volatile int*>(&bar.item_slot[k & 1]) : -1;
+}
+
+// The same for a whole warp (every lane reads the item; the lanes agree).
+__device__ __forceinline__ int read_item2_warp(Bars2& bar, uint32_t k, volatile int* abortp,
+                                               bool& ok) {
+  const int it = read_item2(bar, k, abortp, ok);
+  ok = __all_sync(0xffffffffu, ok);
+  return it;
+}
+
+// A wait done by every lane of a warp: the lanes agree on the outcome, so a
+// timeout seen by one lane alone cannot split the warp before a warp-wide
+// (.sync.aligned) instruction.
+__device__ __forceinline__ bool wait_warp(uint64_t* bar, uint32_t parity, volatile int* abortp) {
+  const bool ok = mbar_wait_cluster(bar, parity, abortp);
+  return __all_sync(0xffffffffu, ok);
+}
+
+__device__ __forceinline__ void raise_abort(Bars2& bar, const Remote& rm) {
+  *reinterpret_cast<volatile int*>(&bar.abort_flag) = 1;
+  st_cluster_u32(rm.abort_peer, 1u);
+}
+
+// ------------------------------------------------------------------ producer
+__device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar,
+                          const Remote& rm, const int* item_start, int total_items,
+                          const Geom2& geo, const CUtensorMap* map_q, const CUtensorMap* map_kv,
+                          const int32_t* __restrict__ block_table,
+                          const int32_t* __restrict__ prefix_lens,
+                          const int32_t* __restrict__ new_lens,
+                          const int32_t* __restrict__ cu_new_lens, int32_t* status,
+                          int* work_counter) {
+  const int lane = threadIdx.x & 31;
+  volatile int* abortp = &bar.abort_flag;
+  uint32_t use = 0;                      // ring uses so far (K at 2t, V at 2t+1)
+  uint32_t armed = 0, armed_par = 0;     // per slot: a copy in flight, and its phase parity
+  int armed_q = -1;
+  bool ok = true;
+  const uint32_t box_bytes = static_cast<uint32_t>(geo.box_rows) * 128;
+  const int boxes_k = (64 >> geo.box_shift) * 2;  // K half: 64 keys x 2 column blocks
+  const int boxes_v = kKeys >> geo.box_shift;     // V half: 128 keys x 1 column block
+
+  for (uint32_t k = 0; ok; ++k) {
+    int it = -1;
+    if (rank == 0) {
+      // claim the next item and publish it to both CTAs
+      const int s = k & 1;
+      ok = wait_warp(&bar.item_empty[s], ((k >> 1) & 1) ^ 1, abortp);
+      if (!ok) break;
+      if (lane == 0) {
+        it = atomicAdd(work_counter, 1);
+        if (it >= total_items) it = -1;
+        bar.item_slot[s] = it;
+        st_cluster_u32(rm.item_slot + 4 * s, static_cast<uint32_t>(it));
+        mbar_arrive(&bar.item_full[s]);
+        mbar_arrive_cluster(rm.item_full + 8 * s);
+      }
+      it = __shfl_sync(0xffffffffu, it, 0);
+    } else {
+      it = read_item2_warp(bar, k, abortp, ok);
+      if (!ok) break;
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
+    }
+    if (it < 0) break;
+    Item2 w;
+    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
+    // ---- this CTA's Q half: 128 rows = 128/G tokens x G heads, two column blocks
+    const int qb = k & 1;
+    ok = wait_warp(&bar.q_empty[qb], ((k >> 1) & 1) ^ 1, abortp);
+    if (!ok) break;
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&bar.q_landed[qb], kQBytes);
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+        tma_load_3d(smem_q + qb * kQBytes + h * (kRows * 128), map_q, &bar.q_landed[qb], h * 64,
+                    w.g * geo.G, w.cu + w.tok0);
+    }
+    armed_q = qb | (((k >> 1) & 1) << 1);
+    // ---- K/V halves, step by step
+    const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
+    for (int j = 0; ok && j < w.nt; ++j) {
+      const int key0 = j * kKeys;
+#pragma unroll 1
+      for (int kv = 0; kv < 2; ++kv) {
+        const int slot = use % kStages;
+        ok = wait_warp(&bar.empty[slot], ((use / kStages) & 1) ^ 1, abortp);
+        if (!ok) break;
+        // box `lane`: K: column block lane & 1, rows of chunk lane >> 1 of
+        // this CTA's 64 keys; V: column block `rank`, chunk lane of 128 keys
+        const int nbox = kv == 0 ? boxes_k : boxes_v;
+        int kc = 0, col = 0, dst = 0;
+        if (kv == 0) {
+          kc = key0 + static_cast<int>(rank) * 64 + (lane >> 1) * geo.box_rows;
+          col = (lane & 1) * 64;
+          dst = (lane & 1) * (64 * 128) + (lane >> 1) * geo.box_rows * 128;
+        } else {
+          kc = key0 + lane * geo.box_rows;
+          col = static_cast<int>(rank) * 64;
+          dst = lane * geo.box_rows * 128;
+        }
+        int row = -1;
+        if (lane < nbox && kc < w.T) {
+          const int blk = kc >> geo.ps_shift;
+          const int page = blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
+          if (page < 0 || page >= geo.num_pages) {
+            record_error(status, GC_ERR_OUT_OF_RANGE);
+          } else {
+            const int plane_row = (geo.layer * 2 + kv) * geo.num_pages;
+            row = (((plane_row + page) * geo.Hkv + w.g) << geo.ps_shift) + (kc & (geo.ps - 1));
+          }
+        }
+        const int good = __popc(__ballot_sync(0xffffffffu, row >= 0));
+        if (lane == 0) mbar_arrive_expect_tx(&bar.landed[slot], static_cast<uint32_t>(good) * box_bytes);
+        __syncwarp();
+        if (row >= 0) tma_load_2d(smem_kv + slot * kSlotBytes + dst, map_kv, &bar.landed[slot], col, row);
+        armed |= 1u << slot;
+        armed_par = (armed_par & ~(1u << slot)) | (((use / kStages) & 1u) << slot);
+        ++use;
+      }
+    }
+  }
+  if (!ok && lane == 0) {
+    // let this CTA's copies still in flight land before it exits (bounded,
+    // ignores the abort flag); a slot's copy may already have been waited
+    // for, in which case its phase has completed and the wait returns at once
+    int no_abort = 0;
+    if (armed_q >= 0) mbar_wait(&bar.q_landed[armed_q & 1], (armed_q >> 1) & 1, &no_abort);
+    for (int s = 0; s < kStages; ++s)
+      if (armed & (1u << s)) mbar_wait(&bar.landed[s], (armed_par >> s) & 1u, &no_abort);
+  }
+}
+
+// ----------------------------------------------------------------- forwarder
+// Reports each of this CTA's copies to the even CTA once it has landed (and,
+// for a V half that ends past the sequence, once its tail rows are zero).
+__device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
+                           const int* item_start, const Geom2& geo,
+                           const int32_t* __restrict__ prefix_lens,
+                           const int32_t* __restrict__ new_lens,
+                           const int32_t* __restrict__ cu_new_lens) {
+  const int lane = threadIdx.x & 31;
+  volatile int* abortp = &bar.abort_flag;
+  uint32_t use = 0;
+  bool ok = true;
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = read_item2_warp(bar, k, abortp, ok);
+    if (!ok) break;
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
+    if (it < 0) break;
+    Item2 w;
+    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
+    const int qb = k & 1;
+    ok = wait_warp(&bar.q_landed[qb], (k >> 1) & 1, abortp);
+    if (!ok) break;
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(rm.q_full + 8 * qb);
+    for (int j = 0; ok && j < w.nt; ++j) {
+      for (int kv = 0; kv < 2; ++kv) {
+        const int slot = use % kStages;
+        ok = wait_warp(&bar.landed[slot], (use / kStages) & 1, abortp);
+        if (!ok) break;
+        const int nkeys = min(kKeys, w.T - j * kKeys);
+        if (kv == 1 && nkeys < kKeys) {
+          // V rows [nkeys, 128) of this CTA's column block (128 bytes each)
+          uint4* z = reinterpret_cast<uint4*>(smem_kv + slot * kSlotBytes + nkeys * 128);
+          for (int e = lane; e < (kKeys - nkeys) * 8; e += 32) z[e] = make_uint4(0, 0, 0, 0);
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(rm.full + 8 * slot);
+        ++use;
+      }
+    }
+  }
+}
+
+// -------------------------------------------------------------- MMA issuer
+// One thread of the even CTA.  Per step t of an item: S(t) once K(t) is in
+// and the softmax has read S(t-2) out of the buffer; then PV(t-1) once the
+// softmax has written P(t-1) and V(t-1) is in.
+__device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
+                        uint32_t tmem, const int* item_start, const Geom2& geo,
+                        const int32_t* __restrict__ prefix_lens,
+                        const int32_t* __restrict__ new_lens,
+                        const int32_t* __restrict__ cu_new_lens) {
+  volatile int* abortp = &bar.abort_flag;
+  const uint32_t q_smem = smem_addr(smem_q), kv_smem = smem_addr(smem_kv);
+  uint32_t u = 0;     // global step counter
+  bool ok = true;
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = read_item2(bar, k, abortp, ok);
+    if (!ok) break;
+    mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
+    if (it < 0) break;
+    Item2 w;
+    decode_item2(it, item_start, geo, 0, prefix_lens, new_lens, cu_new_lens, w);
+    const int qb = k & 1;
+    ok = mbar_wait_cluster(&bar.q_full[qb], (k >> 1) & 1, abortp);
+    if (!ok) break;
+    const uint32_t u_first = u;
+    const uint32_t q_addr = q_smem + qb * kQBytes;
+    // PV of step v (an earlier step of this item)
+    auto pv = [&](uint32_t v) -> bool {
+      const uint32_t pb = v & 1;
+      if (!mbar_wait_cluster(&bar.p_full[pb], (v >> 1) & 1, abortp)) return false;
+      const uint32_t vu = 2 * v + 1;
+      if (!mbar_wait_cluster(&bar.full[vu % kStages], (vu / kStages) & 1, abortp)) return false;
+      const bool first = v == u_first;
+      if (first && k > 0 && !mbar_wait_cluster(&bar.o_free, (k - 1) & 1, abortp)) return false;
+      tc_fence_after();
+      const uint32_t v_addr = kv_smem + (vu % kStages) * kSlotBytes;
+#pragma unroll
+      for (int kk = 0; kk < kKeys / 16; ++kk)
+        mma2_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
+                sdesc_sw128(v_addr + kk * 16 * 128, kSlotBytes, 1024), kIdescPV,
+                (!first || kk > 0) ? 1u : 0u);
+      mma2_commit_mc(&bar.pv_done[pb], 0x3);
+      return true;
+    };
+    for (int j = 0; j < w.nt; ++j, ++u) {
+      const uint32_t sb = u & 1;
+      const uint32_t ku = 2 * u;
+      ok = mbar_wait_cluster(&bar.full[ku % kStages], (ku / kStages) & 1, abortp);
+      if (ok && u >= 2) ok = mbar_wait_cluster(&bar.s_free[sb], ((u - 2) >> 1) & 1, abortp);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t k_addr = kv_smem + (ku % kStages) * kSlotBytes;
+#pragma unroll
+      for (int kk = 0; kk < kD / 16; ++kk) {
+        const uint32_t qo = (kk >> 2) * (kRows * 128) + (kk & 3) * 32;
+        const uint32_t ko = (kk >> 2) * (64 * 128) + (kk & 3) * 32;
+        mma2_ss(tmem + kColS + sb * 128, sdesc_sw128(q_addr + qo, 16, 1024),
+                sdesc_sw128(k_addr + ko, 16, 1024), kIdescQK, kk > 0);
+      }
+      mma2_commit_mc(&bar.s_full[sb], 0x3);
+      if (j == w.nt - 1) mma2_commit_mc(&bar.q_empty[qb], 0x3);
+      if (j > 0 && !pv(u - 1)) {
+        ok = false;
+        break;
+      }
+    }
+    if (!ok) break;
+    if (w.nt > 0 && !pv(u - 1)) ok = false;
+  }
+  // every MMA this thread issued must be complete before tensor memory is freed
+  mma2_commit_mc(&bar.drain, 0x1);
+  int no_abort = 0;
+  mbar_wait(&bar.drain, 0, &no_abort);
+}
+
+// ------------------------------------------------------------------ softmax
+__device__ __forceinline__ float tile_max2(const uint32_t (&sr)[4][32]) {
+  float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+  for (int c = 0; c < 4; ++c)
+#pragma unroll
+    for (int e = 0; e < 32; e += 8) {
+      mx[0] = fmax3(mx[0], __uint_as_float(sr[c][e + 0]), __uint_as_float(sr[c][e + 1]));
+      mx[1] = fmax3(mx[1], __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
+      mx[2] = fmax3(mx[2], __uint_as_float(sr[c][e + 4]), __uint_as_float(sr[c][e + 5]));
+      mx[3] = fmax3(mx[3], __uint_as_float(sr[c][e + 6]), __uint_as_float(sr[c][e + 7]));
+    }
+  return fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
+}
+
+// p = 2^(s * scale*log2(e) - m) for one row of the tile, written to tensor
+// memory at tP as bf16 pairs (64 columns); returns sum p (fp32).
+__device__ __forceinline__ float tile_exp2(const uint32_t (&sr)[4][32], uint32_t tP,
+                                           float scale_log2, float m) {
+  const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
+  const uint64_t nm2 = f2_pack(-m, -m);
+  uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    uint32_t pk[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      const uint64_t t = f2_fma(f2_pack(__uint_as_float(sr[c][2 * e]),
+                                        __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
+      float t0, t1;
+      f2_unpack(t, t0, t1);
+      const float p0 = ex2_approx(t0), p1 = ex2_approx(t1);
+      acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
+      pk[e] = pack_bf16x2(p0, p1);
+    }
+    tmem_st16(tP + c * 16, pk);
+  }
+  float s0, s1, s2, s3;
+  f2_unpack(f2_add(acc[0], acc[1]), s0, s1);
+  f2_unpack(f2_add(acc[2], acc[3]), s2, s3);
+  return (s0 + s2) + (s1 + s3);
+}
+
+__device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t tmem,
+                         const int* item_start, const Geom2& geo,
+                         const int32_t* __restrict__ prefix_lens,
+                         const int32_t* __restrict__ new_lens,
+                         const int32_t* __restrict__ cu_new_lens,
+                         __nv_bfloat16* __restrict__ out) {
+  volatile int* abortp = &bar.abort_flag;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = threadIdx.x - 128;  // q row of this CTA's half = tensor-memory lane
+  const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+  const bool rel = r == 0;  // frees ring slots
+  uint32_t u = 0;           // global step counter
+  uint32_t v_released = 0;  // V ring uses of steps [0, v_released) freed
+  bool ok = true;
+  auto release_v_upto = [&](uint32_t v) {  // steps <= v have finished their PV
+    if (rel)
+      while (v_released <= v) {
+        const uint32_t vu = 2 * v_released + 1;
+        mbar_arrive(&bar.empty[vu % kStages]);
+        ++v_released;
+      }
+  };
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = read_item2_warp(bar, k, abortp, ok);
+    if (!ok) break;
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
+    if (it < 0) break;
+    Item2 w;
+    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
+    const int tok = w.tok0 + r / geo.G;
+    const bool row_valid = tok < w.n;
+    const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
+    float m_run = -INFINITY, l = 0.f;
+    const float sl2 = geo.scale_log2;
+    for (int j = 0; j < w.nt; ++j, ++u) {
+      const uint32_t sb = u & 1;
+      const uint32_t tS = lane_addr + kColS + sb * 128;
+      const uint32_t tP = lane_addr + kColP + sb * 64;
+      ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
+      if (!ok) break;
+      if (rel) mbar_arrive(&bar.empty[(2 * u) % kStages]);  // K(u) has been read
+      tc_fence_after();
+      uint32_t sr[4][32];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+      tmem_wait_ld();
+      // S buffer free for S(u+2)
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(rm.s_free + 8 * sb);
+      const int key0 = j * kKeys;
+      if (key0 + kKeys - 1 > kmax) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (key0 + c * 32 + e > kmax) sr[c][e] = __float_as_uint(-INFINITY);
+      }
+      // P buffer sb is free once PV(u-2) is done
+      if (u >= 2) {
+        ok = wait_warp(&bar.pv_done[sb], ((u - 2) >> 1) & 1, abortp);
+        if (!ok) break;
+        release_v_upto(u - 2);
+      }
+      float lt;
+      if (j == 0) {
+        // first tile of the row: exact max (key 0 is always visible)
+        m_run = tile_max2(sr) * sl2;
+        lt = tile_exp2(sr, tP, sl2, m_run);
+      } else {
+        lt = tile_exp2(sr, tP, sl2, m_run);
+        if (__any_sync(0xffffffffu, !(lt < kSpecLimit))) {
+          // O must hold every earlier step before it is rescaled
+          ok = wait_warp(&bar.pv_done[(u - 1) & 1], ((u - 1) >> 1) & 1, abortp);
+          if (!ok) break;
+          release_v_upto(u - 1);
+          tmem_wait_st();
+          tc_fence_after();
+          const float m_new = fmaxf(m_run, tile_max2(sr) * sl2);
+          const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
+#pragma unroll 1
+          for (int c = 0; c < kD / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(lane_addr + kColO + c * 32, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+            tmem_st32(lane_addr + kColO + c * 32, o);
+          }
+          l *= alpha;
+          m_run = m_new;
+          lt = tile_exp2(sr, tP, sl2, m_run);
+        }
+      }
+      l += lt;
+      // publish P(u)
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(rm.p_full + 8 * sb);
+    }
+    if (!ok) break;
+    // ---- epilogue: O / l -> bf16, once the item's last PV is done
+    const uint32_t ul = u - 1;
+    ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
+    if (!ok) break;
+    release_v_upto(ul);
+    tc_fence_after();
+    const int h = w.g * geo.G + r % geo.G;
+    const float inv_l = 1.f / l;
+    uint4* orow = reinterpret_cast<uint4*>(
+        out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * kD);
+#pragma unroll 1
+    for (int c = 0; c < kD / 32; ++c) {
+      uint32_t o[32];
+      tmem_ld32(lane_addr + kColO + c * 32, o);
+      tmem_wait_ld();
+      if (row_valid) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 pk;
+          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+          orow[c * 4 + v] = pk;
+        }
+      }
+    }
+    // O may now be overwritten by the next item's first PV
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(rm.o_free);
+  }
+}
+
+// ------------------------------------------------------------------- kernel
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc2_kernel(const __grid_constant__ CUtensorMap map_q,
+                    const __grid_constant__ CUtensorMap map_kv,
+                    const int32_t* __restrict__ block_table,
+                    const int32_t* __restrict__ prefix_lens,
+                    const int32_t* __restrict__ new_lens,
+                    const int32_t* __restrict__ cu_new_lens, __nv_bfloat16* __restrict__ out,
+                    Geom2 geo, int32_t* status, int* work_counter) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint8_t* smem_q = base;                     // 2 x 32 KB
+  uint8_t* smem_kv = base + 2 * kQBytes;      // kStages x 16 KB
+  Bars2& bar = *reinterpret_cast<Bars2*>(smem_kv + kStages * kSlotBytes);
+  int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
+  int16_t* order = reinterpret_cast<int16_t*>(item_start + geo.batch + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bar.q_landed[i], 1);
+      mbar_init(&bar.q_full[i], 2);
+      mbar_init(&bar.q_empty[i], 1);
+      mbar_init(&bar.s_full[i], 1);
+      mbar_init(&bar.s_free[i], 8);
+      mbar_init(&bar.p_full[i], 8);
+      mbar_init(&bar.pv_done[i], 1);
+      mbar_init(&bar.item_full[i], 1);
+      mbar_init(&bar.item_empty[i], kItemConsumers);
+    }
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&bar.landed[s], 1);
+      mbar_init(&bar.full[s], 2);
+      mbar_init(&bar.empty[s], 1);
+    }
+    mbar_init(&bar.o_free, 8);
+    mbar_init(&bar.drain, 1);
+    bar.abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&map_q);
+    prefetch_tensormap(&map_kv);
+  }
+  if (warp == 1) {
+    tmem_alloc2(&bar.tmem_base, 512);
+    tmem_relinquish2();
+  }
+  if (geo.batch <= kSortMax) {
+    // rank requests by total length, longest first (ties by index)
+    for (int b = threadIdx.x; b < geo.batch; b += kThreads) {
+      const int tb = __ldg(prefix_lens + b) + __ldg(new_lens + b);
+      int rk = 0;
+      for (int o = 0; o < geo.batch; ++o) {
+        const int to = __ldg(prefix_lens + o) + __ldg(new_lens + o);
+        rk += (to > tb) || (to == tb && o < b);
+      }
+      order[rk] = static_cast<int16_t>(b);
+    }
+  }
+  __syncthreads();
+  if (warp == 2) {
+    // work items per request: Hkv * ceil(n_b * G / 256); exclusive scan in work order
+    int running = 0;
+    for (int b0 = 0; b0 < geo.batch; b0 += 32) {
+      const int p = b0 + lane;
+      const int b = p < geo.batch ? (geo.batch <= kSortMax ? order[p] : p) : p;
+      int cnt = 0;
+      if (p < geo.batch) {
+        const int n = __ldg(new_lens + b), P = __ldg(prefix_lens + b);
+        const int cu = __ldg(cu_new_lens + b);
+        const bool sane = n >= 0 && P >= 0 && cu >= 0 && cu + n <= geo.total_new;
+        if (!sane && n != 0 && rank == 0) record_error(status, GC_ERR_OUT_OF_RANGE);
+        if (sane && n > 0) cnt = geo.Hkv * ((n * geo.G + 2 * kRows - 1) / (2 * kRows));
+      }
+      int incl = cnt;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (p < geo.batch) item_start[p] = running + incl - cnt;
+      running += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) item_start[geo.batch] = running;
+  }
+  Remote rm;
+  {
+    const uint32_t lead = 0, peer = rank ^ 1u;
+    rm.q_full = mapa(smem_addr(&bar.q_full[0]), lead);
+    rm.full = mapa(smem_addr(&bar.full[0]), lead);
+    rm.s_free = mapa(smem_addr(&bar.s_free[0]), lead);
+    rm.p_full = mapa(smem_addr(&bar.p_full[0]), lead);
+    rm.o_free = mapa(smem_addr(&bar.o_free), lead);
+    rm.item_empty = mapa(smem_addr(&bar.item_empty[0]), lead);
+    rm.item_full = mapa(smem_addr(&bar.item_full[0]), peer);
+    rm.item_slot = mapa(smem_addr(&bar.item_slot[0]), peer);
+    rm.abort_peer = mapa(smem_addr(&bar.abort_flag), peer);
+  }
+  tc_fence_before();
+  // both CTAs' barriers are initialised before either CTA touches the other's
+  cluster_sync();
+  tc_fence_after();
+  const uint32_t tmem = bar.tmem_base;
+  const int total_items = item_start[geo.batch];
+
+  if (warp == 0) {
+    producer2(rank, smem_q, smem_kv, bar, rm, item_start, total_items, geo, &map_q, &map_kv,
+              block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
+  } else if (warp == 1) {
+    if (rank == 0 && lane == 0)
+      issuer2(smem_q, smem_kv, bar, rm, tmem, item_start, geo, prefix_lens, new_lens,
+              cu_new_lens);
+    __syncwarp();
+  } else if (warp == 3) {
+    forwarder2(rank, smem_kv, bar, rm, item_start, geo, prefix_lens, new_lens, cu_new_lens);
+  } else if (warp >= 4) {
+    softmax2(rank, bar, rm, tmem, item_start, geo, prefix_lens, new_lens, cu_new_lens, out);
+  }
+  // a CTA that gave up tells its peer, so that the peer's roles leave their
+  // loops instead of waiting for arrivals that will not come
+  if (*reinterpret_cast<volatile int*>(&bar.abort_flag) && lane == 0) raise_abort(bar, rm);
+  tc_fence_before();
+  __syncthreads();
+  // neither CTA leaves (or frees tensor memory) while the other may still
+  // read its shared memory or arrive on its barriers
+  cluster_sync();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc2(tmem, 512);
+  }
+  if (threadIdx.x == 0 && bar.abort_flag) record_error(status, GC_ERR_TIMEOUT);
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn2() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+size_t smem_bytes2(int batch) {
+  return 1024 + 2 * kQBytes + static_cast<size_t>(kStages) * kSlotBytes + sizeof(Bars2) +
+         (static_cast<size_t>(batch) + 1) * sizeof(int) + kSortMax * sizeof(int16_t);
+}
+
+}  // namespace
+
+// Clusters of two that fit on the device at once with this kernel's shared
+// memory (the persistent grid), 0 if the query fails.
+int attn_tc2_pairs(const gc_kv_pool* pool, int batch) {
+  const size_t smem = smem_bytes2(batch);
+  if (cudaFuncSetAttribute(attn_tc2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(smem)) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3(2 * (pool->num_sms / 2));
+  lc.blockDim = dim3(kThreads);
+  lc.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  lc.attrs = attr;
+  lc.numAttrs = 1;
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, attn_tc2_kernel, &lc) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return clusters;
+}
+
+gc_status launch_attn_tc2(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
+                          int* work_counter) {
+  const auto& cfg = pool->cfg;
+  if (cfg.head_dim != kD)
+    return fail(GC_ERR_UNSUPPORTED, "gc_prefix_prefill_attn: pair kernel needs head_dim 128");
+  const int pairs = attn_tc2_pairs(pool, a.batch);
+  if (pairs <= 0)
+    return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: no CTA pair fits on the device");
+  gc_status bound = check_item_bound(pool, a, nullptr, 2 * pairs);
+  if (bound != GC_OK) return bound;
+  auto enc = encode_fn2();
+  if (!enc) return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: cuTensorMapEncodeTiled unavailable");
+  Geom2 geo;
+  geo.batch = a.batch;
+  geo.Hq = a.num_q_heads;
+  geo.Hkv = cfg.num_kv_heads;
+  geo.G = geo.Hq / geo.Hkv;
+  geo.ps = cfg.page_size;
+  int s = 0;
+  while ((1 << s) < geo.ps) ++s;
+  geo.ps_shift = s;
+  geo.box_rows = geo.ps < 64 ? geo.ps : 64;
+  s = 0;
+  while ((1 << s) < geo.box_rows) ++s;
+  geo.box_shift = s;
+  geo.num_pages = cfg.num_pages;
+  geo.max_blocks = a.max_blocks;
+  geo.layer = a.layer;
+  geo.total_new = a.total_new_tokens;
+  geo.scale_log2 = a.softmax_scale * 1.4426950408889634f;
+
+  const uint64_t pool_rows = static_cast<uint64_t>(cfg.num_layers) * 2 * cfg.num_pages *
+                             cfg.num_kv_heads * cfg.page_size;
+  if (pool_rows >= (1ull << 31))
+    return fail(GC_ERR_UNSUPPORTED, "gc_prefix_prefill_attn: pool has %llu rows (limit 2^31)",
+                static_cast<unsigned long long>(pool_rows));
+  CUtensorMap map_q, map_kv;
+  {
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(geo.Hq),
+                          static_cast<cuuint64_t>(geo.total_new)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(kD) * 2,
+                             static_cast<cuuint64_t>(geo.Hq) * kD * 2};
+    cuuint32_t box[3] = {64, static_cast<cuuint32_t>(geo.G),
+                         static_cast<cuuint32_t>(kRows / geo.G)};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = enc(&map_q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.q), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: q tensor map (CUresult %d)", (int)r);
+  }
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(kD), pool_rows};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(kD) * 2};
+    cuuint32_t box[2] = {64, static_cast<cuuint32_t>(geo.box_rows)};
+    cuuint32_t es[2] = {1, 1};
+    CUresult r = enc(&map_kv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool->data, dims, strides, box,
+                     es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: pool tensor map (CUresult %d)", (int)r);
+  }
+  const size_t smem = smem_bytes2(a.batch);
+  // the work items are claimed from the given counter (the pool's control
+  // block, or the static scratch of the allocation-free entry point)
+  cudaError_t e = cudaMemsetAsync(work_counter, 0, sizeof(int), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: clearing the work counter");
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3(2 * pairs);
+  lc.blockDim = dim3(kThreads);
+  lc.dynamicSmemBytes = smem;
+  lc.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  lc.attrs = attr;
+  lc.numAttrs = 1;
+  e = cudaLaunchKernelEx(&lc, attn_tc2_kernel, map_q, map_kv, a.block_table, a.prefix_lens,
+                         a.new_lens, a.cu_new_lens, static_cast<__nv_bfloat16*>(a.out), geo,
+                         pool->status, work_counter);
+  if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: launch");
+  return GC_OK;
+}
+
+}  // namespace gc

@@ -81,6 +81,10 @@ struct AttnArgs {
 gc_status launch_attn_simt(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
+// head_dim 128 prefill on CTA pairs (attn_tc2.cu), work items claimed from
+// `work_counter` (zeroed by the launch).
+gc_status launch_attn_tc2(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
+                          int* work_counter);
 // The same kernel in decode mode: one new token per request (AttnArgs'
 // prefix_lens / new_lens / cu_new_lens unused), keys cut into ranges.
 struct DecodeMode {
