@@ -41,8 +41,7 @@
 //            reference max (the exact max of the row's first tile; raised,
 //            with O and l rescaled, only if a later tile would approach fp32
 //            overflow), P as bf16 into tensor memory, final 1/l and the bf16
-//            store of O.  Thread 0 also frees ring slots once the products
-//            that read them are complete.
+//            store of O.
 //  * Every wait and spin is bounded; a CTA that gives up raises its own and
 //    its peer's abort flag, every role leaves its loop, copies and MMAs in
 //    flight are drained, both CTAs meet at a cluster barrier, tensor memory
@@ -85,7 +84,7 @@ struct Bars2 {
   uint64_t q_empty[2];        // the item's last S product done (commit, both CTAs)
   uint64_t landed[kStages];   // this CTA's ring slot copied (tx)
   uint64_t full[kStages];     // even CTA: both halves of the slot ready (2 forwards)
-  uint64_t empty[kStages];    // this CTA's slot read by its products (softmax thread 0)
+  uint64_t empty[kStages];    // this CTA's slot read by its products (commit, both CTAs)
   uint64_t s_full[2];         // S buffer computed (commit, both CTAs)
   uint64_t s_free[2];         // even CTA: S buffer read by all 8 softmax warps
   uint64_t p_full[2];         // even CTA: P buffer written by all 8 softmax warps
@@ -327,9 +326,12 @@ __device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Re
 }
 
 // -------------------------------------------------------------- MMA issuer
-// One thread of the even CTA.  Per step t of an item: S(t) once K(t) is in
-// and the softmax has read S(t-2) out of the buffer; then PV(t-1) once the
-// softmax has written P(t-1) and V(t-1) is in.
+// One thread of the even CTA.  Per step t of an item it issues S(t+1) — once
+// K(t+1) is in and the softmax has read S(t-1) out of that buffer, which it
+// does first thing in step t-1 — and then PV(t), once the softmax has
+// written P(t) and V(t) is in.  S therefore runs a step ahead of the
+// softmax, which finds each S buffer computed when it gets to it.  Ring
+// slots are freed by commits, as soon as the product reading them is done.
 __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
                         uint32_t tmem, const int* item_start, const Geom2& geo,
                         const int32_t* __restrict__ prefix_lens,
@@ -337,7 +339,7 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
                         const int32_t* __restrict__ cu_new_lens) {
   volatile int* abortp = &bar.abort_flag;
   const uint32_t q_smem = smem_addr(smem_q), kv_smem = smem_addr(smem_kv);
-  uint32_t u = 0;     // global step counter
+  uint32_t u = 0;     // global step counter: first step of the current item
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
     const int it = read_item2(bar, k, abortp, ok);
@@ -349,9 +351,29 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
     const int qb = k & 1;
     ok = mbar_wait_cluster(&bar.q_full[qb], (k >> 1) & 1, abortp);
     if (!ok) break;
-    const uint32_t u_first = u;
+    const uint32_t u_first = u, u_last = u + w.nt - 1;
     const uint32_t q_addr = q_smem + qb * kQBytes;
-    // PV of step v (an earlier step of this item)
+    // S of step v of this item
+    auto s_prod = [&](uint32_t v) -> bool {
+      const uint32_t sb = v & 1;
+      const uint32_t ku = 2 * v;
+      if (!mbar_wait_cluster(&bar.full[ku % kStages], (ku / kStages) & 1, abortp)) return false;
+      if (v >= 2 && !mbar_wait_cluster(&bar.s_free[sb], ((v - 2) >> 1) & 1, abortp)) return false;
+      tc_fence_after();
+      const uint32_t k_addr = kv_smem + (ku % kStages) * kSlotBytes;
+#pragma unroll
+      for (int kk = 0; kk < kD / 16; ++kk) {
+        const uint32_t qo = (kk >> 2) * (kRows * 128) + (kk & 3) * 32;
+        const uint32_t ko = (kk >> 2) * (64 * 128) + (kk & 3) * 32;
+        mma2_ss(tmem + kColS + sb * 128, sdesc_sw128(q_addr + qo, 16, 1024),
+                sdesc_sw128(k_addr + ko, 16, 1024), kIdescQK, kk > 0);
+      }
+      mma2_commit_mc(&bar.s_full[sb], 0x3);
+      mma2_commit_mc(&bar.empty[ku % kStages], 0x3);
+      if (v == u_last) mma2_commit_mc(&bar.q_empty[qb], 0x3);
+      return true;
+    };
+    // PV of step v of this item
     auto pv = [&](uint32_t v) -> bool {
       const uint32_t pb = v & 1;
       if (!mbar_wait_cluster(&bar.p_full[pb], (v >> 1) & 1, abortp)) return false;
@@ -367,32 +389,15 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
                 sdesc_sw128(v_addr + kk * 16 * 128, kSlotBytes, 1024), kIdescPV,
                 (!first || kk > 0) ? 1u : 0u);
       mma2_commit_mc(&bar.pv_done[pb], 0x3);
+      mma2_commit_mc(&bar.empty[vu % kStages], 0x3);
       return true;
     };
-    for (int j = 0; j < w.nt; ++j, ++u) {
-      const uint32_t sb = u & 1;
-      const uint32_t ku = 2 * u;
-      ok = mbar_wait_cluster(&bar.full[ku % kStages], (ku / kStages) & 1, abortp);
-      if (ok && u >= 2) ok = mbar_wait_cluster(&bar.s_free[sb], ((u - 2) >> 1) & 1, abortp);
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t k_addr = kv_smem + (ku % kStages) * kSlotBytes;
-#pragma unroll
-      for (int kk = 0; kk < kD / 16; ++kk) {
-        const uint32_t qo = (kk >> 2) * (kRows * 128) + (kk & 3) * 32;
-        const uint32_t ko = (kk >> 2) * (64 * 128) + (kk & 3) * 32;
-        mma2_ss(tmem + kColS + sb * 128, sdesc_sw128(q_addr + qo, 16, 1024),
-                sdesc_sw128(k_addr + ko, 16, 1024), kIdescQK, kk > 0);
-      }
-      mma2_commit_mc(&bar.s_full[sb], 0x3);
-      if (j == w.nt - 1) mma2_commit_mc(&bar.q_empty[qb], 0x3);
-      if (j > 0 && !pv(u - 1)) {
-        ok = false;
-        break;
-      }
+    ok = s_prod(u_first);
+    for (uint32_t v = u_first; ok && v <= u_last; ++v) {
+      if (v < u_last) ok = s_prod(v + 1);
+      if (ok) ok = pv(v);
     }
-    if (!ok) break;
-    if (w.nt > 0 && !pv(u - 1)) ok = false;
+    u = u_last + 1;
   }
   // every MMA this thread issued must be complete before tensor memory is freed
   mma2_commit_mc(&bar.drain, 0x1);
@@ -453,18 +458,8 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = threadIdx.x - 128;  // q row of this CTA's half = tensor-memory lane
   const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
-  const bool rel = r == 0;  // frees ring slots
   uint32_t u = 0;           // global step counter
-  uint32_t v_released = 0;  // V ring uses of steps [0, v_released) freed
   bool ok = true;
-  auto release_v_upto = [&](uint32_t v) {  // steps <= v have finished their PV
-    if (rel)
-      while (v_released <= v) {
-        const uint32_t vu = 2 * v_released + 1;
-        mbar_arrive(&bar.empty[vu % kStages]);
-        ++v_released;
-      }
-  };
   for (uint32_t k = 0; ok; ++k) {
     const int it = read_item2_warp(bar, k, abortp, ok);
     if (!ok) break;
@@ -484,7 +479,6 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
       const uint32_t tP = lane_addr + kColP + sb * 64;
       ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
       if (!ok) break;
-      if (rel) mbar_arrive(&bar.empty[(2 * u) % kStages]);  // K(u) has been read
       tc_fence_after();
       uint32_t sr[4][32];
 #pragma unroll
@@ -506,7 +500,6 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
       if (u >= 2) {
         ok = wait_warp(&bar.pv_done[sb], ((u - 2) >> 1) & 1, abortp);
         if (!ok) break;
-        release_v_upto(u - 2);
       }
       float lt;
       if (j == 0) {
@@ -519,7 +512,6 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
           // O must hold every earlier step before it is rescaled
           ok = wait_warp(&bar.pv_done[(u - 1) & 1], ((u - 1) >> 1) & 1, abortp);
           if (!ok) break;
-          release_v_upto(u - 1);
           tmem_wait_st();
           tc_fence_after();
           const float m_new = fmaxf(m_run, tile_max2(sr) * sl2);
@@ -550,7 +542,6 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
     const uint32_t ul = u - 1;
     ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
     if (!ok) break;
-    release_v_upto(ul);
     tc_fence_after();
     const int h = w.g * geo.G + r % geo.G;
     const float inv_l = 1.f / l;
