@@ -145,6 +145,7 @@ __device__ __forceinline__ void decode_item2(int it, const int* item_start, cons
 // slot with one arrival per consumer warp on the even CTA's item_empty.
 __device__ __forceinline__ int read_item2(Bars2& bar, uint32_t k, volatile int* abortp,
                                           bool& ok) {
+  // the item id was written by the even CTA's producer: acquire at cluster scope
   ok = mbar_wait_cluster(&bar.item_full[k & 1], (k >> 1) & 1, abortp);
   return ok ? *reinterpret_cast<volatile int*>(&bar.item_slot[k & 1]) : -1;
 }
@@ -161,7 +162,7 @@ __device__ __forceinline__ int read_item2_warp(Bars2& bar, uint32_t k, volatile 
 // timeout seen by one lane alone cannot split the warp before a warp-wide
 // (.sync.aligned) instruction.
 __device__ __forceinline__ bool wait_warp(uint64_t* bar, uint32_t parity, volatile int* abortp) {
-  const bool ok = mbar_wait_cluster(bar, parity, abortp);
+  const bool ok = mbar_wait(bar, parity, abortp);
   return __all_sync(0xffffffffu, ok);
 }
 
@@ -304,21 +305,27 @@ __device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Re
     ok = wait_warp(&bar.q_landed[qb], (k >> 1) & 1, abortp);
     if (!ok) break;
     __syncwarp();
-    if (lane == 0) mbar_arrive_cluster(rm.q_full + 8 * qb);
+    if (lane == 0) mbar_arrive_remote(rm.q_full + 8 * qb);
     for (int j = 0; ok && j < w.nt; ++j) {
       for (int kv = 0; kv < 2; ++kv) {
         const int slot = use % kStages;
         ok = wait_warp(&bar.landed[slot], (use / kStages) & 1, abortp);
         if (!ok) break;
         const int nkeys = min(kKeys, w.T - j * kKeys);
-        if (kv == 1 && nkeys < kKeys) {
+        const bool zero = kv == 1 && nkeys < kKeys;
+        if (zero) {
           // V rows [nkeys, 128) of this CTA's column block (128 bytes each)
           uint4* z = reinterpret_cast<uint4*>(smem_kv + slot * kSlotBytes + nkeys * 128);
           for (int e = lane; e < (kKeys - nkeys) * 8; e += 32) z[e] = make_uint4(0, 0, 0, 0);
           fence_proxy_async_smem();
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive_cluster(rm.full + 8 * slot);
+        // the zeroed rows are generic-proxy writes the other SM's tensor core
+        // reads: publish them at cluster scope; a plain landed copy needs no fence
+        if (lane == 0) {
+          if (zero) mbar_arrive_cluster(rm.full + 8 * slot);
+          else mbar_arrive_remote(rm.full + 8 * slot);
+        }
         ++use;
       }
     }
@@ -326,11 +333,11 @@ __device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Re
 }
 
 // -------------------------------------------------------------- MMA issuer
-// One thread of the even CTA.  Per step t of an item it issues S(t+1) — once
-// K(t+1) is in and the softmax has read S(t-1) out of that buffer, which it
-// does first thing in step t-1 — and then PV(t), once the softmax has
-// written P(t) and V(t) is in.  S therefore runs a step ahead of the
-// softmax, which finds each S buffer computed when it gets to it.  Ring
+// One thread of the even CTA.  Per step t of an item it issues S(t+2) —
+// once K(t+2) is in and the softmax has read S(t) out of that buffer, which
+// it does first thing in step t — and then PV(t), once the softmax has
+// written P(t) and V(t) is in.  S therefore runs up to two steps ahead of
+// the softmax, which finds each S buffer computed when it gets to it.  Ring
 // slots are freed by commits, as soon as the product reading them is done.
 __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
                         uint32_t tmem, const int* item_start, const Geom2& geo,
@@ -349,7 +356,7 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
     Item2 w;
     decode_item2(it, item_start, geo, 0, prefix_lens, new_lens, cu_new_lens, w);
     const int qb = k & 1;
-    ok = mbar_wait_cluster(&bar.q_full[qb], (k >> 1) & 1, abortp);
+    ok = mbar_wait(&bar.q_full[qb], (k >> 1) & 1, abortp);
     if (!ok) break;
     const uint32_t u_first = u, u_last = u + w.nt - 1;
     const uint32_t q_addr = q_smem + qb * kQBytes;
@@ -357,8 +364,8 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
     auto s_prod = [&](uint32_t v) -> bool {
       const uint32_t sb = v & 1;
       const uint32_t ku = 2 * v;
-      if (!mbar_wait_cluster(&bar.full[ku % kStages], (ku / kStages) & 1, abortp)) return false;
-      if (v >= 2 && !mbar_wait_cluster(&bar.s_free[sb], ((v - 2) >> 1) & 1, abortp)) return false;
+      if (!mbar_wait(&bar.full[ku % kStages], (ku / kStages) & 1, abortp)) return false;
+      if (v >= 2 && !mbar_wait(&bar.s_free[sb], ((v - 2) >> 1) & 1, abortp)) return false;
       tc_fence_after();
       const uint32_t k_addr = kv_smem + (ku % kStages) * kSlotBytes;
 #pragma unroll
@@ -376,11 +383,11 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
     // PV of step v of this item
     auto pv = [&](uint32_t v) -> bool {
       const uint32_t pb = v & 1;
-      if (!mbar_wait_cluster(&bar.p_full[pb], (v >> 1) & 1, abortp)) return false;
+      if (!mbar_wait(&bar.p_full[pb], (v >> 1) & 1, abortp)) return false;
       const uint32_t vu = 2 * v + 1;
-      if (!mbar_wait_cluster(&bar.full[vu % kStages], (vu / kStages) & 1, abortp)) return false;
+      if (!mbar_wait(&bar.full[vu % kStages], (vu / kStages) & 1, abortp)) return false;
       const bool first = v == u_first;
-      if (first && k > 0 && !mbar_wait_cluster(&bar.o_free, (k - 1) & 1, abortp)) return false;
+      if (first && k > 0 && !mbar_wait(&bar.o_free, (k - 1) & 1, abortp)) return false;
       tc_fence_after();
       const uint32_t v_addr = kv_smem + (vu % kStages) * kSlotBytes;
 #pragma unroll
@@ -393,8 +400,9 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
       return true;
     };
     ok = s_prod(u_first);
+    if (ok && u_first < u_last) ok = s_prod(u_first + 1);
     for (uint32_t v = u_first; ok && v <= u_last; ++v) {
-      if (v < u_last) ok = s_prod(v + 1);
+      if (v + 2 <= u_last) ok = s_prod(v + 2);
       if (ok) ok = pv(v);
     }
     u = u_last + 1;
@@ -487,7 +495,7 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
       // S buffer free for S(u+2)
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(rm.s_free + 8 * sb);
+      if (lane == 0) mbar_arrive_remote(rm.s_free + 8 * sb);
       const int key0 = j * kKeys;
       if (key0 + kKeys - 1 > kmax) {
 #pragma unroll
@@ -535,7 +543,7 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(rm.p_full + 8 * sb);
+      if (lane == 0) mbar_arrive_remote(rm.p_full + 8 * sb);
     }
     if (!ok) break;
     // ---- epilogue: O / l -> bf16, once the item's last PV is done
@@ -567,7 +575,7 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
     // O may now be overwritten by the next item's first PV
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive_cluster(rm.o_free);
+    if (lane == 0) mbar_arrive_remote(rm.o_free);
   }
 }
 

@@ -107,10 +107,20 @@ __device__ __forceinline__ uint32_t mapa(uint32_t saddr, uint32_t rank) {
 }
 
 // Arrive once on the mbarrier at shared::cluster address `caddr` (this
-// CTA's or a peer's), releasing this thread's prior writes at cluster scope.
+// CTA's or a peer's), releasing this thread's prior writes at cluster scope
+// (a cluster-wide fence: for signals that publish generic-proxy data to the
+// other CTA).
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t caddr) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(caddr)
                : "memory");
+}
+
+// Arrive once on the mbarrier at shared::cluster address `caddr` with the
+// default (CTA-scope) release: for signals that order tensor-memory or
+// tensor-core work (with the tcgen05 fences) or copies the barrier itself
+// tracked, where no generic-proxy data crosses to the other CTA.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t caddr) {
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(caddr) : "memory");
 }
 
 __device__ __forceinline__ void st_cluster_u32(uint32_t caddr, uint32_t v) {
