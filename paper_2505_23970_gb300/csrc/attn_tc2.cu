@@ -57,7 +57,10 @@ namespace {
 using namespace ptx;
 
 constexpr int kD = 128;
-constexpr int kThreads = 256;
+// softmax by two warpgroups, half a row each (true), or one, whole rows (false)
+constexpr bool kHalfRows = true;
+constexpr int kSoftmaxWarps = kHalfRows ? 8 : 4;
+constexpr int kThreads = 128 + 32 * kSoftmaxWarps;
 constexpr int kRows = 128;            // q rows per SM
 constexpr int kKeys = 128;            // keys per K/V step
 constexpr int kStages = 8;            // ring slots of 16 KB (K and V halves alternate)
@@ -68,9 +71,9 @@ constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 constexpr float kSpecLimit = 9.223372036854775808e18f;  // 2^63, as in the single-SM kernel
-// consumers of the work-item ring per CTA: forwarder + 4 softmax warps +
+// consumers of the work-item ring per CTA: forwarder + softmax warps +
 // (even CTA) the MMA issuer or (odd CTA) the producer
-constexpr int kItemConsumers = 2 * 6;
+constexpr int kItemConsumers = 2 * (2 + kSoftmaxWarps);
 
 struct Geom2 {
   int32_t batch, Hq, Hkv, G, ps, ps_shift, num_pages, max_blocks, layer, total_new;
@@ -93,6 +96,7 @@ struct Bars2 {
   uint64_t item_full[2];      // work-item ring, written by the even CTA's producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: the issuer's last commit
+  uint64_t xch[4];            // half-row softmax: the two warps of a quadrant exchanged
   int item_slot[2];
   uint32_t tmem_base;
   int abort_flag;
@@ -579,6 +583,206 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
   }
 }
 
+// Half-row softmax: two warpgroups, warps 4-7 taking key columns [0, 64)
+// and warps 8-11 columns [64, 128) of every row of this CTA (warps w and
+// w + 4 share the tensor-memory lanes of quadrant w & 3).  Each thread
+// exponentiates 64 scores per step, so a step's softmax takes about half the
+// time; the two halves of a row agree on its reference max through a
+// per-step exchange of their half-tile maxima in shared memory (a 64-thread
+// named barrier per quadrant), and add their partial sums at the end.
+constexpr float kRescaleLog2 = 56.f;  // a term above 2^56 against the reference max
+
+// fp32 -> bf16 bits rounded toward +inf (finite and infinite inputs)
+__device__ __forceinline__ uint16_t bf16_bits_ru(float x) {
+  uint16_t r;
+  asm("cvt.rp.bf16.f32 %0, %1;" : "=h"(r) : "f"(x));
+  return r;
+}
+
+__device__ __forceinline__ float bf16_bits_to_f32(uint16_t b) {
+  return __uint_as_float(static_cast<uint32_t>(b) << 16);
+}
+
+
+__device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t tmem,
+                          uint16_t* xch, const int* item_start, const Geom2& geo,
+                          const int32_t* __restrict__ prefix_lens,
+                          const int32_t* __restrict__ new_lens,
+                          const int32_t* __restrict__ cu_new_lens,
+                          __nv_bfloat16* __restrict__ out) {
+  volatile int* abortp = &bar.abort_flag;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int hw = (warp - 4) >> 2;          // which 64 key columns
+  const int quad = warp & 3;
+  const int r = quad * 32 + lane;          // q row of this CTA's half = tensor-memory lane
+  const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+  uint32_t xn = 0;  // exchanges so far
+  // The partner thread's value (same row, other half): both warps of the
+  // quadrant write, then arrive once each on the quadrant's barrier (bounded
+  // wait).  Values are double-buffered: a warp that runs ahead writes the
+  // other buffer, and cannot come back to this one before its partner has
+  // arrived for the exchange after, i.e. has read this one.
+  auto exchange = [&](uint16_t v, bool& good) -> uint16_t {
+    const uint32_t xb = xn & 1;
+    xch[(xb * 2 + hw) * kRows + r] = v;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&bar.xch[quad]);
+    good = wait_warp(&bar.xch[quad], xn & 1, abortp);
+    ++xn;
+    return xch[(xb * 2 + (hw ^ 1)) * kRows + r];
+  };
+  uint32_t u = 0;  // global step counter
+  bool ok = true;
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = read_item2_warp(bar, k, abortp, ok);
+    if (!ok) break;
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
+    if (it < 0) break;
+    Item2 w;
+    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
+    const int tok = w.tok0 + r / geo.G;
+    const bool row_valid = tok < w.n;
+    const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
+    float m_run = -INFINITY, l = 0.f;
+    const float sl2 = geo.scale_log2;
+    for (int j = 0; j < w.nt; ++j, ++u) {
+      const uint32_t sb = u & 1;
+      const uint32_t tS = lane_addr + kColS + sb * 128 + hw * 64;
+      const uint32_t tP = lane_addr + kColP + sb * 64 + hw * 32;
+      ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t sr[2][32];
+      tmem_ld32(tS, sr[0]);
+      tmem_ld32(tS + 32, sr[1]);
+      tmem_wait_ld();
+      // S buffer free for S(u+2)
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(rm.s_free + 8 * sb);
+      const int key0 = j * kKeys + hw * 64;
+      if (key0 + 63 > kmax) {
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (key0 + c * 32 + e > kmax) sr[c][e] = __float_as_uint(-INFINITY);
+      }
+      float mh0 = -INFINITY, mh1 = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 2; ++c)
+#pragma unroll
+        for (int e = 0; e < 32; e += 4) {
+          mh0 = fmax3(mh0, __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
+          mh1 = fmax3(mh1, __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
+        }
+      // this half's max, rounded up to bf16 (16 bits to exchange); both
+      // halves of the row then take the max of the same two rounded values,
+      // a reference at or above the row's true tile max
+      const uint16_t mh = bf16_bits_ru(fmaxf(mh0, mh1));
+      const uint16_t mo = exchange(mh, ok);
+      if (!ok) break;
+      const float mt = fmaxf(bf16_bits_to_f32(mh), bf16_bits_to_f32(mo)) * sl2;
+      if (j == 0) {
+        m_run = mt;  // first tile of the row: exact max (key 0 is always visible)
+      } else if (__any_sync(0xffffffffu, mt - m_run > kRescaleLog2)) {
+        // O must hold every earlier step before it is rescaled; both halves of
+        // each row take the same decision from the same two maxima
+        ok = wait_warp(&bar.pv_done[(u - 1) & 1], ((u - 1) >> 1) & 1, abortp);
+        if (!ok) break;
+        tc_fence_after();
+        const float m_new = fmaxf(m_run, mt);
+        const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < 2; ++c) {
+          uint32_t o[32];
+          const uint32_t tO = lane_addr + kColO + hw * 64 + c * 32;
+          tmem_ld32(tO, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          tmem_st32(tO, o);
+        }
+        l *= alpha;
+        m_run = m_new;
+      }
+      // P buffer sb is free once PV(u-2) is done
+      if (u >= 2) {
+        ok = wait_warp(&bar.pv_done[sb], ((u - 2) >> 1) & 1, abortp);
+        if (!ok) break;
+      }
+      {
+        const uint64_t sc2 = f2_pack(sl2, sl2);
+        const uint64_t nm2 = f2_pack(-m_run, -m_run);
+        uint64_t acc[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const uint64_t t = f2_fma(f2_pack(__uint_as_float(sr[c][2 * e]),
+                                              __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
+            float t0, t1;
+            f2_unpack(t, t0, t1);
+            const float p0 = ex2_approx(t0), p1 = ex2_approx(t1);
+            acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
+            pk[e] = pack_bf16x2(p0, p1);
+          }
+          tmem_st16(tP + c * 16, pk);
+        }
+        float s0, s1, s2, s3;
+        f2_unpack(f2_add(acc[0], acc[1]), s0, s1);
+        f2_unpack(f2_add(acc[2], acc[3]), s2, s3);
+        l += (s0 + s2) + (s1 + s3);
+      }
+      // publish this half of P(u)
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(rm.p_full + 8 * sb);
+    }
+    if (!ok) break;
+    // ---- epilogue: O / l -> bf16 (this half's 64 columns), once the item's last PV is done
+    // the partner's partial sum, 16 bits at a time
+    const uint32_t lb = __float_as_uint(l);
+    const uint32_t lo_hi = exchange(static_cast<uint16_t>(lb >> 16), ok);
+    if (!ok) break;
+    const uint32_t lo_lo = exchange(static_cast<uint16_t>(lb & 0xffffu), ok);
+    if (!ok) break;
+    const float l_row = l + __uint_as_float((lo_hi << 16) | lo_lo);
+    const uint32_t ul = u - 1;
+    ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
+    if (!ok) break;
+    tc_fence_after();
+    const int h = w.g * geo.G + r % geo.G;
+    const float inv_l = 1.f / l_row;
+    uint4* orow = reinterpret_cast<uint4*>(
+        out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * kD + hw * 64);
+#pragma unroll 1
+    for (int c = 0; c < 2; ++c) {
+      uint32_t o[32];
+      tmem_ld32(lane_addr + kColO + hw * 64 + c * 32, o);
+      tmem_wait_ld();
+      if (row_valid) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 pk;
+          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+          orow[c * 4 + v] = pk;
+        }
+      }
+    }
+    // O may now be overwritten by the next item's first PV
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive_remote(rm.o_free);
+  }
+}
+
 // ------------------------------------------------------------------- kernel
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap map_q,
@@ -596,6 +800,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   Bars2& bar = *reinterpret_cast<Bars2*>(smem_kv + kStages * kSlotBytes);
   int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
   int16_t* order = reinterpret_cast<int16_t*>(item_start + geo.batch + 1);
+  // half-row softmax exchange area [2 buffers][2 halves][128 rows]
+  uint16_t* xch = reinterpret_cast<uint16_t*>(order + (geo.batch <= kSortMax ? kSortMax : 0));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
 
@@ -605,8 +811,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.q_full[i], 2);
       mbar_init(&bar.q_empty[i], 1);
       mbar_init(&bar.s_full[i], 1);
-      mbar_init(&bar.s_free[i], 8);
-      mbar_init(&bar.p_full[i], 8);
+      mbar_init(&bar.s_free[i], 2 * kSoftmaxWarps);
+      mbar_init(&bar.p_full[i], 2 * kSoftmaxWarps);
       mbar_init(&bar.pv_done[i], 1);
       mbar_init(&bar.item_full[i], 1);
       mbar_init(&bar.item_empty[i], kItemConsumers);
@@ -616,8 +822,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.full[s], 2);
       mbar_init(&bar.empty[s], 1);
     }
-    mbar_init(&bar.o_free, 8);
+    mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
     mbar_init(&bar.drain, 1);
+    for (int q = 0; q < 4; ++q) mbar_init(&bar.xch[q], 2);
     bar.abort_flag = 0;
     fence_barrier_init();
   }
@@ -698,7 +905,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 3) {
     forwarder2(rank, smem_kv, bar, rm, item_start, geo, prefix_lens, new_lens, cu_new_lens);
   } else if (warp >= 4) {
-    softmax2(rank, bar, rm, tmem, item_start, geo, prefix_lens, new_lens, cu_new_lens, out);
+    if (kHalfRows)
+      softmax2h(rank, bar, rm, tmem, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
+                out);
+    else
+      softmax2(rank, bar, rm, tmem, item_start, geo, prefix_lens, new_lens, cu_new_lens, out);
   }
   // a CTA that gave up tells its peer, so that the peer's roles leave their
   // loops instead of waiting for arrivals that will not come
@@ -730,7 +941,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn2() {
 
 size_t smem_bytes2(int batch) {
   return 1024 + 2 * kQBytes + static_cast<size_t>(kStages) * kSlotBytes + sizeof(Bars2) +
-         (static_cast<size_t>(batch) + 1) * sizeof(int) + kSortMax * sizeof(int16_t);
+         (static_cast<size_t>(batch) + 1) * sizeof(int) +
+         (batch <= kSortMax ? kSortMax * sizeof(int16_t) : 0) + 2 * 2 * kRows * sizeof(uint16_t);
 }
 
 }  // namespace
