@@ -97,15 +97,15 @@ struct Bars2 {
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: the issuer's last commit
   uint64_t xch[4];            // half-row softmax: the two warps of a quadrant exchanged
-  int item_slot[2];
+  int item_msg[2][8];         // a claimed item, decoded: it, b, tile, g, P, n, cu (it < 0: end)
   uint32_t tmem_base;
   int abort_flag;
 };
 
 // Shared::cluster addresses of the barriers that live in the even CTA, and
-// of the peer's abort flag and item slots.
+// of the peer's abort flag and item messages.
 struct Remote {
-  uint32_t q_full, full, s_free, p_full, o_free, item_empty, item_full, item_slot, abort_peer;
+  uint32_t q_full, full, s_free, p_full, o_free, item_empty, item_full, item_msg, abort_peer;
 };
 
 struct Item2 {
@@ -115,10 +115,14 @@ struct Item2 {
   bool rows_ok;  // this CTA has at least one valid row
 };
 
-__device__ __forceinline__ void decode_item2(int it, const int* item_start, const Geom2& geo,
-                                             uint32_t rank, const int32_t* __restrict__ prefix_lens,
+// Which request, kv head and 256-row tile item `it` is (item_start: first
+// item of each request in work order, then the order itself when the batch
+// was ranked), with the request's lengths: the message the even CTA's
+// producer sends to every role of both CTAs.
+__device__ __forceinline__ void item_message(int it, const int* item_start, const Geom2& geo,
+                                             const int32_t* __restrict__ prefix_lens,
                                              const int32_t* __restrict__ new_lens,
-                                             const int32_t* __restrict__ cu_new_lens, Item2& w) {
+                                             const int32_t* __restrict__ cu_new_lens, int* m) {
   int lo = 0, hi = geo.batch;  // last p with item_start[p] <= it
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
@@ -129,15 +133,26 @@ __device__ __forceinline__ void decode_item2(int it, const int* item_start, cons
                                        : lo;
   const int local = it - item_start[lo];
   const int tiles = (item_start[lo + 1] - item_start[lo]) / geo.Hkv;
-  const int tile = tiles - 1 - local / geo.Hkv;  // later rows (more keys) first
-  w.b = b;
-  w.g = local % geo.Hkv;
-  w.P = __ldg(prefix_lens + b);
-  w.n = __ldg(new_lens + b);
-  w.cu = __ldg(cu_new_lens + b);
+  m[0] = it;
+  m[1] = b;
+  m[2] = tiles - 1 - local / geo.Hkv;  // later rows (more keys) first
+  m[3] = local % geo.Hkv;
+  m[4] = __ldg(prefix_lens + b);
+  m[5] = __ldg(new_lens + b);
+  m[6] = __ldg(cu_new_lens + b);
+}
+
+// The quantities a role of CTA `rank` derives from an item message.
+__device__ __forceinline__ void item_from_message(const int* m, const Geom2& geo, uint32_t rank,
+                                                  Item2& w) {
+  w.b = m[1];
+  w.g = m[3];
+  w.P = m[4];
+  w.n = m[5];
+  w.cu = m[6];
   w.T = w.P + w.n;
   const int rows = w.n * geo.G;
-  const int r0 = tile * 2 * kRows;
+  const int r0 = m[2] * 2 * kRows;
   w.tok0 = (r0 + static_cast<int>(rank) * kRows) / geo.G;
   w.rows_ok = r0 + static_cast<int>(rank) * kRows < rows;
   const int r_last = min(r0 + 2 * kRows - 1, rows - 1);  // last valid row of the item
@@ -147,17 +162,26 @@ __device__ __forceinline__ void decode_item2(int it, const int* item_start, cons
 
 // Read item k of the ring (every consumer thread); the caller releases the
 // slot with one arrival per consumer warp on the even CTA's item_empty.
-__device__ __forceinline__ int read_item2(Bars2& bar, uint32_t k, volatile int* abortp,
+// Returns the item number, -1 at the end.
+__device__ __forceinline__ int read_item2(Bars2& bar, uint32_t k, const Geom2& geo,
+                                          uint32_t rank, Item2& w, volatile int* abortp,
                                           bool& ok) {
-  // the item id was written by the even CTA's producer: acquire at cluster scope
+  // the message was written by the even CTA's producer: acquire at cluster scope
   ok = mbar_wait_cluster(&bar.item_full[k & 1], (k >> 1) & 1, abortp);
-  return ok ? *reinterpret_cast<volatile int*>(&bar.item_slot[k & 1]) : -1;
+  if (!ok) return -1;
+  const volatile int* m = bar.item_msg[k & 1];
+  int mm[7];
+#pragma unroll
+  for (int i = 0; i < 7; ++i) mm[i] = m[i];
+  if (mm[0] >= 0) item_from_message(mm, geo, rank, w);
+  return mm[0];
 }
 
 // The same for a whole warp (every lane reads the item; the lanes agree).
-__device__ __forceinline__ int read_item2_warp(Bars2& bar, uint32_t k, volatile int* abortp,
+__device__ __forceinline__ int read_item2_warp(Bars2& bar, uint32_t k, const Geom2& geo,
+                                               uint32_t rank, Item2& w, volatile int* abortp,
                                                bool& ok) {
-  const int it = read_item2(bar, k, abortp, ok);
+  const int it = read_item2(bar, k, geo, rank, w, abortp, ok);
   ok = __all_sync(0xffffffffu, ok);
   return it;
 }
@@ -193,32 +217,42 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars
   const uint32_t box_bytes = static_cast<uint32_t>(geo.box_rows) * 128;
   const int boxes_k = (64 >> geo.box_shift) * 2;  // K half: 64 keys x 2 column blocks
   const int boxes_v = kKeys >> geo.box_shift;     // V half: 128 keys x 1 column block
+  const int pages_per_step = kKeys >> geo.ps_shift;
 
   for (uint32_t k = 0; ok; ++k) {
     int it = -1;
+    Item2 w;
     if (rank == 0) {
-      // claim the next item and publish it to both CTAs
+      // claim the next item and send it, decoded, to every role of both CTAs
       const int s = k & 1;
       ok = wait_warp(&bar.item_empty[s], ((k >> 1) & 1) ^ 1, abortp);
       if (!ok) break;
+      int m[7];
       if (lane == 0) {
         it = atomicAdd(work_counter, 1);
         if (it >= total_items) it = -1;
-        bar.item_slot[s] = it;
-        st_cluster_u32(rm.item_slot + 4 * s, static_cast<uint32_t>(it));
+        m[0] = it;
+        if (it >= 0) item_message(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, m);
+#pragma unroll
+        for (int i = 0; i < 7; ++i) {
+          bar.item_msg[s][i] = m[i];
+          st_cluster_u32(rm.item_msg + 32 * s + 4 * i, static_cast<uint32_t>(m[i]));
+          if (it < 0) break;
+        }
         mbar_arrive(&bar.item_full[s]);
         mbar_arrive_cluster(rm.item_full + 8 * s);
       }
-      it = __shfl_sync(0xffffffffu, it, 0);
+      __syncwarp();
+      it = read_item2(bar, k, geo, rank, w, abortp, ok);  // the message just written
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
     } else {
-      it = read_item2_warp(bar, k, abortp, ok);
+      it = read_item2_warp(bar, k, geo, rank, w, abortp, ok);
       if (!ok) break;
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     }
     if (it < 0) break;
-    Item2 w;
-    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
     // ---- this CTA's Q half: 128 rows = 128/G tokens x G heads, two column blocks
     const int qb = k & 1;
     ok = wait_warp(&bar.q_empty[qb], ((k >> 1) & 1) ^ 1, abortp);
@@ -231,40 +265,50 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars
                     w.g * geo.G, w.cu + w.tok0);
     }
     armed_q = qb | (((k >> 1) & 1) << 1);
-    // ---- K/V halves, step by step
+    // ---- K/V halves, step by step.  Lane i holds the block-table entry of
+    // page i of a step (-2: no such page before the end of the sequence);
+    // the next step's entries are loaded while this step's copies are issued.
     const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
+    auto lookup = [&](int j) -> int {
+      const int key = j * kKeys + lane * geo.ps;  // first key of page `lane` of step j
+      if (lane >= pages_per_step || key >= w.T) return -2;
+      const int blk = key >> geo.ps_shift;
+      return blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
+    };
+    int pages = lookup(0);
     for (int j = 0; ok && j < w.nt; ++j) {
       const int key0 = j * kKeys;
+      const int pages_next = j + 1 < w.nt ? lookup(j + 1) : -2;
 #pragma unroll 1
       for (int kv = 0; kv < 2; ++kv) {
         const int slot = use % kStages;
-        ok = wait_warp(&bar.empty[slot], ((use / kStages) & 1) ^ 1, abortp);
-        if (!ok) break;
         // box `lane`: K: column block lane & 1, rows of chunk lane >> 1 of
         // this CTA's 64 keys; V: column block `rank`, chunk lane of 128 keys
         const int nbox = kv == 0 ? boxes_k : boxes_v;
-        int kc = 0, col = 0, dst = 0;
+        int ko = 0, col = 0, dst = 0;  // ko: first key of the box within the step
         if (kv == 0) {
-          kc = key0 + static_cast<int>(rank) * 64 + (lane >> 1) * geo.box_rows;
+          ko = static_cast<int>(rank) * 64 + (lane >> 1) * geo.box_rows;
           col = (lane & 1) * 64;
           dst = (lane & 1) * (64 * 128) + (lane >> 1) * geo.box_rows * 128;
         } else {
-          kc = key0 + lane * geo.box_rows;
+          ko = lane * geo.box_rows;
           col = static_cast<int>(rank) * 64;
           dst = lane * geo.box_rows * 128;
         }
+        const int page = __shfl_sync(0xffffffffu, pages, min(ko >> geo.ps_shift, 31));
         int row = -1;
-        if (lane < nbox && kc < w.T) {
-          const int blk = kc >> geo.ps_shift;
-          const int page = blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
+        if (lane < nbox && page != -2 && key0 + ko < w.T) {
           if (page < 0 || page >= geo.num_pages) {
             record_error(status, GC_ERR_OUT_OF_RANGE);
           } else {
             const int plane_row = (geo.layer * 2 + kv) * geo.num_pages;
-            row = (((plane_row + page) * geo.Hkv + w.g) << geo.ps_shift) + (kc & (geo.ps - 1));
+            row = (((plane_row + page) * geo.Hkv + w.g) << geo.ps_shift) +
+                  ((key0 + ko) & (geo.ps - 1));
           }
         }
         const int good = __popc(__ballot_sync(0xffffffffu, row >= 0));
+        ok = wait_warp(&bar.empty[slot], ((use / kStages) & 1) ^ 1, abortp);
+        if (!ok) break;
         if (lane == 0) mbar_arrive_expect_tx(&bar.landed[slot], static_cast<uint32_t>(good) * box_bytes);
         __syncwarp();
         if (row >= 0) tma_load_2d(smem_kv + slot * kSlotBytes + dst, map_kv, &bar.landed[slot], col, row);
@@ -272,6 +316,7 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars
         armed_par = (armed_par & ~(1u << slot)) | (((use / kStages) & 1u) << slot);
         ++use;
       }
+      pages = pages_next;
     }
   }
   if (!ok && lane == 0) {
@@ -298,13 +343,12 @@ __device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Re
   uint32_t use = 0;
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
-    const int it = read_item2_warp(bar, k, abortp, ok);
+    Item2 w;
+    const int it = read_item2_warp(bar, k, geo, rank, w, abortp, ok);
     if (!ok) break;
     __syncwarp();
     if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
-    Item2 w;
-    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
     const int qb = k & 1;
     ok = wait_warp(&bar.q_landed[qb], (k >> 1) & 1, abortp);
     if (!ok) break;
@@ -353,12 +397,11 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
   uint32_t u = 0;     // global step counter: first step of the current item
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
-    const int it = read_item2(bar, k, abortp, ok);
+    Item2 w;
+    const int it = read_item2(bar, k, geo, 0, w, abortp, ok);
     if (!ok) break;
     mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
-    Item2 w;
-    decode_item2(it, item_start, geo, 0, prefix_lens, new_lens, cu_new_lens, w);
     const int qb = k & 1;
     ok = mbar_wait(&bar.q_full[qb], (k >> 1) & 1, abortp);
     if (!ok) break;
@@ -473,13 +516,12 @@ __device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t t
   uint32_t u = 0;           // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
-    const int it = read_item2_warp(bar, k, abortp, ok);
+    Item2 w;
+    const int it = read_item2_warp(bar, k, geo, rank, w, abortp, ok);
     if (!ok) break;
     __syncwarp();
     if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
-    Item2 w;
-    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
     const int tok = w.tok0 + r / geo.G;
     const bool row_valid = tok < w.n;
     const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
@@ -634,13 +676,12 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
   uint32_t u = 0;  // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
-    const int it = read_item2_warp(bar, k, abortp, ok);
+    Item2 w;
+    const int it = read_item2_warp(bar, k, geo, rank, w, abortp, ok);
     if (!ok) break;
     __syncwarp();
     if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
-    Item2 w;
-    decode_item2(it, item_start, geo, rank, prefix_lens, new_lens, cu_new_lens, w);
     const int tok = w.tok0 + r / geo.G;
     const bool row_valid = tok < w.n;
     const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
@@ -884,7 +925,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     rm.o_free = mapa(smem_addr(&bar.o_free), lead);
     rm.item_empty = mapa(smem_addr(&bar.item_empty[0]), lead);
     rm.item_full = mapa(smem_addr(&bar.item_full[0]), peer);
-    rm.item_slot = mapa(smem_addr(&bar.item_slot[0]), peer);
+    rm.item_msg = mapa(smem_addr(&bar.item_msg[0][0]), peer);
     rm.abort_peer = mapa(smem_addr(&bar.abort_flag), peer);
   }
   tc_fence_before();
