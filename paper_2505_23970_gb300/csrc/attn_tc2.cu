@@ -24,15 +24,16 @@
 //                   V MN-major in smem)
 //  * Tensor memory per SM: S double-buffered [0,128) [128,256), O [256,384),
 //    P double-buffered [384,448) [448,512) (bf16 pairs).  P has its own
-//    columns, so S(t+1) is computed while the softmax works on S(t); the
-//    issuer's order S(t+1), PV(t) keeps the tensor pipe fed from one chain.
+//    columns, so S(t+1) and S(t+2) are computed while the softmax works on
+//    S(t), and PV(t) overlaps the softmax of step t+1.
 //  * Warps per CTA:
 //      0     TMA producer: this SM's Q half, then per 128-key step its K
 //            half (64 keys x 128 d) and V half (128 keys x 64 d) into a ring
 //            of 16 KB slots; page boxes issued by several lanes at once.
-//      1     tensor-memory owner (both CTAs allocate together); lane 0 of
-//            the even CTA issues every MMA of the pair.
-//      2     item table at start-up.
+//      1     tensor-memory owner (both CTAs allocate together); in the
+//            even CTA lane 0 issues the pair's S products
+//      2     item table at start-up; in the even CTA lane 0 then issues the
+//            pair's PV products.
 //      3     forwarder: waits for this SM's copies to land, zeroes V rows
 //            past the end of the sequence (their P is 0 but 0 * NaN is
 //            NaN), and reports the slot as full to the even CTA.
@@ -71,9 +72,9 @@ constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 constexpr float kSpecLimit = 9.223372036854775808e18f;  // 2^63, as in the single-SM kernel
-// consumers of the work-item ring per CTA: forwarder + softmax warps +
-// (even CTA) the MMA issuer or (odd CTA) the producer
-constexpr int kItemConsumers = 2 * (2 + kSoftmaxWarps);
+// consumers of the work-item ring: in each CTA the forwarder and the softmax
+// warps, plus the two MMA issuers of the even CTA and the odd CTA's producer
+constexpr int kItemConsumers = 2 * (1 + kSoftmaxWarps) + 3;
 
 struct Geom2 {
   int32_t batch, Hq, Hkv, G, ps, ps_shift, num_pages, max_blocks, layer, total_new;
@@ -95,7 +96,7 @@ struct Bars2 {
   uint64_t o_free;            // even CTA: O read by the epilogue (8 warps)
   uint64_t item_full[2];      // work-item ring, written by the even CTA's producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
-  uint64_t drain;             // even CTA: the issuer's last commit
+  uint64_t drain;             // even CTA: both issuers' last commits
   uint64_t xch[4];            // half-row softmax: the two warps of a quadrant exchanged
   int item_msg[2][8];         // a claimed item, decoded: it, b, tile, g, P, n, cu (it < 0: end)
   uint32_t tmem_base;
@@ -380,21 +381,23 @@ __device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Re
   }
 }
 
-// -------------------------------------------------------------- MMA issuer
-// One thread of the even CTA.  Per step t of an item it issues S(t+2) —
-// once K(t+2) is in and the softmax has read S(t) out of that buffer, which
-// it does first thing in step t — and then PV(t), once the softmax has
-// written P(t) and V(t) is in.  S therefore runs up to two steps ahead of
-// the softmax, which finds each S buffer computed when it gets to it.  Ring
-// slots are freed by commits, as soon as the product reading them is done.
-__device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
-                        uint32_t tmem, const int* item_start, const Geom2& geo,
-                        const int32_t* __restrict__ prefix_lens,
-                        const int32_t* __restrict__ new_lens,
-                        const int32_t* __restrict__ cu_new_lens) {
+// -------------------------------------------------------------- MMA issuers
+// Two threads of the even CTA, in different warps, issue the pair's MMAs:
+// one the S products, one the PV products.  They touch disjoint tensor
+// memory (S buffers / P buffers and O) and disjoint ring slots (K / V), so
+// they need no order between them, and a single thread issuing both (each
+// tcgen05.mma costs its issuing thread tens of cycles) could not keep the
+// tensor pipe busy.  Operand descriptors are built once per tile and
+// advanced by constant offsets.
+//
+// S issuer: S(t) once K(t) is in and the softmax has read S(t-2) out of the
+// buffer (which it does first thing in step t-2), so S runs up to two steps
+// ahead of the softmax.  Frees K slots and the Q buffer by commits.
+__device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
+                          uint32_t tmem, const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
   const uint32_t q_smem = smem_addr(smem_q), kv_smem = smem_addr(smem_kv);
-  uint32_t u = 0;     // global step counter: first step of the current item
+  uint32_t u = 0;  // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
     Item2 w;
@@ -405,56 +408,71 @@ __device__ void issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Rem
     const int qb = k & 1;
     ok = mbar_wait(&bar.q_full[qb], (k >> 1) & 1, abortp);
     if (!ok) break;
-    const uint32_t u_first = u, u_last = u + w.nt - 1;
-    const uint32_t q_addr = q_smem + qb * kQBytes;
-    // S of step v of this item
-    auto s_prod = [&](uint32_t v) -> bool {
-      const uint32_t sb = v & 1;
-      const uint32_t ku = 2 * v;
-      if (!mbar_wait(&bar.full[ku % kStages], (ku / kStages) & 1, abortp)) return false;
-      if (v >= 2 && !mbar_wait(&bar.s_free[sb], ((v - 2) >> 1) & 1, abortp)) return false;
+    const uint64_t dq = sdesc_sw128(q_smem + qb * kQBytes, 16, 1024);
+    const uint32_t u_last = u + w.nt - 1;
+    for (; ok && u <= u_last; ++u) {
+      const uint32_t sb = u & 1;
+      const uint32_t ku = 2 * u, slot = ku % kStages;
+      ok = mbar_wait(&bar.full[slot], (ku / kStages) & 1, abortp);
+      if (ok && u >= 2) ok = mbar_wait(&bar.s_free[sb], ((u - 2) >> 1) & 1, abortp);
+      if (!ok) break;
       tc_fence_after();
-      const uint32_t k_addr = kv_smem + (ku % kStages) * kSlotBytes;
+      const uint64_t dk = sdesc_sw128(kv_smem + slot * kSlotBytes, 16, 1024);
+      const uint32_t d = tmem + kColS + sb * 128;
 #pragma unroll
       for (int kk = 0; kk < kD / 16; ++kk) {
-        const uint32_t qo = (kk >> 2) * (kRows * 128) + (kk & 3) * 32;
-        const uint32_t ko = (kk >> 2) * (64 * 128) + (kk & 3) * 32;
-        mma2_ss(tmem + kColS + sb * 128, sdesc_sw128(q_addr + qo, 16, 1024),
-                sdesc_sw128(k_addr + ko, 16, 1024), kIdescQK, kk > 0);
+        // 16-column steps: 32 bytes within a 128-byte row, then the next
+        // 64-column block (Q: 128 rows x 128 B, K half: 64 rows x 128 B)
+        constexpr uint32_t kQBlk = kRows * 128 >> 4, kKBlk = 64 * 128 >> 4;
+        mma2_ss(d, dq + ((kk >> 2) * kQBlk + (kk & 3) * 2), dk + ((kk >> 2) * kKBlk + (kk & 3) * 2),
+                kIdescQK, kk > 0);
       }
       mma2_commit_mc(&bar.s_full[sb], 0x3);
-      mma2_commit_mc(&bar.empty[ku % kStages], 0x3);
-      if (v == u_last) mma2_commit_mc(&bar.q_empty[qb], 0x3);
-      return true;
-    };
-    // PV of step v of this item
-    auto pv = [&](uint32_t v) -> bool {
-      const uint32_t pb = v & 1;
-      if (!mbar_wait(&bar.p_full[pb], (v >> 1) & 1, abortp)) return false;
-      const uint32_t vu = 2 * v + 1;
-      if (!mbar_wait(&bar.full[vu % kStages], (vu / kStages) & 1, abortp)) return false;
-      const bool first = v == u_first;
-      if (first && k > 0 && !mbar_wait(&bar.o_free, (k - 1) & 1, abortp)) return false;
-      tc_fence_after();
-      const uint32_t v_addr = kv_smem + (vu % kStages) * kSlotBytes;
-#pragma unroll
-      for (int kk = 0; kk < kKeys / 16; ++kk)
-        mma2_ts(tmem + kColO, tmem + kColP + pb * 64 + kk * 8,
-                sdesc_sw128(v_addr + kk * 16 * 128, kSlotBytes, 1024), kIdescPV,
-                (!first || kk > 0) ? 1u : 0u);
-      mma2_commit_mc(&bar.pv_done[pb], 0x3);
-      mma2_commit_mc(&bar.empty[vu % kStages], 0x3);
-      return true;
-    };
-    ok = s_prod(u_first);
-    if (ok && u_first < u_last) ok = s_prod(u_first + 1);
-    for (uint32_t v = u_first; ok && v <= u_last; ++v) {
-      if (v + 2 <= u_last) ok = s_prod(v + 2);
-      if (ok) ok = pv(v);
+      mma2_commit_mc(&bar.empty[slot], 0x3);
+      if (u == u_last) mma2_commit_mc(&bar.q_empty[qb], 0x3);
     }
-    u = u_last + 1;
   }
   // every MMA this thread issued must be complete before tensor memory is freed
+  mma2_commit_mc(&bar.drain, 0x1);
+  int no_abort = 0;
+  mbar_wait(&bar.drain, 0, &no_abort);
+}
+
+// PV issuer: O += P(t) V(t) once the softmax has written P(t) and V(t) is
+// in; an item's first product (which overwrites O) also waits until the
+// previous item's epilogue has read O.  Frees V slots by commits.
+__device__ void pv_issuer2(uint8_t* smem_kv, Bars2& bar, const Remote& rm, uint32_t tmem,
+                           const Geom2& geo) {
+  volatile int* abortp = &bar.abort_flag;
+  const uint32_t kv_smem = smem_addr(smem_kv);
+  uint32_t u = 0;  // global step counter
+  bool ok = true;
+  for (uint32_t k = 0; ok; ++k) {
+    Item2 w;
+    const int it = read_item2(bar, k, geo, 0, w, abortp, ok);
+    if (!ok) break;
+    mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
+    if (it < 0) break;
+    const uint32_t u_first = u, u_last = u + w.nt - 1;
+    for (; ok && u <= u_last; ++u) {
+      const uint32_t pb = u & 1;
+      const uint32_t vu = 2 * u + 1, slot = vu % kStages;
+      ok = mbar_wait(&bar.p_full[pb], (u >> 1) & 1, abortp);
+      if (ok) ok = mbar_wait(&bar.full[slot], (vu / kStages) & 1, abortp);
+      const bool first = u == u_first;
+      if (ok && first && k > 0) ok = mbar_wait(&bar.o_free, (k - 1) & 1, abortp);
+      if (!ok) break;
+      tc_fence_after();
+      const uint64_t dv = sdesc_sw128(kv_smem + slot * kSlotBytes, kSlotBytes, 1024);
+      const uint32_t a = tmem + kColP + pb * 64;
+#pragma unroll
+      for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys = two 8-row groups of 1 KB
+        mma2_ts(tmem + kColO, a + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
+                (!first || kk > 0) ? 1u : 0u);
+      mma2_commit_mc(&bar.pv_done[pb], 0x3);
+      mma2_commit_mc(&bar.empty[slot], 0x3);
+    }
+  }
   mma2_commit_mc(&bar.drain, 0x1);
   int no_abort = 0;
   mbar_wait(&bar.drain, 0, &no_abort);
@@ -864,7 +882,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.empty[s], 1);
     }
     mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
-    mbar_init(&bar.drain, 1);
+    mbar_init(&bar.drain, 2);
     for (int q = 0; q < 4; ++q) mbar_init(&bar.xch[q], 2);
     bar.abort_flag = 0;
     fence_barrier_init();
@@ -939,9 +957,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     producer2(rank, smem_q, smem_kv, bar, rm, item_start, total_items, geo, &map_q, &map_kv,
               block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
   } else if (warp == 1) {
-    if (rank == 0 && lane == 0)
-      issuer2(smem_q, smem_kv, bar, rm, tmem, item_start, geo, prefix_lens, new_lens,
-              cu_new_lens);
+    if (rank == 0 && lane == 0) s_issuer2(smem_q, smem_kv, bar, rm, tmem, geo);
+    __syncwarp();
+  } else if (warp == 2) {
+    if (rank == 0 && lane == 0) pv_issuer2(smem_kv, bar, rm, tmem, geo);
     __syncwarp();
   } else if (warp == 3) {
     forwarder2(rank, smem_kv, bar, rm, item_start, geo, prefix_lens, new_lens, cu_new_lens);
