@@ -27,22 +27,23 @@
 //    columns, so S(t+1) and S(t+2) are computed while the softmax works on
 //    S(t), and PV(t) overlaps the softmax of step t+1.
 //  * Warps per CTA:
-//      0     TMA producer: this SM's Q half, then per 128-key step its K
-//            half (64 keys x 128 d) and V half (128 keys x 64 d) into a ring
-//            of 16 KB slots; page boxes issued by several lanes at once.
-//      1     tensor-memory owner (both CTAs allocate together); in the
-//            even CTA lane 0 issues the pair's S products
+//      0     K producer: this SM's Q half of each item, then per 128-key step
+//            its K half (64 keys x 128 d, one 4-D box per page) into a ring
+//            of 16 KB slots.
+//      3     V producer: per step its V half (128 keys x 64 d, one box per
+//            page) into a second ring.  Each producer reports its own copies
+//            to the even CTA once they have landed, zeroing V rows past the
+//            end of the sequence first (their P is 0 but 0 * NaN is NaN).
+//      1     tensor-memory owner (both CTAs allocate together); in the even
+//            CTA lane 0 issues the pair's S products.
 //      2     item table at start-up; in the even CTA lane 0 then issues the
 //            pair's PV products.
-//      3     forwarder: waits for this SM's copies to land, zeroes V rows
-//            past the end of the sequence (their P is 0 but 0 * NaN is
-//            NaN), and reports the slot as full to the even CTA.
-//      4-7   softmax, one thread per q row (= tensor-memory lane): S row from
-//            tensor memory, causal mask, p = 2^(s*scale*log2 e - m) against a
-//            reference max (the exact max of the row's first tile; raised,
-//            with O and l rescaled, only if a later tile would approach fp32
-//            overflow), P as bf16 into tensor memory, final 1/l and the bf16
-//            store of O.
+//      4-11  softmax in two warpgroups, key columns [0, 64) and [64, 128) of
+//            every q row (= tensor-memory lane): S from tensor memory, causal
+//            mask, p = 2^(s*scale*log2 e - m) against a reference max (the
+//            row's first-tile max; raised, with O and l rescaled, only if a
+//            later tile would approach fp32 overflow), P as bf16 into tensor
+//            memory, final 1/l and the bf16 store of O.
 //  * Every wait and spin is bounded; a CTA that gives up raises its own and
 //    its peer's abort flag, every role leaves its loop, copies and MMAs in
 //    flight are drained, both CTAs meet at a cluster barrier, tensor memory
@@ -64,7 +65,7 @@ constexpr int kSoftmaxWarps = kHalfRows ? 8 : 4;
 constexpr int kThreads = 128 + 32 * kSoftmaxWarps;
 constexpr int kRows = 128;            // q rows per SM
 constexpr int kKeys = 128;            // keys per K/V step
-constexpr int kStages = 8;            // ring slots of 16 KB (K and V halves alternate)
+constexpr int kRing = 4;              // slots of 16 KB in each of the K and V rings
 constexpr int kSlotBytes = 16384;
 constexpr int kQBytes = kRows * kD * 2;  // 32 KB: two 64-column blocks of 128 rows
 constexpr int kSortMax = 512;
@@ -72,8 +73,9 @@ constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 constexpr float kSpecLimit = 9.223372036854775808e18f;  // 2^63, as in the single-SM kernel
-// consumers of the work-item ring: in each CTA the forwarder and the softmax
-// warps, plus the two MMA issuers of the even CTA and the odd CTA's producer
+// consumers of the work-item ring: in each CTA the V producer and the
+// softmax warps, plus the two MMA issuers of the even CTA and the odd CTA's
+// K producer
 constexpr int kItemConsumers = 2 * (1 + kSoftmaxWarps) + 3;
 
 struct Geom2 {
@@ -86,19 +88,23 @@ struct Bars2 {
   uint64_t q_landed[2];       // this CTA's Q half copied (tx)
   uint64_t q_full[2];         // even CTA: both Q halves landed (2 forwards)
   uint64_t q_empty[2];        // the item's last S product done (commit, both CTAs)
-  uint64_t landed[kStages];   // this CTA's ring slot copied (tx)
-  uint64_t full[kStages];     // even CTA: both halves of the slot ready (2 forwards)
-  uint64_t empty[kStages];    // this CTA's slot read by its products (commit, both CTAs)
+  uint64_t k_landed[kRing];   // this CTA's K slot copied (tx)
+  uint64_t k_full[kRing];     // even CTA: both K halves of the slot ready (2 forwards)
+  uint64_t k_empty[kRing];    // the S product reading the slot done (commit, both CTAs)
+  uint64_t v_landed[kRing];   // the same for the V ring
+  uint64_t v_full[kRing];
+  uint64_t v_empty[kRing];    // the PV product reading the slot done (commit, both CTAs)
   uint64_t s_full[2];         // S buffer computed (commit, both CTAs)
-  uint64_t s_free[2];         // even CTA: S buffer read by all 8 softmax warps
-  uint64_t p_full[2];         // even CTA: P buffer written by all 8 softmax warps
+  uint64_t s_free[2];         // even CTA: S buffer read by all softmax warps
+  uint64_t p_full[2];         // even CTA: P buffer written by all softmax warps
   uint64_t pv_done[2];        // PV product from a P buffer done (commit, both CTAs)
-  uint64_t o_free;            // even CTA: O read by the epilogue (8 warps)
-  uint64_t item_full[2];      // work-item ring, written by the even CTA's producer
+  uint64_t o_free;            // even CTA: O read by the epilogue
+  uint64_t item_full[2];      // work-item ring, written by the even CTA's K producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: both issuers' last commits
   uint64_t xch[4];            // half-row softmax: the two warps of a quadrant exchanged
   int item_msg[2][8];         // a claimed item, decoded: it, b, tile, g, P, n, cu (it < 0: end)
+  int v_keys[kRing];          // keys of the step in each V slot (< 128: rows past it zeroed)
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -106,7 +112,8 @@ struct Bars2 {
 // Shared::cluster addresses of the barriers that live in the even CTA, and
 // of the peer's abort flag and item messages.
 struct Remote {
-  uint32_t q_full, full, s_free, p_full, o_free, item_empty, item_full, item_msg, abort_peer;
+  uint32_t q_full, k_full, v_full, s_free, p_full, o_free, item_empty, item_full, item_msg,
+      abort_peer;
 };
 
 struct Item2 {
@@ -200,8 +207,115 @@ __device__ __forceinline__ void raise_abort(Bars2& bar, const Remote& rm) {
   st_cluster_u32(rm.abort_peer, 1u);
 }
 
-// ------------------------------------------------------------------ producer
-__device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar,
+// ----------------------------------------------------------------- producers
+// Two producer warps per CTA: the K producer (this SM's Q half of each item
+// and its 64-key half of every K tile, one 4-D box per page bringing both
+// 64-column blocks) and the V producer (its 64-column half of every V tile,
+// one 2-D box per page).  Each fills its own ring of 16 KB slots, so that
+// neither waits behind the other's slot releases, and the two issue their
+// copies in parallel (a copy instruction costs its warp tens of cycles per
+// box, and 16-token pages need many boxes).
+//
+// Each producer also reports its own copies, in order, to the even CTA once
+// they have landed (a V slot whose step ends past the sequence gets its tail
+// rows zeroed first: their P is 0, but 0 * NaN is NaN).  It does so whenever
+// it would otherwise wait, so a slot can never wait on a report that the
+// producer, blocked on that slot, has not made.
+template <bool kIsK>
+struct Producer {
+  Bars2& bar;
+  const Remote& rm;
+  uint8_t* ring;         // kRing slots of 16 KB
+  uint64_t* landed;      // this CTA's landed barriers of the ring
+  uint64_t* empty;
+  uint32_t full_remote;  // even CTA's full barriers of the ring
+  volatile int* abortp;
+  int lane;
+  uint32_t issued = 0, fwd = 0;      // ring uses issued / reported
+  uint32_t q_issued = 0, q_fwd = 0;  // K producer: Q halves issued / reported
+
+  // lane 0's probe of a barrier phase, for the whole warp
+  __device__ __forceinline__ bool probe(uint64_t* b, uint32_t parity) {
+    const bool t = lane == 0 ? mbar_test(b, parity) : false;
+    return __shfl_sync(0xffffffffu, t, 0);
+  }
+
+  // Report landed copies in order; with `block`, wait (bounded) for all of
+  // them.  Returns false if the wait gave up.
+  __device__ bool forward(bool block) {
+    const long long t0 = clock64();
+    while (true) {
+      bool progress = false;
+      if (kIsK && q_fwd < q_issued) {
+        const uint32_t qb = q_fwd & 1;
+        if (probe(&bar.q_landed[qb], (q_fwd >> 1) & 1)) {
+          if (lane == 0) mbar_arrive_remote(rm.q_full + 8 * qb);
+          ++q_fwd;
+          progress = true;
+        }
+      }
+      if (fwd < issued) {
+        const uint32_t slot = fwd % kRing;
+        if (probe(&landed[slot], (fwd / kRing) & 1)) {
+          bool zeroed = false;
+          if (!kIsK) {
+            const int nkeys = bar.v_keys[slot];
+            if (nkeys < kKeys) {
+              uint4* z = reinterpret_cast<uint4*>(ring + slot * kSlotBytes + nkeys * 128);
+              for (int e = lane; e < (kKeys - nkeys) * 8; e += 32) z[e] = make_uint4(0, 0, 0, 0);
+              fence_proxy_async_smem();
+              zeroed = true;
+            }
+          }
+          __syncwarp();
+          // zeroed rows are generic-proxy writes the other SM's tensor core
+          // reads: publish them at cluster scope; a plain landed copy needs none
+          if (lane == 0) {
+            if (zeroed) mbar_arrive_cluster(full_remote + 8 * slot);
+            else mbar_arrive_remote(full_remote + 8 * slot);
+          }
+          ++fwd;
+          progress = true;
+        }
+      }
+      const bool done = fwd == issued && (!kIsK || q_fwd == q_issued);
+      if (done || (!block && !progress)) return true;
+      if (*abortp) return false;
+      if (clock64() - t0 > kWaitCycles) {
+        *abortp = 1;
+        return false;
+      }
+    }
+  }
+
+  // Wait (bounded) for a barrier phase, reporting landed copies meanwhile.
+  __device__ bool wait(uint64_t* b, uint32_t parity) {
+    const long long t0 = clock64();
+    while (!probe(b, parity)) {
+      if (!forward(false)) return false;
+      if (*abortp) return false;
+      if (clock64() - t0 > kWaitCycles) {
+        *abortp = 1;
+        return false;
+      }
+    }
+    return true;
+  }
+
+  // Copies in flight when the kernel gives up land before the CTA exits
+  // (bounded, ignores the abort flag).
+  __device__ void drain() {
+    if (lane != 0) return;
+    int no_abort = 0;
+    for (uint32_t q = q_fwd; kIsK && q < q_issued; ++q)
+      mbar_wait(&bar.q_landed[q & 1], (q >> 1) & 1, &no_abort);
+    for (uint32_t x = fwd; x < issued; ++x)
+      mbar_wait(&landed[x % kRing], (x / kRing) & 1, &no_abort);
+  }
+};
+
+template <bool kIsK>
+__device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Bars2& bar,
                           const Remote& rm, const int* item_start, int total_items,
                           const Geom2& geo, const CUtensorMap* map_q, const CUtensorMap* map_kv,
                           const int32_t* __restrict__ block_table,
@@ -210,23 +324,24 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars
                           const int32_t* __restrict__ cu_new_lens, int32_t* status,
                           int* work_counter) {
   const int lane = threadIdx.x & 31;
-  volatile int* abortp = &bar.abort_flag;
-  uint32_t use = 0;                      // ring uses so far (K at 2t, V at 2t+1)
-  uint32_t armed = 0, armed_par = 0;     // per slot: a copy in flight, and its phase parity
-  int armed_q = -1;
+  Producer<kIsK> pr{bar, rm, smem_ring, kIsK ? bar.k_landed : bar.v_landed,
+                    kIsK ? bar.k_empty : bar.v_empty, kIsK ? rm.k_full : rm.v_full,
+                    &bar.abort_flag, lane};
   bool ok = true;
-  const uint32_t box_bytes = static_cast<uint32_t>(geo.box_rows) * 128;
-  const int boxes_k = (64 >> geo.box_shift) * 2;  // K half: 64 keys x 2 column blocks
-  const int boxes_v = kKeys >> geo.box_shift;     // V half: 128 keys x 1 column block
+  // K: 64 keys of this CTA, one box (both column blocks) per box_rows keys;
+  // V: 128 keys of column block `rank`, one box per box_rows keys
+  const int nbox = kIsK ? (64 >> geo.box_shift) : (kKeys >> geo.box_shift);
+  const uint32_t box_bytes = static_cast<uint32_t>(geo.box_rows) * (kIsK ? 256 : 128);
   const int pages_per_step = kKeys >> geo.ps_shift;
+  const bool claims = kIsK && rank == 0;  // the even CTA's K producer claims the items
 
   for (uint32_t k = 0; ok; ++k) {
+    const int s = k & 1;
     int it = -1;
     Item2 w;
-    if (rank == 0) {
+    if (claims) {
       // claim the next item and send it, decoded, to every role of both CTAs
-      const int s = k & 1;
-      ok = wait_warp(&bar.item_empty[s], ((k >> 1) & 1) ^ 1, abortp);
+      ok = pr.wait(&bar.item_empty[s], ((k >> 1) & 1) ^ 1);
       if (!ok) break;
       int m[7];
       if (lane == 0) {
@@ -244,31 +359,42 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars
         mbar_arrive_cluster(rm.item_full + 8 * s);
       }
       __syncwarp();
-      it = read_item2(bar, k, geo, rank, w, abortp, ok);  // the message just written
+    } else {
+      ok = pr.wait(&bar.item_full[s], (k >> 1) & 1);
+      if (!ok) break;
+    }
+    {
+      // read the message (the even CTA's producer wrote it: acquire at cluster scope)
+      ok = mbar_wait_cluster(&bar.item_full[s], (k >> 1) & 1, &bar.abort_flag);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
-    } else {
-      it = read_item2_warp(bar, k, geo, rank, w, abortp, ok);
-      if (!ok) break;
+      const volatile int* mv = bar.item_msg[s];
+      int mm[7];
+#pragma unroll
+      for (int i = 0; i < 7; ++i) mm[i] = mv[i];
+      it = mm[0];
+      if (it >= 0) item_from_message(mm, geo, rank, w);
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
+      if (!claims && lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * s);
     }
     if (it < 0) break;
-    // ---- this CTA's Q half: 128 rows = 128/G tokens x G heads, two column blocks
-    const int qb = k & 1;
-    ok = wait_warp(&bar.q_empty[qb], ((k >> 1) & 1) ^ 1, abortp);
-    if (!ok) break;
-    if (lane == 0) {
-      mbar_arrive_expect_tx(&bar.q_landed[qb], kQBytes);
+    if (kIsK) {
+      // this CTA's Q half: 128 rows = 128/G tokens x G heads, two column blocks
+      const int qb = k & 1;
+      ok = pr.wait(&bar.q_empty[qb], ((k >> 1) & 1) ^ 1);
+      if (!ok) break;
+      if (lane == 0) {
+        mbar_arrive_expect_tx(&bar.q_landed[qb], kQBytes);
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
-        tma_load_3d(smem_q + qb * kQBytes + h * (kRows * 128), map_q, &bar.q_landed[qb], h * 64,
-                    w.g * geo.G, w.cu + w.tok0);
+        for (int h = 0; h < 2; ++h)
+          tma_load_3d(smem_q + qb * kQBytes + h * (kRows * 128), map_q, &bar.q_landed[qb],
+                      h * 64, w.g * geo.G, w.cu + w.tok0);
+      }
+      ++pr.q_issued;
     }
-    armed_q = qb | (((k >> 1) & 1) << 1);
-    // ---- K/V halves, step by step.  Lane i holds the block-table entry of
-    // page i of a step (-2: no such page before the end of the sequence);
-    // the next step's entries are loaded while this step's copies are issued.
+    // K/V steps.  Lane i holds the block-table entry of page i of a step
+    // (-2: no such page before the end of the sequence); the next step's
+    // entries are loaded while this step's copies are issued.
     const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
     auto lookup = [&](int j) -> int {
       const int key = j * kKeys + lane * geo.ps;  // first key of page `lane` of step j
@@ -276,109 +402,47 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_kv, Bars
       const int blk = key >> geo.ps_shift;
       return blk < geo.max_blocks ? __ldg(block_table + bt_row + blk) : -1;
     };
+    const int plane_row = (geo.layer * 2 + (kIsK ? 0 : 1)) * geo.num_pages;
     int pages = lookup(0);
     for (int j = 0; ok && j < w.nt; ++j) {
       const int key0 = j * kKeys;
       const int pages_next = j + 1 < w.nt ? lookup(j + 1) : -2;
-#pragma unroll 1
-      for (int kv = 0; kv < 2; ++kv) {
-        const int slot = use % kStages;
-        // box `lane`: K: column block lane & 1, rows of chunk lane >> 1 of
-        // this CTA's 64 keys; V: column block `rank`, chunk lane of 128 keys
-        const int nbox = kv == 0 ? boxes_k : boxes_v;
-        int ko = 0, col = 0, dst = 0;  // ko: first key of the box within the step
-        if (kv == 0) {
-          ko = static_cast<int>(rank) * 64 + (lane >> 1) * geo.box_rows;
-          col = (lane & 1) * 64;
-          dst = (lane & 1) * (64 * 128) + (lane >> 1) * geo.box_rows * 128;
+      // box `lane`: first key ko of the box within the step
+      const int ko = kIsK ? static_cast<int>(rank) * 64 + lane * geo.box_rows : lane * geo.box_rows;
+      const int page = __shfl_sync(0xffffffffu, pages, min(ko >> geo.ps_shift, 31));
+      int row = -1;
+      if (lane < nbox && page != -2 && key0 + ko < w.T) {
+        if (page < 0 || page >= geo.num_pages) {
+          record_error(status, GC_ERR_OUT_OF_RANGE);
         } else {
-          ko = lane * geo.box_rows;
-          col = static_cast<int>(rank) * 64;
-          dst = lane * geo.box_rows * 128;
+          row = (((plane_row + page) * geo.Hkv + w.g) << geo.ps_shift) +
+                ((key0 + ko) & (geo.ps - 1));
         }
-        const int page = __shfl_sync(0xffffffffu, pages, min(ko >> geo.ps_shift, 31));
-        int row = -1;
-        if (lane < nbox && page != -2 && key0 + ko < w.T) {
-          if (page < 0 || page >= geo.num_pages) {
-            record_error(status, GC_ERR_OUT_OF_RANGE);
-          } else {
-            const int plane_row = (geo.layer * 2 + kv) * geo.num_pages;
-            row = (((plane_row + page) * geo.Hkv + w.g) << geo.ps_shift) +
-                  ((key0 + ko) & (geo.ps - 1));
-          }
-        }
-        const int good = __popc(__ballot_sync(0xffffffffu, row >= 0));
-        ok = wait_warp(&bar.empty[slot], ((use / kStages) & 1) ^ 1, abortp);
-        if (!ok) break;
-        if (lane == 0) mbar_arrive_expect_tx(&bar.landed[slot], static_cast<uint32_t>(good) * box_bytes);
-        __syncwarp();
-        if (row >= 0) tma_load_2d(smem_kv + slot * kSlotBytes + dst, map_kv, &bar.landed[slot], col, row);
-        armed |= 1u << slot;
-        armed_par = (armed_par & ~(1u << slot)) | (((use / kStages) & 1u) << slot);
-        ++use;
       }
+      const int good = __popc(__ballot_sync(0xffffffffu, row >= 0));
+      const uint32_t x = pr.issued, slot = x % kRing;
+      ok = pr.wait(&pr.empty[slot], ((x / kRing) & 1) ^ 1);
+      if (!ok) break;
+      if (lane == 0) {
+        if (!kIsK) bar.v_keys[slot] = min(kKeys, w.T - key0);
+        mbar_arrive_expect_tx(&pr.landed[slot], static_cast<uint32_t>(good) * box_bytes);
+      }
+      __syncwarp();
+      uint8_t* dst = smem_ring + slot * kSlotBytes + lane * box_bytes;
+      if (row >= 0) {
+        if (kIsK)
+          tma_load_4d(dst, map_kv, &pr.landed[slot], 0, 0, 0, row >> 3);
+        else
+          tma_load_2d(dst, map_kv, &pr.landed[slot], static_cast<int>(rank) * 64, row);
+      }
+      ++pr.issued;
+      pr.forward(false);
       pages = pages_next;
     }
   }
-  if (!ok && lane == 0) {
-    // let this CTA's copies still in flight land before it exits (bounded,
-    // ignores the abort flag); a slot's copy may already have been waited
-    // for, in which case its phase has completed and the wait returns at once
-    int no_abort = 0;
-    if (armed_q >= 0) mbar_wait(&bar.q_landed[armed_q & 1], (armed_q >> 1) & 1, &no_abort);
-    for (int s = 0; s < kStages; ++s)
-      if (armed & (1u << s)) mbar_wait(&bar.landed[s], (armed_par >> s) & 1u, &no_abort);
-  }
-}
-
-// ----------------------------------------------------------------- forwarder
-// Reports each of this CTA's copies to the even CTA once it has landed (and,
-// for a V half that ends past the sequence, once its tail rows are zero).
-__device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
-                           const int* item_start, const Geom2& geo,
-                           const int32_t* __restrict__ prefix_lens,
-                           const int32_t* __restrict__ new_lens,
-                           const int32_t* __restrict__ cu_new_lens) {
-  const int lane = threadIdx.x & 31;
-  volatile int* abortp = &bar.abort_flag;
-  uint32_t use = 0;
-  bool ok = true;
-  for (uint32_t k = 0; ok; ++k) {
-    Item2 w;
-    const int it = read_item2_warp(bar, k, geo, rank, w, abortp, ok);
-    if (!ok) break;
-    __syncwarp();
-    if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
-    if (it < 0) break;
-    const int qb = k & 1;
-    ok = wait_warp(&bar.q_landed[qb], (k >> 1) & 1, abortp);
-    if (!ok) break;
-    __syncwarp();
-    if (lane == 0) mbar_arrive_remote(rm.q_full + 8 * qb);
-    for (int j = 0; ok && j < w.nt; ++j) {
-      for (int kv = 0; kv < 2; ++kv) {
-        const int slot = use % kStages;
-        ok = wait_warp(&bar.landed[slot], (use / kStages) & 1, abortp);
-        if (!ok) break;
-        const int nkeys = min(kKeys, w.T - j * kKeys);
-        const bool zero = kv == 1 && nkeys < kKeys;
-        if (zero) {
-          // V rows [nkeys, 128) of this CTA's column block (128 bytes each)
-          uint4* z = reinterpret_cast<uint4*>(smem_kv + slot * kSlotBytes + nkeys * 128);
-          for (int e = lane; e < (kKeys - nkeys) * 8; e += 32) z[e] = make_uint4(0, 0, 0, 0);
-          fence_proxy_async_smem();
-        }
-        __syncwarp();
-        // the zeroed rows are generic-proxy writes the other SM's tensor core
-        // reads: publish them at cluster scope; a plain landed copy needs no fence
-        if (lane == 0) {
-          if (zero) mbar_arrive_cluster(rm.full + 8 * slot);
-          else mbar_arrive_remote(rm.full + 8 * slot);
-        }
-        ++use;
-      }
-    }
-  }
+  // report every copy issued (the issuers wait for them), or drain on failure
+  if (ok) ok = pr.forward(true);
+  if (!ok) pr.drain();
 }
 
 // -------------------------------------------------------------- MMA issuers
@@ -393,10 +457,10 @@ __device__ void forwarder2(uint32_t rank, uint8_t* smem_kv, Bars2& bar, const Re
 // S issuer: S(t) once K(t) is in and the softmax has read S(t-2) out of the
 // buffer (which it does first thing in step t-2), so S runs up to two steps
 // ahead of the softmax.  Frees K slots and the Q buffer by commits.
-__device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const Remote& rm,
+__device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Remote& rm,
                           uint32_t tmem, const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
-  const uint32_t q_smem = smem_addr(smem_q), kv_smem = smem_addr(smem_kv);
+  const uint32_t q_smem = smem_addr(smem_q), k_smem = smem_addr(smem_k);
   uint32_t u = 0;  // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
@@ -412,23 +476,25 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const R
     const uint32_t u_last = u + w.nt - 1;
     for (; ok && u <= u_last; ++u) {
       const uint32_t sb = u & 1;
-      const uint32_t ku = 2 * u, slot = ku % kStages;
-      ok = mbar_wait(&bar.full[slot], (ku / kStages) & 1, abortp);
+      const uint32_t slot = u % kRing;
+      ok = mbar_wait(&bar.k_full[slot], (u / kRing) & 1, abortp);
       if (ok && u >= 2) ok = mbar_wait(&bar.s_free[sb], ((u - 2) >> 1) & 1, abortp);
       if (!ok) break;
       tc_fence_after();
-      const uint64_t dk = sdesc_sw128(kv_smem + slot * kSlotBytes, 16, 1024);
+      // K half: 8-key groups of 2 KB (the group's 8 rows of columns 0-63,
+      // then of columns 64-127), so 8-row groups are 2048 bytes apart
+      const uint64_t dk = sdesc_sw128(k_smem + slot * kSlotBytes, 16, 2048);
       const uint32_t d = tmem + kColS + sb * 128;
 #pragma unroll
       for (int kk = 0; kk < kD / 16; ++kk) {
         // 16-column steps: 32 bytes within a 128-byte row, then the next
-        // 64-column block (Q: 128 rows x 128 B, K half: 64 rows x 128 B)
-        constexpr uint32_t kQBlk = kRows * 128 >> 4, kKBlk = 64 * 128 >> 4;
+        // 64-column block (Q: 16 KB further, K: 1 KB further)
+        constexpr uint32_t kQBlk = kRows * 128 >> 4, kKBlk = 1024 >> 4;
         mma2_ss(d, dq + ((kk >> 2) * kQBlk + (kk & 3) * 2), dk + ((kk >> 2) * kKBlk + (kk & 3) * 2),
                 kIdescQK, kk > 0);
       }
       mma2_commit_mc(&bar.s_full[sb], 0x3);
-      mma2_commit_mc(&bar.empty[slot], 0x3);
+      mma2_commit_mc(&bar.k_empty[slot], 0x3);
       if (u == u_last) mma2_commit_mc(&bar.q_empty[qb], 0x3);
     }
   }
@@ -441,10 +507,10 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_kv, Bars2& bar, const R
 // PV issuer: O += P(t) V(t) once the softmax has written P(t) and V(t) is
 // in; an item's first product (which overwrites O) also waits until the
 // previous item's epilogue has read O.  Frees V slots by commits.
-__device__ void pv_issuer2(uint8_t* smem_kv, Bars2& bar, const Remote& rm, uint32_t tmem,
+__device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
                            const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
-  const uint32_t kv_smem = smem_addr(smem_kv);
+  const uint32_t v_smem = smem_addr(smem_v);
   uint32_t u = 0;  // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
@@ -456,21 +522,21 @@ __device__ void pv_issuer2(uint8_t* smem_kv, Bars2& bar, const Remote& rm, uint3
     const uint32_t u_first = u, u_last = u + w.nt - 1;
     for (; ok && u <= u_last; ++u) {
       const uint32_t pb = u & 1;
-      const uint32_t vu = 2 * u + 1, slot = vu % kStages;
+      const uint32_t slot = u % kRing;
       ok = mbar_wait(&bar.p_full[pb], (u >> 1) & 1, abortp);
-      if (ok) ok = mbar_wait(&bar.full[slot], (vu / kStages) & 1, abortp);
+      if (ok) ok = mbar_wait(&bar.v_full[slot], (u / kRing) & 1, abortp);
       const bool first = u == u_first;
       if (ok && first && k > 0) ok = mbar_wait(&bar.o_free, (k - 1) & 1, abortp);
       if (!ok) break;
       tc_fence_after();
-      const uint64_t dv = sdesc_sw128(kv_smem + slot * kSlotBytes, kSlotBytes, 1024);
+      const uint64_t dv = sdesc_sw128(v_smem + slot * kSlotBytes, kSlotBytes, 1024);
       const uint32_t a = tmem + kColP + pb * 64;
 #pragma unroll
       for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys = two 8-row groups of 1 KB
         mma2_ts(tmem + kColO, a + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
                 (!first || kk > 0) ? 1u : 0u);
       mma2_commit_mc(&bar.pv_done[pb], 0x3);
-      mma2_commit_mc(&bar.empty[slot], 0x3);
+      mma2_commit_mc(&bar.v_empty[slot], 0x3);
     }
   }
   mma2_commit_mc(&bar.drain, 0x1);
@@ -845,7 +911,8 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
 // ------------------------------------------------------------------- kernel
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap map_q,
-                    const __grid_constant__ CUtensorMap map_kv,
+                    const __grid_constant__ CUtensorMap map_k,
+                    const __grid_constant__ CUtensorMap map_v,
                     const int32_t* __restrict__ block_table,
                     const int32_t* __restrict__ prefix_lens,
                     const int32_t* __restrict__ new_lens,
@@ -855,8 +922,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* base = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   uint8_t* smem_q = base;                     // 2 x 32 KB
-  uint8_t* smem_kv = base + 2 * kQBytes;      // kStages x 16 KB
-  Bars2& bar = *reinterpret_cast<Bars2*>(smem_kv + kStages * kSlotBytes);
+  uint8_t* smem_k = base + 2 * kQBytes;       // K ring, kRing x 16 KB
+  uint8_t* smem_v = smem_k + kRing * kSlotBytes;  // V ring
+  Bars2& bar = *reinterpret_cast<Bars2*>(smem_v + kRing * kSlotBytes);
   int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
   int16_t* order = reinterpret_cast<int16_t*>(item_start + geo.batch + 1);
   // half-row softmax exchange area [2 buffers][2 halves][128 rows]
@@ -876,10 +944,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.item_full[i], 1);
       mbar_init(&bar.item_empty[i], kItemConsumers);
     }
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&bar.landed[s], 1);
-      mbar_init(&bar.full[s], 2);
-      mbar_init(&bar.empty[s], 1);
+    for (int s = 0; s < kRing; ++s) {
+      mbar_init(&bar.k_landed[s], 1);
+      mbar_init(&bar.k_full[s], 2);
+      mbar_init(&bar.k_empty[s], 1);
+      mbar_init(&bar.v_landed[s], 1);
+      mbar_init(&bar.v_full[s], 2);
+      mbar_init(&bar.v_empty[s], 1);
     }
     mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
     mbar_init(&bar.drain, 2);
@@ -889,7 +960,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&map_q);
-    prefetch_tensormap(&map_kv);
+    prefetch_tensormap(&map_k);
+    prefetch_tensormap(&map_v);
   }
   if (warp == 1) {
     tmem_alloc2(&bar.tmem_base, 512);
@@ -937,7 +1009,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   {
     const uint32_t lead = 0, peer = rank ^ 1u;
     rm.q_full = mapa(smem_addr(&bar.q_full[0]), lead);
-    rm.full = mapa(smem_addr(&bar.full[0]), lead);
+    rm.k_full = mapa(smem_addr(&bar.k_full[0]), lead);
+    rm.v_full = mapa(smem_addr(&bar.v_full[0]), lead);
     rm.s_free = mapa(smem_addr(&bar.s_free[0]), lead);
     rm.p_full = mapa(smem_addr(&bar.p_full[0]), lead);
     rm.o_free = mapa(smem_addr(&bar.o_free), lead);
@@ -954,16 +1027,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int total_items = item_start[geo.batch];
 
   if (warp == 0) {
-    producer2(rank, smem_q, smem_kv, bar, rm, item_start, total_items, geo, &map_q, &map_kv,
-              block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
+    producer2<true>(rank, smem_q, smem_k, bar, rm, item_start, total_items, geo, &map_q,
+                    &map_k, block_table, prefix_lens, new_lens, cu_new_lens, status,
+                    work_counter);
   } else if (warp == 1) {
-    if (rank == 0 && lane == 0) s_issuer2(smem_q, smem_kv, bar, rm, tmem, geo);
+    if (rank == 0 && lane == 0) s_issuer2(smem_q, smem_k, bar, rm, tmem, geo);
     __syncwarp();
   } else if (warp == 2) {
-    if (rank == 0 && lane == 0) pv_issuer2(smem_kv, bar, rm, tmem, geo);
+    if (rank == 0 && lane == 0) pv_issuer2(smem_v, bar, rm, tmem, geo);
     __syncwarp();
   } else if (warp == 3) {
-    forwarder2(rank, smem_kv, bar, rm, item_start, geo, prefix_lens, new_lens, cu_new_lens);
+    producer2<false>(rank, smem_q, smem_v, bar, rm, item_start, total_items, geo, &map_q,
+                     &map_v, block_table, prefix_lens, new_lens, cu_new_lens, status,
+                     work_counter);
   } else if (warp >= 4) {
     if (kHalfRows)
       softmax2h(rank, bar, rm, tmem, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
@@ -1000,7 +1076,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn2() {
 }
 
 size_t smem_bytes2(int batch) {
-  return 1024 + 2 * kQBytes + static_cast<size_t>(kStages) * kSlotBytes + sizeof(Bars2) +
+  return 1024 + 2 * kQBytes + static_cast<size_t>(2 * kRing) * kSlotBytes + sizeof(Bars2) +
          (static_cast<size_t>(batch) + 1) * sizeof(int) +
          (batch <= kSortMax ? kSortMax * sizeof(int16_t) : 0) + 2 * 2 * kRows * sizeof(uint16_t);
 }
@@ -1069,7 +1145,7 @@ gc_status launch_attn_tc2(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_
   if (pool_rows >= (1ull << 31))
     return fail(GC_ERR_UNSUPPORTED, "gc_prefix_prefill_attn: pool has %llu rows (limit 2^31)",
                 static_cast<unsigned long long>(pool_rows));
-  CUtensorMap map_q, map_kv;
+  CUtensorMap map_q, map_k, map_v;
   {
     cuuint64_t dims[3] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(geo.Hq),
                           static_cast<cuuint64_t>(geo.total_new)};
@@ -1085,15 +1161,31 @@ gc_status launch_attn_tc2(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_
       return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: q tensor map (CUresult %d)", (int)r);
   }
   {
+    // K: 4-D view of the pool rows as (64 columns, 8 rows, 2 column blocks,
+    // 8-row groups), one box per page (or per 64 keys of a 128-row page):
+    // both column blocks of box_rows rows, laid out as 8-row groups of 2 KB
+    cuuint64_t dims[4] = {64, 8, 2, pool_rows / 8};
+    cuuint64_t strides[3] = {static_cast<cuuint64_t>(kD) * 2, 128,
+                             8 * static_cast<cuuint64_t>(kD) * 2};
+    cuuint32_t box[4] = {64, 8, 2, static_cast<cuuint32_t>(geo.box_rows / 8)};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    CUresult r = enc(&map_k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, pool->data, dims, strides, box,
+                     es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: pool K tensor map (CUresult %d)", (int)r);
+  }
+  {
+    // V: 2-D view of the pool rows, one box of 64 columns x box_rows rows
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(kD), pool_rows};
     cuuint64_t strides[1] = {static_cast<cuuint64_t>(kD) * 2};
     cuuint32_t box[2] = {64, static_cast<cuuint32_t>(geo.box_rows)};
     cuuint32_t es[2] = {1, 1};
-    CUresult r = enc(&map_kv, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool->data, dims, strides, box,
+    CUresult r = enc(&map_v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, pool->data, dims, strides, box,
                      es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS)
-      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: pool tensor map (CUresult %d)", (int)r);
+      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: pool V tensor map (CUresult %d)", (int)r);
   }
   const size_t smem = smem_bytes2(a.batch);
   // the work items are claimed from the given counter (the pool's control
@@ -1112,7 +1204,7 @@ gc_status launch_attn_tc2(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_
   attr[0].val.clusterDim.z = 1;
   lc.attrs = attr;
   lc.numAttrs = 1;
-  e = cudaLaunchKernelEx(&lc, attn_tc2_kernel, map_q, map_kv, a.block_table, a.prefix_lens,
+  e = cudaLaunchKernelEx(&lc, attn_tc2_kernel, map_q, map_k, map_v, a.block_table, a.prefix_lens,
                          a.new_lens, a.cu_new_lens, static_cast<__nv_bfloat16*>(a.out), geo,
                          pool->status, work_counter);
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: launch");
