@@ -59,9 +59,8 @@ namespace {
 using namespace ptx;
 
 constexpr int kD = 128;
-// softmax by two warpgroups, half a row each (true), or one, whole rows (false)
-constexpr bool kHalfRows = true;
-constexpr int kSoftmaxWarps = kHalfRows ? 8 : 4;
+// softmax by two warpgroups, half a row each
+constexpr int kSoftmaxWarps = 8;
 constexpr int kThreads = 128 + 32 * kSoftmaxWarps;
 constexpr int kRows = 128;            // q rows per SM
 constexpr int kKeys = 128;            // keys per K/V step
@@ -72,7 +71,6 @@ constexpr int kSortMax = 512;
 constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
-constexpr float kSpecLimit = 9.223372036854775808e18f;  // 2^63, as in the single-SM kernel
 // consumers of the work-item ring: in each CTA the V producer and the
 // softmax warps, plus the two MMA issuers of the even CTA and the odd CTA's
 // K producer
@@ -90,10 +88,10 @@ struct Bars2 {
   uint64_t q_empty[2];        // the item's last S product done (commit, both CTAs)
   uint64_t k_landed[kRing];   // this CTA's K slot copied (tx)
   uint64_t k_full[kRing];     // even CTA: both K halves of the slot ready (2 forwards)
-  uint64_t k_empty[kRing];    // the S product reading the slot done (commit, both CTAs)
+  uint64_t k_empty[kRing];    // the S product reading the slot done (softmax thread 0)
   uint64_t v_landed[kRing];   // the same for the V ring
   uint64_t v_full[kRing];
-  uint64_t v_empty[kRing];    // the PV product reading the slot done (commit, both CTAs)
+  uint64_t v_empty[kRing];    // the PV product reading the slot done (softmax thread 0)
   uint64_t s_full[2];         // S buffer computed (commit, both CTAs)
   uint64_t s_free[2];         // even CTA: S buffer read by all softmax warps
   uint64_t p_full[2];         // even CTA: P buffer written by all softmax warps
@@ -102,7 +100,7 @@ struct Bars2 {
   uint64_t item_full[2];      // work-item ring, written by the even CTA's K producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: both issuers' last commits
-  uint64_t xch[4];            // half-row softmax: the two warps of a quadrant exchanged
+  uint32_t xseq[2][4];        // half-row softmax: exchanges published per warp
   int item_msg[2][8];         // a claimed item, decoded: it, b, tile, g, P, n, cu (it < 0: end)
   int v_keys[kRing];          // keys of the step in each V slot (< 128: rows past it zeroed)
   uint32_t tmem_base;
@@ -456,7 +454,8 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
 //
 // S issuer: S(t) once K(t) is in and the softmax has read S(t-2) out of the
 // buffer (which it does first thing in step t-2), so S runs up to two steps
-// ahead of the softmax.  Frees K slots and the Q buffer by commits.
+// ahead of the softmax.  Frees the Q buffer by a commit after the item's last
+// S product (the softmax frees the ring slots).
 __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Remote& rm,
                           uint32_t tmem, const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
@@ -494,7 +493,6 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
                 kIdescQK, kk > 0);
       }
       mma2_commit_mc(&bar.s_full[sb], 0x3);
-      mma2_commit_mc(&bar.k_empty[slot], 0x3);
       if (u == u_last) mma2_commit_mc(&bar.q_empty[qb], 0x3);
     }
   }
@@ -506,7 +504,7 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
 
 // PV issuer: O += P(t) V(t) once the softmax has written P(t) and V(t) is
 // in; an item's first product (which overwrites O) also waits until the
-// previous item's epilogue has read O.  Frees V slots by commits.
+// previous item's epilogue has read O.
 __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
                            const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
@@ -536,7 +534,6 @@ __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32
         mma2_ts(tmem + kColO, a + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
                 (!first || kk > 0) ? 1u : 0u);
       mma2_commit_mc(&bar.pv_done[pb], 0x3);
-      mma2_commit_mc(&bar.v_empty[slot], 0x3);
     }
   }
   mma2_commit_mc(&bar.drain, 0x1);
@@ -545,170 +542,6 @@ __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32
 }
 
 // ------------------------------------------------------------------ softmax
-__device__ __forceinline__ float tile_max2(const uint32_t (&sr)[4][32]) {
-  float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
-  for (int c = 0; c < 4; ++c)
-#pragma unroll
-    for (int e = 0; e < 32; e += 8) {
-      mx[0] = fmax3(mx[0], __uint_as_float(sr[c][e + 0]), __uint_as_float(sr[c][e + 1]));
-      mx[1] = fmax3(mx[1], __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
-      mx[2] = fmax3(mx[2], __uint_as_float(sr[c][e + 4]), __uint_as_float(sr[c][e + 5]));
-      mx[3] = fmax3(mx[3], __uint_as_float(sr[c][e + 6]), __uint_as_float(sr[c][e + 7]));
-    }
-  return fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
-}
-
-// p = 2^(s * scale*log2(e) - m) for one row of the tile, written to tensor
-// memory at tP as bf16 pairs (64 columns); returns sum p (fp32).
-__device__ __forceinline__ float tile_exp2(const uint32_t (&sr)[4][32], uint32_t tP,
-                                           float scale_log2, float m) {
-  const uint64_t sc2 = f2_pack(scale_log2, scale_log2);
-  const uint64_t nm2 = f2_pack(-m, -m);
-  uint64_t acc[4] = {0, 0, 0, 0};
-#pragma unroll
-  for (int c = 0; c < 4; ++c) {
-    uint32_t pk[16];
-#pragma unroll
-    for (int e = 0; e < 16; ++e) {
-      const uint64_t t = f2_fma(f2_pack(__uint_as_float(sr[c][2 * e]),
-                                        __uint_as_float(sr[c][2 * e + 1])), sc2, nm2);
-      float t0, t1;
-      f2_unpack(t, t0, t1);
-      const float p0 = ex2_approx(t0), p1 = ex2_approx(t1);
-      acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
-      pk[e] = pack_bf16x2(p0, p1);
-    }
-    tmem_st16(tP + c * 16, pk);
-  }
-  float s0, s1, s2, s3;
-  f2_unpack(f2_add(acc[0], acc[1]), s0, s1);
-  f2_unpack(f2_add(acc[2], acc[3]), s2, s3);
-  return (s0 + s2) + (s1 + s3);
-}
-
-__device__ void softmax2(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t tmem,
-                         const int* item_start, const Geom2& geo,
-                         const int32_t* __restrict__ prefix_lens,
-                         const int32_t* __restrict__ new_lens,
-                         const int32_t* __restrict__ cu_new_lens,
-                         __nv_bfloat16* __restrict__ out) {
-  volatile int* abortp = &bar.abort_flag;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int r = threadIdx.x - 128;  // q row of this CTA's half = tensor-memory lane
-  const uint32_t lane_addr = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
-  uint32_t u = 0;           // global step counter
-  bool ok = true;
-  for (uint32_t k = 0; ok; ++k) {
-    Item2 w;
-    const int it = read_item2_warp(bar, k, geo, rank, w, abortp, ok);
-    if (!ok) break;
-    __syncwarp();
-    if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
-    if (it < 0) break;
-    const int tok = w.tok0 + r / geo.G;
-    const bool row_valid = tok < w.n;
-    const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
-    float m_run = -INFINITY, l = 0.f;
-    const float sl2 = geo.scale_log2;
-    for (int j = 0; j < w.nt; ++j, ++u) {
-      const uint32_t sb = u & 1;
-      const uint32_t tS = lane_addr + kColS + sb * 128;
-      const uint32_t tP = lane_addr + kColP + sb * 64;
-      ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
-      if (!ok) break;
-      tc_fence_after();
-      uint32_t sr[4][32];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
-      tmem_wait_ld();
-      // S buffer free for S(u+2)
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_remote(rm.s_free + 8 * sb);
-      const int key0 = j * kKeys;
-      if (key0 + kKeys - 1 > kmax) {
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (key0 + c * 32 + e > kmax) sr[c][e] = __float_as_uint(-INFINITY);
-      }
-      // P buffer sb is free once PV(u-2) is done
-      if (u >= 2) {
-        ok = wait_warp(&bar.pv_done[sb], ((u - 2) >> 1) & 1, abortp);
-        if (!ok) break;
-      }
-      float lt;
-      if (j == 0) {
-        // first tile of the row: exact max (key 0 is always visible)
-        m_run = tile_max2(sr) * sl2;
-        lt = tile_exp2(sr, tP, sl2, m_run);
-      } else {
-        lt = tile_exp2(sr, tP, sl2, m_run);
-        if (__any_sync(0xffffffffu, !(lt < kSpecLimit))) {
-          // O must hold every earlier step before it is rescaled
-          ok = wait_warp(&bar.pv_done[(u - 1) & 1], ((u - 1) >> 1) & 1, abortp);
-          if (!ok) break;
-          tmem_wait_st();
-          tc_fence_after();
-          const float m_new = fmaxf(m_run, tile_max2(sr) * sl2);
-          const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
-#pragma unroll 1
-          for (int c = 0; c < kD / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32(lane_addr + kColO + c * 32, o);
-            tmem_wait_ld();
-#pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-            tmem_st32(lane_addr + kColO + c * 32, o);
-          }
-          l *= alpha;
-          m_run = m_new;
-          lt = tile_exp2(sr, tP, sl2, m_run);
-        }
-      }
-      l += lt;
-      // publish P(u)
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_remote(rm.p_full + 8 * sb);
-    }
-    if (!ok) break;
-    // ---- epilogue: O / l -> bf16, once the item's last PV is done
-    const uint32_t ul = u - 1;
-    ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
-    if (!ok) break;
-    tc_fence_after();
-    const int h = w.g * geo.G + r % geo.G;
-    const float inv_l = 1.f / l;
-    uint4* orow = reinterpret_cast<uint4*>(
-        out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * kD);
-#pragma unroll 1
-    for (int c = 0; c < kD / 32; ++c) {
-      uint32_t o[32];
-      tmem_ld32(lane_addr + kColO + c * 32, o);
-      tmem_wait_ld();
-      if (row_valid) {
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          uint4 pk;
-          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
-          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
-          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
-          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
-          orow[c * 4 + v] = pk;
-        }
-      }
-    }
-    // O may now be overwritten by the next item's first PV
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive_remote(rm.o_free);
-  }
-}
-
 // Half-row softmax: two warpgroups, warps 4-7 taking key columns [0, 64)
 // and warps 8-11 columns [64, 128) of every row of this CTA (warps w and
 // w + 4 share the tensor-memory lanes of quadrant w & 3).  Each thread
@@ -743,21 +576,47 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
   const int r = quad * 32 + lane;          // q row of this CTA's half = tensor-memory lane
   const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quad * 32) << 16);
   uint32_t xn = 0;  // exchanges so far
-  // The partner thread's value (same row, other half): both warps of the
-  // quadrant write, then arrive once each on the quadrant's barrier (bounded
-  // wait).  Values are double-buffered: a warp that runs ahead writes the
-  // other buffer, and cannot come back to this one before its partner has
-  // arrived for the exchange after, i.e. has read this one.
+  volatile uint32_t* my_seq = &bar.xseq[hw][quad];
+  volatile uint32_t* other_seq = &bar.xseq[hw ^ 1][quad];
+  // The partner thread's value (same row, other half): each warp writes its
+  // 32 values, then its lane 0 publishes the exchange count; the warp spins
+  // (bounded) until the partner warp's count has caught up.  Values are
+  // double-buffered: a warp that runs ahead writes the other buffer, and
+  // cannot come back to this one before its partner has published the
+  // exchange after, which it does only once it has read this one.
   auto exchange = [&](uint16_t v, bool& good) -> uint16_t {
     const uint32_t xb = xn & 1;
     xch[(xb * 2 + hw) * kRows + r] = v;
     __syncwarp();
-    if (lane == 0) mbar_arrive(&bar.xch[quad]);
-    good = wait_warp(&bar.xch[quad], xn & 1, abortp);
     ++xn;
+    if (lane == 0) {
+      __threadfence_block();
+      *my_seq = xn;
+    }
+    bool ok_ = true;
+    const long long t0 = clock64();
+    while (*other_seq < xn) {
+      if (*abortp || clock64() - t0 > kWaitCycles) {
+        *abortp = 1;
+        ok_ = false;
+        break;
+      }
+    }
+    __threadfence_block();
+    good = __all_sync(0xffffffffu, ok_);
     return xch[(xb * 2 + (hw ^ 1)) * kRows + r];
   };
   uint32_t u = 0;  // global step counter
+  // One thread per CTA frees ring slots once the products that read them are
+  // known complete: K(u) when S(u) is, V(u) when PV(u) is (steps below
+  // v_released are freed).  This keeps the frees out of the tensor pipe's
+  // instruction stream, whose issue rate bounds the kernel.
+  const bool rel = warp == 4 && lane == 0;
+  uint32_t v_released = 0;
+  auto release_v_upto = [&](uint32_t v) {
+    if (rel)
+      for (; v_released <= v; ++v_released) mbar_arrive(&bar.v_empty[v_released % kRing]);
+  };
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
     Item2 w;
@@ -777,6 +636,7 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
       const uint32_t tP = lane_addr + kColP + sb * 64 + hw * 32;
       ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
       if (!ok) break;
+      if (rel) mbar_arrive(&bar.k_empty[u % kRing]);
       tc_fence_after();
       uint32_t sr[2][32];
       tmem_ld32(tS, sr[0]);
@@ -816,6 +676,7 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
         // each row take the same decision from the same two maxima
         ok = wait_warp(&bar.pv_done[(u - 1) & 1], ((u - 1) >> 1) & 1, abortp);
         if (!ok) break;
+        release_v_upto(u - 1);
         tc_fence_after();
         const float m_new = fmaxf(m_run, mt);
         const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
@@ -836,6 +697,7 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
       if (u >= 2) {
         ok = wait_warp(&bar.pv_done[sb], ((u - 2) >> 1) & 1, abortp);
         if (!ok) break;
+        release_v_upto(u - 2);
       }
       {
         const uint64_t sc2 = f2_pack(sl2, sl2);
@@ -879,6 +741,7 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     const uint32_t ul = u - 1;
     ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
     if (!ok) break;
+    release_v_upto(ul);
     tc_fence_after();
     const int h = w.g * geo.G + r % geo.G;
     const float inv_l = 1.f / l_row;
@@ -954,7 +817,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
     mbar_init(&bar.drain, 2);
-    for (int q = 0; q < 4; ++q) mbar_init(&bar.xch[q], 2);
+    for (int q = 0; q < 8; ++q) bar.xseq[q >> 2][q & 3] = 0;
     bar.abort_flag = 0;
     fence_barrier_init();
   }
@@ -1041,11 +904,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                      &map_v, block_table, prefix_lens, new_lens, cu_new_lens, status,
                      work_counter);
   } else if (warp >= 4) {
-    if (kHalfRows)
-      softmax2h(rank, bar, rm, tmem, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
-                out);
-    else
-      softmax2(rank, bar, rm, tmem, item_start, geo, prefix_lens, new_lens, cu_new_lens, out);
+    softmax2h(rank, bar, rm, tmem, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
+              out);
   }
   // a CTA that gave up tells its peer, so that the peer's roles leave their
   // loops instead of waiting for arrivals that will not come
