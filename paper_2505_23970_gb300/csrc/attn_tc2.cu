@@ -63,13 +63,15 @@ constexpr int kD = 128;
 constexpr int kSoftmaxWarps = 8;
 constexpr int kThreads = 128 + 32 * kSoftmaxWarps;
 constexpr int kRows = 128;            // q rows per SM
-constexpr int kKeys = 256;            // keys per K/V step: one S product
-constexpr int kHalfKeys = kKeys / 2;  // keys of each K tile an SM holds (B split by columns)
-constexpr int kRing = 2;              // slots of 32 KB in each of the K and V rings
-constexpr int kSlotBytes = 32768;
+constexpr int kKeys = 128;            // keys per K/V step
+constexpr int kRing = 4;              // slots of 16 KB in each of the K and V rings
+constexpr int kSlotBytes = 16384;
 constexpr int kQBytes = kRows * kD * 2;  // 32 KB: two 64-column blocks of 128 rows
 constexpr int kSortMax = 512;
-constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;  // S 256 columns, O 128, P 128
+// tensor-memory columns: S (one buffer, the softmax empties it at once), O as
+// two accumulators (even / odd 16-key steps of every PV product, so that the
+// two halves of a product accumulate independently), P double-buffered
+constexpr uint32_t kColS = 0, kColOa = 128, kColOb = 256, kColP = 384;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 // consumers of the work-item ring: in each CTA the V producer and the
@@ -95,15 +97,15 @@ struct Bars2 {
   uint64_t v_empty[kRing];    // the PV product reading the slot done (softmax thread 0)
   uint64_t s_full;            // S computed (commit, both CTAs)
   uint64_t s_free;            // even CTA: S read out by all softmax warps
-  uint64_t p_full;            // even CTA: P written by all softmax warps
-  uint64_t pv_done;           // PV product done: P and O free (commit, both CTAs)
+  uint64_t p_full[2];         // even CTA: P buffer written by all softmax warps
+  uint64_t pv_done[2];        // PV product from a P buffer done (commit, both CTAs)
   uint64_t o_free;            // even CTA: O read by the epilogue
   uint64_t item_full[2];      // work-item ring, written by the even CTA's K producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: both issuers' last commits
   uint32_t xseq[2][4];        // half-row softmax: exchanges published per warp
   int item_msg[2][8];         // a claimed item, decoded: it, b, tile, g, P, n, cu (it < 0: end)
-  int v_keys[kRing];          // keys of the step in each V slot (< 256: rows past it zeroed)
+  int v_keys[kRing];          // keys of the step in each V slot (< 128: rows past it zeroed)
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -314,7 +316,7 @@ struct Producer {
 };
 
 template <bool kIsK>
-__device__ __forceinline__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Bars2& bar,
+__device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Bars2& bar,
                           const Remote& rm, const int* item_start, int total_items,
                           const Geom2& geo, const CUtensorMap* map_q, const CUtensorMap* map_kv,
                           const int32_t* __restrict__ block_table,
@@ -327,9 +329,9 @@ __device__ __forceinline__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_
                     kIsK ? bar.k_empty : bar.v_empty, kIsK ? rm.k_full : rm.v_full,
                     &bar.abort_flag, lane};
   bool ok = true;
-  // K: 128 keys of this CTA, one box (both column blocks) per box_rows keys;
-  // V: 256 keys of column block `rank`, one box per box_rows keys
-  const int nbox = kIsK ? (kHalfKeys >> geo.box_shift) : (kKeys >> geo.box_shift);
+  // K: 64 keys of this CTA, one box (both column blocks) per box_rows keys;
+  // V: 128 keys of column block `rank`, one box per box_rows keys
+  const int nbox = kIsK ? (64 >> geo.box_shift) : (kKeys >> geo.box_shift);
   const uint32_t box_bytes = static_cast<uint32_t>(geo.box_rows) * (kIsK ? 256 : 128);
   const int pages_per_step = kKeys >> geo.ps_shift;
   const bool claims = kIsK && rank == 0;  // the even CTA's K producer claims the items
@@ -407,8 +409,7 @@ __device__ __forceinline__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_
       const int key0 = j * kKeys;
       const int pages_next = j + 1 < w.nt ? lookup(j + 1) : -2;
       // box `lane`: first key ko of the box within the step
-      const int ko = kIsK ? static_cast<int>(rank) * kHalfKeys + lane * geo.box_rows
-                          : lane * geo.box_rows;
+      const int ko = kIsK ? static_cast<int>(rank) * 64 + lane * geo.box_rows : lane * geo.box_rows;
       const int page = __shfl_sync(0xffffffffu, pages, min(ko >> geo.ps_shift, 31));
       int row = -1;
       if (lane < nbox && page != -2 && key0 + ko < w.T) {
@@ -448,17 +449,17 @@ __device__ __forceinline__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_
 // -------------------------------------------------------------- MMA issuers
 // Two threads of the even CTA, in different warps, issue the pair's MMAs:
 // one the S products, one the PV products.  They touch disjoint tensor
-// memory (S / P and O) and disjoint rings (K / V), so they need no order
-// between them, and the tensor pipe interleaves the two streams (a stream
-// of products into one accumulator runs well below the pipe's rate).
-// Operand descriptors are built once per tile and advanced by constant
-// offsets.
+// memory (S buffers / P buffers and O) and disjoint ring slots (K / V), so
+// they need no order between them, and a single thread issuing both (each
+// tcgen05.mma costs its issuing thread tens of cycles) could not keep the
+// tensor pipe busy.  Operand descriptors are built once per tile and
+// advanced by constant offsets.
 //
-// S issuer: S(t) = Q K(t)^T over the step's 256 keys (N = 256: each SM holds
-// 128 of the keys), once K(t) is in and the softmax has read S(t-1) out of
-// the buffer, which it does first thing in step t-1.  Frees the Q buffer by
-// a commit after the item's last S product (the softmax frees the rings).
-__device__ __forceinline__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Remote& rm,
+// S issuer: S(t) once K(t) is in and the softmax has read S(t-1) out of the
+// buffer, which it does first thing in step t-1, so S(t) is computed while
+// the softmax works on step t-1.  Frees the Q buffer by a commit after the item's last
+// S product (the softmax frees the ring slots).
+__device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Remote& rm,
                           uint32_t tmem, const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
   const uint32_t q_smem = smem_addr(smem_q), k_smem = smem_addr(smem_k);
@@ -484,13 +485,14 @@ __device__ __forceinline__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars
       // K half: 8-key groups of 2 KB (the group's 8 rows of columns 0-63,
       // then of columns 64-127), so 8-row groups are 2048 bytes apart
       const uint64_t dk = sdesc_sw128(k_smem + slot * kSlotBytes, 16, 2048);
+      const uint32_t d = tmem + kColS;
 #pragma unroll
       for (int kk = 0; kk < kD / 16; ++kk) {
         // 16-column steps: 32 bytes within a 128-byte row, then the next
         // 64-column block (Q: 16 KB further, K: 1 KB further)
         constexpr uint32_t kQBlk = kRows * 128 >> 4, kKBlk = 1024 >> 4;
-        mma2_ss(tmem + kColS, dq + ((kk >> 2) * kQBlk + (kk & 3) * 2),
-                dk + ((kk >> 2) * kKBlk + (kk & 3) * 2), kIdescQK, kk > 0);
+        mma2_ss(d, dq + ((kk >> 2) * kQBlk + (kk & 3) * 2), dk + ((kk >> 2) * kKBlk + (kk & 3) * 2),
+                kIdescQK, kk > 0);
       }
       mma2_commit_mc(&bar.s_full, 0x3);
       if (u == u_last) mma2_commit_mc(&bar.q_empty[qb], 0x3);
@@ -502,10 +504,10 @@ __device__ __forceinline__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars
   mbar_wait(&bar.drain, 0, &no_abort);
 }
 
-// PV issuer: O += P(t) V(t) over the step's 256 keys once the softmax has
-// written P(t) and V(t) is in; an item's first product (which overwrites O)
-// also waits until the previous item's epilogue has read O.
-__device__ __forceinline__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
+// PV issuer: O += P(t) V(t) once the softmax has written P(t) and V(t) is
+// in; an item's first product (which overwrites O) also waits until the
+// previous item's epilogue has read O.
+__device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
                            const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
   const uint32_t v_smem = smem_addr(smem_v);
@@ -519,19 +521,21 @@ __device__ __forceinline__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Re
     if (it < 0) break;
     const uint32_t u_first = u, u_last = u + w.nt - 1;
     for (; ok && u <= u_last; ++u) {
+      const uint32_t pb = u & 1;
       const uint32_t slot = u % kRing;
-      ok = mbar_wait(&bar.p_full, u & 1, abortp);
+      ok = mbar_wait(&bar.p_full[pb], (u >> 1) & 1, abortp);
       if (ok) ok = mbar_wait(&bar.v_full[slot], (u / kRing) & 1, abortp);
       const bool first = u == u_first;
       if (ok && first && k > 0) ok = mbar_wait(&bar.o_free, (k - 1) & 1, abortp);
       if (!ok) break;
       tc_fence_after();
       const uint64_t dv = sdesc_sw128(v_smem + slot * kSlotBytes, kSlotBytes, 1024);
+      const uint32_t a = tmem + kColP + pb * 64;
 #pragma unroll
       for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys = two 8-row groups of 1 KB
-        mma2_ts(tmem + kColO, tmem + kColP + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
-                (!first || kk > 0) ? 1u : 0u);
-      mma2_commit_mc(&bar.pv_done, 0x3);
+        mma2_ts(tmem + ((kk & 1) ? kColOb : kColOa), a + kk * 8, dv + kk * (2048 >> 4),
+                kIdescPV, (!first || kk > 1) ? 1u : 0u);
+      mma2_commit_mc(&bar.pv_done[pb], 0x3);
     }
   }
   mma2_commit_mc(&bar.drain, 0x1);
@@ -539,15 +543,14 @@ __device__ __forceinline__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Re
   mbar_wait(&bar.drain, 0, &no_abort);
 }
 
-// Half-row softmax: two warpgroups, warps 4-7 taking keys [0, 128) and
-// warps 8-11 keys [128, 256) of every step, for every row of this CTA
-// (warps w and w + 4 share the tensor-memory lanes of quadrant w & 3).  A
-// step: load this half of the row's S and release the S buffer at once (the
-// next S product may start), mask, agree with the other half on the row's
-// reference max through a per-step exchange in shared memory, compute the
-// 128 probabilities into registers, and only then wait for the previous
-// step's PV product to release the P buffer (and O), store P and publish
-// it.  The two halves add their partial sums at the end.
+// ------------------------------------------------------------------ softmax
+// Half-row softmax: two warpgroups, warps 4-7 taking key columns [0, 64)
+// and warps 8-11 columns [64, 128) of every row of this CTA (warps w and
+// w + 4 share the tensor-memory lanes of quadrant w & 3).  Each thread
+// exponentiates 64 scores per step, so a step's softmax takes about half the
+// time; the two halves of a row agree on its reference max through a
+// per-step exchange of their half-tile maxima in shared memory (a 64-thread
+// named barrier per quadrant), and add their partial sums at the end.
 constexpr float kRescaleLog2 = 56.f;  // a term above 2^56 against the reference max
 
 // fp32 -> bf16 bits rounded toward +inf (finite and infinite inputs)
@@ -561,16 +564,19 @@ __device__ __forceinline__ float bf16_bits_to_f32(uint16_t b) {
   return __uint_as_float(static_cast<uint32_t>(b) << 16);
 }
 
-__device__ __forceinline__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t tmem,
-                          uint16_t* xch, const Geom2& geo, __nv_bfloat16* __restrict__ out) {
+
+__device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t tmem,
+                          uint16_t* xch, const int* item_start, const Geom2& geo,
+                          const int32_t* __restrict__ prefix_lens,
+                          const int32_t* __restrict__ new_lens,
+                          const int32_t* __restrict__ cu_new_lens,
+                          __nv_bfloat16* __restrict__ out) {
   volatile int* abortp = &bar.abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int hw = (warp - 4) >> 2;          // which 128 keys of a step
+  const int hw = (warp - 4) >> 2;          // which 64 key columns
   const int quad = warp & 3;
   const int r = quad * 32 + lane;          // q row of this CTA's half = tensor-memory lane
   const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-  const uint32_t tS = lane_addr + kColS + hw * kHalfKeys;
-  const uint32_t tP = lane_addr + kColP + hw * (kHalfKeys / 2);
   uint32_t xn = 0;  // exchanges so far
   volatile uint32_t* my_seq = &bar.xseq[hw][quad];
   volatile uint32_t* other_seq = &bar.xseq[hw ^ 1][quad];
@@ -602,17 +608,17 @@ __device__ __forceinline__ void softmax2h(uint32_t rank, Bars2& bar, const Remot
     good = __all_sync(0xffffffffu, ok_);
     return xch[(xb * 2 + (hw ^ 1)) * kRows + r];
   };
+  uint32_t u = 0;  // global step counter
   // One thread per CTA frees ring slots once the products that read them are
   // known complete: K(u) when S(u) is, V(u) when PV(u) is (steps below
   // v_released are freed).  This keeps the frees out of the tensor pipe's
-  // instruction stream.
+  // instruction stream, whose issue rate bounds the kernel.
   const bool rel = warp == 4 && lane == 0;
   uint32_t v_released = 0;
   auto release_v_upto = [&](uint32_t v) {
     if (rel)
       for (; v_released <= v; ++v_released) mbar_arrive(&bar.v_empty[v_released % kRing]);
   };
-  uint32_t u = 0;  // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
     Item2 w;
@@ -627,78 +633,80 @@ __device__ __forceinline__ void softmax2h(uint32_t rank, Bars2& bar, const Remot
     float m_run = -INFINITY, l = 0.f;
     const float sl2 = geo.scale_log2;
     for (int j = 0; j < w.nt; ++j, ++u) {
+      const uint32_t sb = u & 1;
+      const uint32_t tS = lane_addr + kColS + hw * 64;
+      const uint32_t tP = lane_addr + kColP + sb * 64 + hw * 32;
       ok = wait_warp(&bar.s_full, u & 1, abortp);
       if (!ok) break;
       if (rel) mbar_arrive(&bar.k_empty[u % kRing]);
       tc_fence_after();
-      uint32_t sr[4][32];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, sr[c]);
+      uint32_t sr[2][32];
+      tmem_ld32(tS, sr[0]);
+      tmem_ld32(tS + 32, sr[1]);
       tmem_wait_ld();
       // the S buffer is free for S(u+1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(rm.s_free);
-      const int key0 = j * kKeys + hw * kHalfKeys;
-      if (key0 + kHalfKeys - 1 > kmax) {
+      const int key0 = j * kKeys + hw * 64;
+      if (key0 + 63 > kmax) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
+        for (int c = 0; c < 2; ++c)
 #pragma unroll
           for (int e = 0; e < 32; ++e)
             if (key0 + c * 32 + e > kmax) sr[c][e] = __float_as_uint(-INFINITY);
       }
-      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      float mh0 = -INFINITY, mh1 = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 4; ++c)
+      for (int c = 0; c < 2; ++c)
 #pragma unroll
-        for (int e = 0; e < 32; e += 2)
-          mx[c] = fmax3(mx[c], __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
+        for (int e = 0; e < 32; e += 4) {
+          mh0 = fmax3(mh0, __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
+          mh1 = fmax3(mh1, __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
+        }
       // this half's max, rounded up to bf16 (16 bits to exchange); both
       // halves of the row then take the max of the same two rounded values,
       // a reference at or above the row's true tile max
-      const uint16_t mh = bf16_bits_ru(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])));
+      const uint16_t mh = bf16_bits_ru(fmaxf(mh0, mh1));
       const uint16_t mo = exchange(mh, ok);
       if (!ok) break;
       const float mt = fmaxf(bf16_bits_to_f32(mh), bf16_bits_to_f32(mo)) * sl2;
       if (j == 0) {
         m_run = mt;  // first tile of the row: exact max (key 0 is always visible)
       } else if (__any_sync(0xffffffffu, mt - m_run > kRescaleLog2)) {
-        // rescale O, which must hold every earlier step first (both halves of
-        // each row take the same decision from the same two maxima)
-        ok = wait_warp(&bar.pv_done, (u - 1) & 1, abortp);
+        // O must hold every earlier step before it is rescaled; both halves of
+        // each row take the same decision from the same two maxima
+        ok = wait_warp(&bar.pv_done[(u - 1) & 1], ((u - 1) >> 1) & 1, abortp);
         if (!ok) break;
         release_v_upto(u - 1);
         tc_fence_after();
         const float m_new = fmaxf(m_run, mt);
         const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
 #pragma unroll 1
-        for (int c = 0; c < 2; ++c) {
+        for (int c = 0; c < 4; ++c) {  // this half's 64 columns of both accumulators
           uint32_t o[32];
-          const uint32_t tO = lane_addr + kColO + hw * 64 + c * 32;
+          const uint32_t tO = lane_addr + ((c & 2) ? kColOb : kColOa) + hw * 64 + (c & 1) * 32;
           tmem_ld32(tO, o);
           tmem_wait_ld();
 #pragma unroll
           for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
           tmem_st32(tO, o);
         }
-        tmem_wait_st();
         l *= alpha;
         m_run = m_new;
       }
-      // the P buffer is free once PV(u-1) is done
-      if (u >= 1) {
-        ok = wait_warp(&bar.pv_done, (u - 1) & 1, abortp);
+      // P buffer sb is free once PV(u-2) is done
+      if (u >= 2) {
+        ok = wait_warp(&bar.pv_done[sb], ((u - 2) >> 1) & 1, abortp);
         if (!ok) break;
-        release_v_upto(u - 1);
+        release_v_upto(u - 2);
       }
-      tc_fence_after();
-      // probabilities of this half row, stored to the P buffer as bf16 pairs
       {
         const uint64_t sc2 = f2_pack(sl2, sl2);
         const uint64_t nm2 = f2_pack(-m_run, -m_run);
         uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < 2; ++c) {
           uint32_t pk[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
@@ -721,7 +729,7 @@ __device__ __forceinline__ void softmax2h(uint32_t rank, Bars2& bar, const Remot
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_remote(rm.p_full);
+      if (lane == 0) mbar_arrive_remote(rm.p_full + 8 * sb);
     }
     if (!ok) break;
     // ---- epilogue: O / l -> bf16 (this half's 64 columns), once the item's last PV is done
@@ -733,7 +741,7 @@ __device__ __forceinline__ void softmax2h(uint32_t rank, Bars2& bar, const Remot
     if (!ok) break;
     const float l_row = l + __uint_as_float((lo_hi << 16) | lo_lo);
     const uint32_t ul = u - 1;
-    ok = wait_warp(&bar.pv_done, ul & 1, abortp);
+    ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
     if (!ok) break;
     release_v_upto(ul);
     tc_fence_after();
@@ -743,18 +751,23 @@ __device__ __forceinline__ void softmax2h(uint32_t rank, Bars2& bar, const Remot
         out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * kD + hw * 64);
 #pragma unroll 1
     for (int c = 0; c < 2; ++c) {
-      uint32_t o[32];
-      tmem_ld32(lane_addr + kColO + hw * 64 + c * 32, o);
+      // O = the two accumulators added
+      uint32_t o[32], o2[32];
+      tmem_ld32(lane_addr + kColOa + hw * 64 + c * 32, o);
+      tmem_ld32(lane_addr + kColOb + hw * 64 + c * 32, o2);
       tmem_wait_ld();
+#pragma unroll
+      for (int e = 0; e < 32; ++e)
+        o[e] = __float_as_uint(__uint_as_float(o[e]) + __uint_as_float(o2[e]));
       if (row_valid) {
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
-          uint4 q;
-          q.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
-          q.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
-          q.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
-          q.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
-          orow[c * 4 + v] = q;
+          uint4 pk;
+          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+          orow[c * 4 + v] = pk;
         }
       }
     }
@@ -790,10 +803,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t rank = cluster_ctarank();
 
   if (threadIdx.x == 0) {
+    mbar_init(&bar.s_full, 1);
+    mbar_init(&bar.s_free, 2 * kSoftmaxWarps);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bar.q_landed[i], 1);
       mbar_init(&bar.q_full[i], 2);
       mbar_init(&bar.q_empty[i], 1);
+      mbar_init(&bar.p_full[i], 2 * kSoftmaxWarps);
+      mbar_init(&bar.pv_done[i], 1);
       mbar_init(&bar.item_full[i], 1);
       mbar_init(&bar.item_empty[i], kItemConsumers);
     }
@@ -805,10 +822,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.v_full[s], 2);
       mbar_init(&bar.v_empty[s], 1);
     }
-    mbar_init(&bar.s_full, 1);
-    mbar_init(&bar.s_free, 2 * kSoftmaxWarps);
-    mbar_init(&bar.p_full, 2 * kSoftmaxWarps);
-    mbar_init(&bar.pv_done, 1);
     mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
     mbar_init(&bar.drain, 2);
     for (int q = 0; q < 8; ++q) bar.xseq[q >> 2][q & 3] = 0;
@@ -869,7 +882,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     rm.k_full = mapa(smem_addr(&bar.k_full[0]), lead);
     rm.v_full = mapa(smem_addr(&bar.v_full[0]), lead);
     rm.s_free = mapa(smem_addr(&bar.s_free), lead);
-    rm.p_full = mapa(smem_addr(&bar.p_full), lead);
+    rm.p_full = mapa(smem_addr(&bar.p_full[0]), lead);
     rm.o_free = mapa(smem_addr(&bar.o_free), lead);
     rm.item_empty = mapa(smem_addr(&bar.item_empty[0]), lead);
     rm.item_full = mapa(smem_addr(&bar.item_full[0]), peer);
@@ -898,7 +911,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                      &map_v, block_table, prefix_lens, new_lens, cu_new_lens, status,
                      work_counter);
   } else if (warp >= 4) {
-    softmax2h(rank, bar, rm, tmem, xch, geo, out);
+    softmax2h(rank, bar, rm, tmem, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
+              out);
   }
   // a CTA that gave up tells its peer, so that the peer's roles leave their
   // loops instead of waiting for arrivals that will not come
