@@ -68,10 +68,10 @@ constexpr int kRing = 4;              // slots of 16 KB in each of the K and V r
 constexpr int kSlotBytes = 16384;
 constexpr int kQBytes = kRows * kD * 2;  // 32 KB: two 64-column blocks of 128 rows
 constexpr int kSortMax = 512;
-// tensor-memory columns: S (one buffer, the softmax empties it at once), O as
-// two accumulators (even / odd 16-key steps of every PV product, so that the
-// two halves of a product accumulate independently), P double-buffered
-constexpr uint32_t kColS = 0, kColOa = 128, kColOb = 256, kColP = 384;
+// tensor-memory columns: S (one buffer, the softmax empties it at once), O
+// double-buffered by item (the next item accumulates while the previous
+// one's epilogue reads its O), P double-buffered by step
+constexpr uint32_t kColS = 0, kColO = 128, kColP = 384;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 // consumers of the work-item ring: in each CTA the V producer and the
@@ -99,7 +99,7 @@ struct Bars2 {
   uint64_t s_free;            // even CTA: S read out by all softmax warps
   uint64_t p_full[2];         // even CTA: P buffer written by all softmax warps
   uint64_t pv_done[2];        // PV product from a P buffer done (commit, both CTAs)
-  uint64_t o_free;            // even CTA: O read by the epilogue
+  uint64_t o_free[2];         // even CTA: an O buffer read by the epilogue
   uint64_t item_full[2];      // work-item ring, written by the even CTA's K producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: both issuers' last commits
@@ -505,8 +505,9 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
 }
 
 // PV issuer: O += P(t) V(t) once the softmax has written P(t) and V(t) is
-// in; an item's first product (which overwrites O) also waits until the
-// previous item's epilogue has read O.
+// in, into the O buffer of the item's parity; an item's first product (which
+// overwrites O) also waits until the epilogue of the item two before has
+// read that buffer.
 __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
                            const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
@@ -526,15 +527,16 @@ __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32
       ok = mbar_wait(&bar.p_full[pb], (u >> 1) & 1, abortp);
       if (ok) ok = mbar_wait(&bar.v_full[slot], (u / kRing) & 1, abortp);
       const bool first = u == u_first;
-      if (ok && first && k > 0) ok = mbar_wait(&bar.o_free, (k - 1) & 1, abortp);
+      // the item's O buffer was last read by the epilogue of item k - 2
+      if (ok && first && k >= 2) ok = mbar_wait(&bar.o_free[k & 1], ((k >> 1) & 1) ^ 1, abortp);
       if (!ok) break;
       tc_fence_after();
       const uint64_t dv = sdesc_sw128(v_smem + slot * kSlotBytes, kSlotBytes, 1024);
       const uint32_t a = tmem + kColP + pb * 64;
 #pragma unroll
       for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys = two 8-row groups of 1 KB
-        mma2_ts(tmem + ((kk & 1) ? kColOb : kColOa), a + kk * 8, dv + kk * (2048 >> 4),
-                kIdescPV, (!first || kk > 1) ? 1u : 0u);
+        mma2_ts(tmem + kColO + (k & 1) * kD, a + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
+                (!first || kk > 0) ? 1u : 0u);
       mma2_commit_mc(&bar.pv_done[pb], 0x3);
     }
   }
@@ -619,6 +621,55 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     if (rel)
       for (; v_released <= v; ++v_released) mbar_arrive(&bar.v_empty[v_released % kRing]);
   };
+  // An item's epilogue (O / l -> bf16) is deferred until the first step of
+  // the next item has published its P: the item's last PV product is then
+  // done, and the tensor pipe has the next item's products to work on while
+  // the epilogue runs.  The next item accumulates into the other O buffer.
+  struct Pending {
+    bool on = false;
+    float l;
+    int64_t out_off;  // element offset of this thread's 64 outputs
+    bool row_valid;
+    uint32_t ob, ul;  // O buffer, last step
+  } pend;
+  auto epilogue = [&]() -> bool {
+    bool good = true;
+    // the partner's partial sum, 16 bits at a time
+    const uint32_t lb = __float_as_uint(pend.l);
+    const uint32_t lo_hi = exchange(static_cast<uint16_t>(lb >> 16), good);
+    if (!good) return false;
+    const uint32_t lo_lo = exchange(static_cast<uint16_t>(lb & 0xffffu), good);
+    if (!good) return false;
+    const float inv_l = 1.f / (pend.l + __uint_as_float((lo_hi << 16) | lo_lo));
+    if (!wait_warp(&bar.pv_done[pend.ul & 1], (pend.ul >> 1) & 1, abortp)) return false;
+    release_v_upto(pend.ul);
+    tc_fence_after();
+    uint4* orow = reinterpret_cast<uint4*>(out + pend.out_off);
+    const uint32_t tO = lane_addr + kColO + pend.ob * kD + hw * 64;
+#pragma unroll 1
+    for (int c = 0; c < 2; ++c) {
+      uint32_t o[32];
+      tmem_ld32(tO + c * 32, o);
+      tmem_wait_ld();
+      if (pend.row_valid) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 pk;
+          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+          orow[c * 4 + v] = pk;
+        }
+      }
+    }
+    // the O buffer may now be overwritten by the item two later
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive_remote(rm.o_free + 8 * pend.ob);
+    pend.on = false;
+    return true;
+  };
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
     Item2 w;
@@ -627,6 +678,7 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     __syncwarp();
     if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
+    const uint32_t ob = k & 1;  // this item's O buffer
     const int tok = w.tok0 + r / geo.G;
     const bool row_valid = tok < w.n;
     const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
@@ -683,9 +735,9 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
         const float m_new = fmaxf(m_run, mt);
         const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {  // this half's 64 columns of both accumulators
+        for (int c = 0; c < 2; ++c) {  // this half's 64 columns of the item's O
           uint32_t o[32];
-          const uint32_t tO = lane_addr + ((c & 2) ? kColOb : kColOa) + hw * 64 + (c & 1) * 32;
+          const uint32_t tO = lane_addr + kColO + ob * kD + hw * 64 + c * 32;
           tmem_ld32(tO, o);
           tmem_wait_ld();
 #pragma unroll
@@ -730,52 +782,18 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(rm.p_full + 8 * sb);
+      // the previous item's epilogue, now that this item's pipeline is going
+      if (j == 0 && pend.on && !(ok = epilogue())) break;
     }
     if (!ok) break;
-    // ---- epilogue: O / l -> bf16 (this half's 64 columns), once the item's last PV is done
-    // the partner's partial sum, 16 bits at a time
-    const uint32_t lb = __float_as_uint(l);
-    const uint32_t lo_hi = exchange(static_cast<uint16_t>(lb >> 16), ok);
-    if (!ok) break;
-    const uint32_t lo_lo = exchange(static_cast<uint16_t>(lb & 0xffffu), ok);
-    if (!ok) break;
-    const float l_row = l + __uint_as_float((lo_hi << 16) | lo_lo);
-    const uint32_t ul = u - 1;
-    ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
-    if (!ok) break;
-    release_v_upto(ul);
-    tc_fence_after();
-    const int h = w.g * geo.G + r % geo.G;
-    const float inv_l = 1.f / l_row;
-    uint4* orow = reinterpret_cast<uint4*>(
-        out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * kD + hw * 64);
-#pragma unroll 1
-    for (int c = 0; c < 2; ++c) {
-      // O = the two accumulators added
-      uint32_t o[32], o2[32];
-      tmem_ld32(lane_addr + kColOa + hw * 64 + c * 32, o);
-      tmem_ld32(lane_addr + kColOb + hw * 64 + c * 32, o2);
-      tmem_wait_ld();
-#pragma unroll
-      for (int e = 0; e < 32; ++e)
-        o[e] = __float_as_uint(__uint_as_float(o[e]) + __uint_as_float(o2[e]));
-      if (row_valid) {
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          uint4 pk;
-          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
-          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
-          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
-          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
-          orow[c * 4 + v] = pk;
-        }
-      }
-    }
-    // O may now be overwritten by the next item's first PV
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive_remote(rm.o_free);
+    pend.on = true;
+    pend.l = l;
+    pend.out_off = (static_cast<int64_t>(w.cu + tok) * geo.Hq + w.g * geo.G + r % geo.G) * kD + hw * 64;
+    pend.row_valid = row_valid;
+    pend.ob = ob;
+    pend.ul = u - 1;
   }
+  if (ok && pend.on) epilogue();
 }
 
 // ------------------------------------------------------------------- kernel
@@ -822,7 +840,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.v_full[s], 2);
       mbar_init(&bar.v_empty[s], 1);
     }
-    mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
+    for (int i = 0; i < 2; ++i) mbar_init(&bar.o_free[i], 2 * kSoftmaxWarps);
     mbar_init(&bar.drain, 2);
     for (int q = 0; q < 8; ++q) bar.xseq[q >> 2][q & 3] = 0;
     bar.abort_flag = 0;
@@ -883,7 +901,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     rm.v_full = mapa(smem_addr(&bar.v_full[0]), lead);
     rm.s_free = mapa(smem_addr(&bar.s_free), lead);
     rm.p_full = mapa(smem_addr(&bar.p_full[0]), lead);
-    rm.o_free = mapa(smem_addr(&bar.o_free), lead);
+    rm.o_free = mapa(smem_addr(&bar.o_free[0]), lead);
     rm.item_empty = mapa(smem_addr(&bar.item_empty[0]), lead);
     rm.item_full = mapa(smem_addr(&bar.item_full[0]), peer);
     rm.item_msg = mapa(smem_addr(&bar.item_msg[0][0]), peer);
