@@ -64,14 +64,18 @@ constexpr int kSoftmaxWarps = 8;
 constexpr int kThreads = 128 + 32 * kSoftmaxWarps;
 constexpr int kRows = 128;            // q rows per SM
 constexpr int kKeys = 128;            // keys per K/V step
-constexpr int kRing = 4;              // slots of 16 KB in each of the K and V rings
+constexpr int kRing = 3;              // slots of 16 KB in each of the K and V rings
 constexpr int kSlotBytes = 16384;
 constexpr int kQBytes = kRows * kD * 2;  // 32 KB: two 64-column blocks of 128 rows
+constexpr int kQBuf = 1;              // Q buffers (one: shared memory holds P instead)
+constexpr int kPBytes = kRows * kKeys * 2;  // 32 KB: P of one step, two 64-key column blocks
 constexpr int kSortMax = 512;
-// tensor-memory columns: S (one buffer, the softmax empties it at once), O
-// double-buffered by item (the next item accumulates while the previous
-// one's epilogue reads its O), P double-buffered by step
-constexpr uint32_t kColS = 0, kColO = 128, kColP = 384;
+// tensor-memory columns: S double-buffered by step [0, 256), O double-buffered
+// by item [256, 512) (the next item accumulates while the previous one's
+// epilogue reads its O).  P lives in shared memory: a PV product with P in
+// tensor memory occupies the pair's tensor pipe about 1.7 times as long as
+// one with both operands in shared memory.
+constexpr uint32_t kColS = 0, kColO = 256;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 // consumers of the work-item ring: in each CTA the V producer and the
@@ -95,8 +99,8 @@ struct Bars2 {
   uint64_t v_landed[kRing];   // the same for the V ring
   uint64_t v_full[kRing];
   uint64_t v_empty[kRing];    // the PV product reading the slot done (softmax thread 0)
-  uint64_t s_full;            // S computed (commit, both CTAs)
-  uint64_t s_free;            // even CTA: S read out by all softmax warps
+  uint64_t s_full[2];         // an S buffer computed (commit, both CTAs)
+  uint64_t s_free[2];         // even CTA: an S buffer read out by all softmax warps
   uint64_t p_full[2];         // even CTA: P buffer written by all softmax warps
   uint64_t pv_done[2];        // PV product from a P buffer done (commit, both CTAs)
   uint64_t o_free[2];         // even CTA: an O buffer read by the epilogue
@@ -248,8 +252,8 @@ struct Producer {
     while (true) {
       bool progress = false;
       if (kIsK && q_fwd < q_issued) {
-        const uint32_t qb = q_fwd & 1;
-        if (probe(&bar.q_landed[qb], (q_fwd >> 1) & 1)) {
+        const uint32_t qb = q_fwd % kQBuf;
+        if (probe(&bar.q_landed[qb], (q_fwd / kQBuf) & 1)) {
           if (lane == 0) mbar_arrive_remote(rm.q_full + 8 * qb);
           ++q_fwd;
           progress = true;
@@ -309,7 +313,7 @@ struct Producer {
     if (lane != 0) return;
     int no_abort = 0;
     for (uint32_t q = q_fwd; kIsK && q < q_issued; ++q)
-      mbar_wait(&bar.q_landed[q & 1], (q >> 1) & 1, &no_abort);
+      mbar_wait(&bar.q_landed[q % kQBuf], (q / kQBuf) & 1, &no_abort);
     for (uint32_t x = fwd; x < issued; ++x)
       mbar_wait(&landed[x % kRing], (x / kRing) & 1, &no_abort);
   }
@@ -381,8 +385,8 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
     if (it < 0) break;
     if (kIsK) {
       // this CTA's Q half: 128 rows = 128/G tokens x G heads, two column blocks
-      const int qb = k & 1;
-      ok = pr.wait(&bar.q_empty[qb], ((k >> 1) & 1) ^ 1);
+      const int qb = k % kQBuf;
+      ok = pr.wait(&bar.q_empty[qb], ((k / kQBuf) & 1) ^ 1);
       if (!ok) break;
       if (lane == 0) {
         mbar_arrive_expect_tx(&bar.q_landed[qb], kQBytes);
@@ -455,9 +459,9 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
 // tensor pipe busy.  Operand descriptors are built once per tile and
 // advanced by constant offsets.
 //
-// S issuer: S(t) once K(t) is in and the softmax has read S(t-1) out of the
-// buffer, which it does first thing in step t-1, so S(t) is computed while
-// the softmax works on step t-1.  Frees the Q buffer by a commit after the item's last
+// S issuer: S(t) once K(t) is in and the softmax has read S(t-2) out of the
+// buffer (which it does first thing in step t-2), so S runs up to two steps
+// ahead of the softmax.  Frees the Q buffer by a commit after the item's last
 // S product (the softmax frees the ring slots).
 __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Remote& rm,
                           uint32_t tmem, const Geom2& geo) {
@@ -471,21 +475,22 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
     if (!ok) break;
     mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
-    const int qb = k & 1;
-    ok = mbar_wait(&bar.q_full[qb], (k >> 1) & 1, abortp);
+    const int qb = k % kQBuf;
+    ok = mbar_wait(&bar.q_full[qb], (k / kQBuf) & 1, abortp);
     if (!ok) break;
     const uint64_t dq = sdesc_sw128(q_smem + qb * kQBytes, 16, 1024);
     const uint32_t u_last = u + w.nt - 1;
     for (; ok && u <= u_last; ++u) {
+      const uint32_t sb = u & 1;
       const uint32_t slot = u % kRing;
       ok = mbar_wait(&bar.k_full[slot], (u / kRing) & 1, abortp);
-      if (ok && u >= 1) ok = mbar_wait(&bar.s_free, (u - 1) & 1, abortp);
+      if (ok && u >= 2) ok = mbar_wait(&bar.s_free[sb], ((u - 2) >> 1) & 1, abortp);
       if (!ok) break;
       tc_fence_after();
       // K half: 8-key groups of 2 KB (the group's 8 rows of columns 0-63,
       // then of columns 64-127), so 8-row groups are 2048 bytes apart
       const uint64_t dk = sdesc_sw128(k_smem + slot * kSlotBytes, 16, 2048);
-      const uint32_t d = tmem + kColS;
+      const uint32_t d = tmem + kColS + sb * kKeys;
 #pragma unroll
       for (int kk = 0; kk < kD / 16; ++kk) {
         // 16-column steps: 32 bytes within a 128-byte row, then the next
@@ -494,7 +499,7 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
         mma2_ss(d, dq + ((kk >> 2) * kQBlk + (kk & 3) * 2), dk + ((kk >> 2) * kKBlk + (kk & 3) * 2),
                 kIdescQK, kk > 0);
       }
-      mma2_commit_mc(&bar.s_full, 0x3);
+      mma2_commit_mc(&bar.s_full[sb], 0x3);
       if (u == u_last) mma2_commit_mc(&bar.q_empty[qb], 0x3);
     }
   }
@@ -508,10 +513,10 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
 // in, into the O buffer of the item's parity; an item's first product (which
 // overwrites O) also waits until the epilogue of the item two before has
 // read that buffer.
-__device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
-                           const Geom2& geo) {
+__device__ void pv_issuer2(uint8_t* smem_p, uint8_t* smem_v, Bars2& bar, const Remote& rm,
+                           uint32_t tmem, const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
-  const uint32_t v_smem = smem_addr(smem_v);
+  const uint32_t v_smem = smem_addr(smem_v), p_smem = smem_addr(smem_p);
   uint32_t u = 0;  // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
@@ -532,11 +537,12 @@ __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32
       if (!ok) break;
       tc_fence_after();
       const uint64_t dv = sdesc_sw128(v_smem + slot * kSlotBytes, kSlotBytes, 1024);
-      const uint32_t a = tmem + kColP + pb * 64;
+      // P: K-major, 64-key column blocks of 128 rows x 128 bytes (16 KB apart)
+      const uint64_t dp = sdesc_sw128(p_smem + pb * kPBytes, 16, 1024);
 #pragma unroll
-      for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys = two 8-row groups of 1 KB
-        mma2_ts(tmem + kColO + (k & 1) * kD, a + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
-                (!first || kk > 0) ? 1u : 0u);
+      for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys: 32 bytes of P, two 8-row groups of V
+        mma2_ss(tmem + kColO + (k & 1) * kD, dp + ((kk >> 2) * (kRows * 128 >> 4) + (kk & 3) * 2),
+                dv + kk * (2048 >> 4), kIdescPV, (!first || kk > 0) ? 1u : 0u);
       mma2_commit_mc(&bar.pv_done[pb], 0x3);
     }
   }
@@ -568,7 +574,7 @@ __device__ __forceinline__ float bf16_bits_to_f32(uint16_t b) {
 
 
 __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t tmem,
-                          uint16_t* xch, const int* item_start, const Geom2& geo,
+                          uint8_t* smem_p, uint16_t* xch, const int* item_start, const Geom2& geo,
                           const int32_t* __restrict__ prefix_lens,
                           const int32_t* __restrict__ new_lens,
                           const int32_t* __restrict__ cu_new_lens,
@@ -686,9 +692,10 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     const float sl2 = geo.scale_log2;
     for (int j = 0; j < w.nt; ++j, ++u) {
       const uint32_t sb = u & 1;
-      const uint32_t tS = lane_addr + kColS + hw * 64;
-      const uint32_t tP = lane_addr + kColP + sb * 64 + hw * 32;
-      ok = wait_warp(&bar.s_full, u & 1, abortp);
+      const uint32_t tS = lane_addr + kColS + sb * kKeys + hw * 64;
+      // this thread's 128-byte row of P: row r of 64-key column block hw
+      uint8_t* prow = smem_p + sb * kPBytes + hw * (kRows * 128) + r * 128;
+      ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
       if (!ok) break;
       if (rel) mbar_arrive(&bar.k_empty[u % kRing]);
       tc_fence_after();
@@ -696,10 +703,10 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
       tmem_ld32(tS, sr[0]);
       tmem_ld32(tS + 32, sr[1]);
       tmem_wait_ld();
-      // the S buffer is free for S(u+1)
+      // S buffer sb is free for S(u+2)
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_remote(rm.s_free);
+      if (lane == 0) mbar_arrive_remote(rm.s_free + 8 * sb);
       const int key0 = j * kKeys + hw * 64;
       if (key0 + 63 > kmax) {
 #pragma unroll
@@ -770,16 +777,20 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
             acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
             pk[e] = pack_bf16x2(p0, p1);
           }
-          tmem_st16(tP + c * 16, pk);
+          // 16-byte chunks 4c..4c+3 of the row, 128-byte swizzled (chunk q
+          // of row r sits at chunk q ^ (r & 7))
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            *reinterpret_cast<uint4*>(prow + (((4 * c + q) ^ (r & 7)) << 4)) =
+                make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
         }
         float s0, s1, s2, s3;
         f2_unpack(f2_add(acc[0], acc[1]), s0, s1);
         f2_unpack(f2_add(acc[2], acc[3]), s2, s3);
         l += (s0 + s2) + (s1 + s3);
       }
-      // publish this half of P(u)
-      tmem_wait_st();
-      tc_fence_before();
+      // publish this half of P(u): the tensor core reads it through the async proxy
+      fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(rm.p_full + 8 * sb);
       // the previous item's epilogue, now that this item's pipeline is going
@@ -809,8 +820,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint8_t* smem_q = base;                     // 2 x 32 KB
-  uint8_t* smem_k = base + 2 * kQBytes;       // K ring, kRing x 16 KB
+  uint8_t* smem_p = base;                         // P, 2 x 32 KB
+  uint8_t* smem_q = smem_p + 2 * kPBytes;         // Q, kQBuf x 32 KB
+  uint8_t* smem_k = smem_q + kQBuf * kQBytes;     // K ring, kRing x 16 KB
   uint8_t* smem_v = smem_k + kRing * kSlotBytes;  // V ring
   Bars2& bar = *reinterpret_cast<Bars2*>(smem_v + kRing * kSlotBytes);
   int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
@@ -821,9 +833,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t rank = cluster_ctarank();
 
   if (threadIdx.x == 0) {
-    mbar_init(&bar.s_full, 1);
-    mbar_init(&bar.s_free, 2 * kSoftmaxWarps);
     for (int i = 0; i < 2; ++i) {
+      mbar_init(&bar.s_full[i], 1);
+      mbar_init(&bar.s_free[i], 2 * kSoftmaxWarps);
       mbar_init(&bar.q_landed[i], 1);
       mbar_init(&bar.q_full[i], 2);
       mbar_init(&bar.q_empty[i], 1);
@@ -899,7 +911,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     rm.q_full = mapa(smem_addr(&bar.q_full[0]), lead);
     rm.k_full = mapa(smem_addr(&bar.k_full[0]), lead);
     rm.v_full = mapa(smem_addr(&bar.v_full[0]), lead);
-    rm.s_free = mapa(smem_addr(&bar.s_free), lead);
+    rm.s_free = mapa(smem_addr(&bar.s_free[0]), lead);
     rm.p_full = mapa(smem_addr(&bar.p_full[0]), lead);
     rm.o_free = mapa(smem_addr(&bar.o_free[0]), lead);
     rm.item_empty = mapa(smem_addr(&bar.item_empty[0]), lead);
@@ -922,14 +934,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (rank == 0 && lane == 0) s_issuer2(smem_q, smem_k, bar, rm, tmem, geo);
     __syncwarp();
   } else if (warp == 2) {
-    if (rank == 0 && lane == 0) pv_issuer2(smem_v, bar, rm, tmem, geo);
+    if (rank == 0 && lane == 0) pv_issuer2(smem_p, smem_v, bar, rm, tmem, geo);
     __syncwarp();
   } else if (warp == 3) {
     producer2<false>(rank, smem_q, smem_v, bar, rm, item_start, total_items, geo, &map_q,
                      &map_v, block_table, prefix_lens, new_lens, cu_new_lens, status,
                      work_counter);
   } else if (warp >= 4) {
-    softmax2h(rank, bar, rm, tmem, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
+    softmax2h(rank, bar, rm, tmem, smem_p, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
               out);
   }
   // a CTA that gave up tells its peer, so that the peer's roles leave their
@@ -961,7 +973,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn2() {
 }
 
 size_t smem_bytes2(int batch) {
-  return 1024 + 2 * kQBytes + static_cast<size_t>(2 * kRing) * kSlotBytes + sizeof(Bars2) +
+  return 1024 + 2 * kPBytes + kQBuf * kQBytes + static_cast<size_t>(2 * kRing) * kSlotBytes +
+         sizeof(Bars2) +
          (static_cast<size_t>(batch) + 1) * sizeof(int) +
          (batch <= kSortMax ? kSortMax * sizeof(int16_t) : 0) + 2 * 2 * kRows * sizeof(uint16_t);
 }
