@@ -826,7 +826,10 @@ def bench_configs(args, pk):
         r_gbs = 2 * payload / (r_ms / 1e3) / 1e9 if nb else None
         res[w.name] = {
             "batch": w.B, "new_tokens": w.T_new, "prefix_tokens": int(w.prefix_lens.sum()),
-            "page_size": w.ps, "steps": steps, "ms_per_step": ms, "tok_per_s": w.T_new / (ms / 1e3),
+            "page_size": w.ps,
+            "attn_kernel": ("attn_tc2_kernel (CTA pairs)" if w.d == 128 and w.max_blocks * w.ps >= 65536
+                            else f"attn_tc_kernel<{w.d}>"),
+            "steps": steps, "ms_per_step": ms, "tok_per_s": w.T_new / (ms / 1e3),
             "attn_ms": at_ms, "attn_tflops": at_tf, "attn_frac_burst": at_tf / peak_t,
             "restore_ms": r_ms if nb else 0.0, "restore_gbs": r_gbs,
             "restore_frac_hbm": (r_gbs / peak_h) if nb else None, "append_ms": ap_ms,

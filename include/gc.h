@@ -337,6 +337,11 @@ GC_API gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v
  *   total_new_tokens  T_new = cu_new_lens[batch], passed from the host; it
  *               bounds every q / out row access.  A request whose rows would
  *               pass it is skipped and recorded as GC_ERR_OUT_OF_RANGE.
+ *   Kernels (head_dim 128): a call whose block table can describe contexts
+ *   of 65536 tokens or more (max_blocks_per_seq * page_size >= 65536) runs
+ *   on pairs of SMs (tcgen05 cta_group::2, each K/V tile split between the
+ *   two SMs); other calls run one work item per SM.  Both compute the same
+ *   operation to the same tolerance.
  *   Size limit: the kernel numbers its work items (a kv head of a request
  *   and 256 of its q rows) with 32-bit ints, so T_new * (Hq/Hkv) + 256 and
  *   Hkv * (T_new * (Hq/Hkv) / 256 + batch) + 2 * (SM count) must both stay

@@ -899,10 +899,24 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   return GC_OK;
 }
 
+// head_dim 128: contexts of up to kPairMinKeys tokens run on the single-SM
+// kernel above; calls whose block table can describe longer contexts run on
+// the CTA-pair kernel (attn_tc2.cu), which is faster when every work item
+// spans hundreds of K/V steps (measured on the 131072-token document layer)
+// and slower when items are short (its per-item start-up is longer).
+constexpr long long kPairMinKeys = 65536;
+
+gc_status launch_d128(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
+                      int* work_counter) {
+  if (static_cast<long long>(a.max_blocks) * pool->cfg.page_size >= kPairMinKeys)
+    return launch_attn_tc2(pool, a, stream, work_counter);
+  return launch<128>(pool, a, stream, work_counter);
+}
+
 }  // namespace
 
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
-  if (pool->cfg.head_dim == 128) return launch_attn_tc2(pool, a, stream, pool->work_counter);
+  if (pool->cfg.head_dim == 128) return launch_d128(pool, a, stream, pool->work_counter);
   return launch<64>(pool, a, stream, pool->work_counter);
 }
 
@@ -999,7 +1013,7 @@ gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a,
   int* counter = nullptr;
   st = noalloc_scratch(device, &counter);
   if (st != GC_OK) return st;
-  if (pool->cfg.head_dim == 128) return launch_attn_tc2(pool, a, stream, counter);
+  if (pool->cfg.head_dim == 128) return launch_d128(pool, a, stream, counter);
   return launch<64>(pool, a, stream, counter);
 }
 

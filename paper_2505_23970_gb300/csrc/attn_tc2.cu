@@ -64,18 +64,11 @@ constexpr int kSoftmaxWarps = 8;
 constexpr int kThreads = 128 + 32 * kSoftmaxWarps;
 constexpr int kRows = 128;            // q rows per SM
 constexpr int kKeys = 128;            // keys per K/V step
-constexpr int kRing = 3;              // slots of 16 KB in each of the K and V rings
+constexpr int kRing = 4;              // slots of 16 KB in each of the K and V rings
 constexpr int kSlotBytes = 16384;
 constexpr int kQBytes = kRows * kD * 2;  // 32 KB: two 64-column blocks of 128 rows
-constexpr int kQBuf = 1;              // Q buffers (one: shared memory holds P instead)
-constexpr int kPBytes = kRows * kKeys * 2;  // 32 KB: P of one step, two 64-key column blocks
 constexpr int kSortMax = 512;
-// tensor-memory columns: S double-buffered by step [0, 256), O double-buffered
-// by item [256, 512) (the next item accumulates while the previous one's
-// epilogue reads its O).  P lives in shared memory: a PV product with P in
-// tensor memory occupies the pair's tensor pipe about 1.7 times as long as
-// one with both operands in shared memory.
-constexpr uint32_t kColS = 0, kColO = 256;
+constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 // consumers of the work-item ring: in each CTA the V producer and the
@@ -99,11 +92,11 @@ struct Bars2 {
   uint64_t v_landed[kRing];   // the same for the V ring
   uint64_t v_full[kRing];
   uint64_t v_empty[kRing];    // the PV product reading the slot done (softmax thread 0)
-  uint64_t s_full[2];         // an S buffer computed (commit, both CTAs)
-  uint64_t s_free[2];         // even CTA: an S buffer read out by all softmax warps
+  uint64_t s_full[2];         // S buffer computed (commit, both CTAs)
+  uint64_t s_free[2];         // even CTA: S buffer read by all softmax warps
   uint64_t p_full[2];         // even CTA: P buffer written by all softmax warps
   uint64_t pv_done[2];        // PV product from a P buffer done (commit, both CTAs)
-  uint64_t o_free[2];         // even CTA: an O buffer read by the epilogue
+  uint64_t o_free;            // even CTA: O read by the epilogue
   uint64_t item_full[2];      // work-item ring, written by the even CTA's K producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: both issuers' last commits
@@ -252,8 +245,8 @@ struct Producer {
     while (true) {
       bool progress = false;
       if (kIsK && q_fwd < q_issued) {
-        const uint32_t qb = q_fwd % kQBuf;
-        if (probe(&bar.q_landed[qb], (q_fwd / kQBuf) & 1)) {
+        const uint32_t qb = q_fwd & 1;
+        if (probe(&bar.q_landed[qb], (q_fwd >> 1) & 1)) {
           if (lane == 0) mbar_arrive_remote(rm.q_full + 8 * qb);
           ++q_fwd;
           progress = true;
@@ -313,7 +306,7 @@ struct Producer {
     if (lane != 0) return;
     int no_abort = 0;
     for (uint32_t q = q_fwd; kIsK && q < q_issued; ++q)
-      mbar_wait(&bar.q_landed[q % kQBuf], (q / kQBuf) & 1, &no_abort);
+      mbar_wait(&bar.q_landed[q & 1], (q >> 1) & 1, &no_abort);
     for (uint32_t x = fwd; x < issued; ++x)
       mbar_wait(&landed[x % kRing], (x / kRing) & 1, &no_abort);
   }
@@ -385,8 +378,8 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
     if (it < 0) break;
     if (kIsK) {
       // this CTA's Q half: 128 rows = 128/G tokens x G heads, two column blocks
-      const int qb = k % kQBuf;
-      ok = pr.wait(&bar.q_empty[qb], ((k / kQBuf) & 1) ^ 1);
+      const int qb = k & 1;
+      ok = pr.wait(&bar.q_empty[qb], ((k >> 1) & 1) ^ 1);
       if (!ok) break;
       if (lane == 0) {
         mbar_arrive_expect_tx(&bar.q_landed[qb], kQBytes);
@@ -475,8 +468,8 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
     if (!ok) break;
     mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
-    const int qb = k % kQBuf;
-    ok = mbar_wait(&bar.q_full[qb], (k / kQBuf) & 1, abortp);
+    const int qb = k & 1;
+    ok = mbar_wait(&bar.q_full[qb], (k >> 1) & 1, abortp);
     if (!ok) break;
     const uint64_t dq = sdesc_sw128(q_smem + qb * kQBytes, 16, 1024);
     const uint32_t u_last = u + w.nt - 1;
@@ -490,7 +483,7 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
       // K half: 8-key groups of 2 KB (the group's 8 rows of columns 0-63,
       // then of columns 64-127), so 8-row groups are 2048 bytes apart
       const uint64_t dk = sdesc_sw128(k_smem + slot * kSlotBytes, 16, 2048);
-      const uint32_t d = tmem + kColS + sb * kKeys;
+      const uint32_t d = tmem + kColS + sb * 128;
 #pragma unroll
       for (int kk = 0; kk < kD / 16; ++kk) {
         // 16-column steps: 32 bytes within a 128-byte row, then the next
@@ -510,13 +503,12 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
 }
 
 // PV issuer: O += P(t) V(t) once the softmax has written P(t) and V(t) is
-// in, into the O buffer of the item's parity; an item's first product (which
-// overwrites O) also waits until the epilogue of the item two before has
-// read that buffer.
-__device__ void pv_issuer2(uint8_t* smem_p, uint8_t* smem_v, Bars2& bar, const Remote& rm,
-                           uint32_t tmem, const Geom2& geo) {
+// in; an item's first product (which overwrites O) also waits until the
+// previous item's epilogue has read O.
+__device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
+                           const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
-  const uint32_t v_smem = smem_addr(smem_v), p_smem = smem_addr(smem_p);
+  const uint32_t v_smem = smem_addr(smem_v);
   uint32_t u = 0;  // global step counter
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
@@ -532,17 +524,15 @@ __device__ void pv_issuer2(uint8_t* smem_p, uint8_t* smem_v, Bars2& bar, const R
       ok = mbar_wait(&bar.p_full[pb], (u >> 1) & 1, abortp);
       if (ok) ok = mbar_wait(&bar.v_full[slot], (u / kRing) & 1, abortp);
       const bool first = u == u_first;
-      // the item's O buffer was last read by the epilogue of item k - 2
-      if (ok && first && k >= 2) ok = mbar_wait(&bar.o_free[k & 1], ((k >> 1) & 1) ^ 1, abortp);
+      if (ok && first && k > 0) ok = mbar_wait(&bar.o_free, (k - 1) & 1, abortp);
       if (!ok) break;
       tc_fence_after();
       const uint64_t dv = sdesc_sw128(v_smem + slot * kSlotBytes, kSlotBytes, 1024);
-      // P: K-major, 64-key column blocks of 128 rows x 128 bytes (16 KB apart)
-      const uint64_t dp = sdesc_sw128(p_smem + pb * kPBytes, 16, 1024);
+      const uint32_t a = tmem + kColP + pb * 64;
 #pragma unroll
-      for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys: 32 bytes of P, two 8-row groups of V
-        mma2_ss(tmem + kColO + (k & 1) * kD, dp + ((kk >> 2) * (kRows * 128 >> 4) + (kk & 3) * 2),
-                dv + kk * (2048 >> 4), kIdescPV, (!first || kk > 0) ? 1u : 0u);
+      for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys = two 8-row groups of 1 KB
+        mma2_ts(tmem + kColO, a + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
+                (!first || kk > 0) ? 1u : 0u);
       mma2_commit_mc(&bar.pv_done[pb], 0x3);
     }
   }
@@ -574,7 +564,7 @@ __device__ __forceinline__ float bf16_bits_to_f32(uint16_t b) {
 
 
 __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t tmem,
-                          uint8_t* smem_p, uint16_t* xch, const int* item_start, const Geom2& geo,
+                          uint16_t* xch, const int* item_start, const Geom2& geo,
                           const int32_t* __restrict__ prefix_lens,
                           const int32_t* __restrict__ new_lens,
                           const int32_t* __restrict__ cu_new_lens,
@@ -627,55 +617,6 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     if (rel)
       for (; v_released <= v; ++v_released) mbar_arrive(&bar.v_empty[v_released % kRing]);
   };
-  // An item's epilogue (O / l -> bf16) is deferred until the first step of
-  // the next item has published its P: the item's last PV product is then
-  // done, and the tensor pipe has the next item's products to work on while
-  // the epilogue runs.  The next item accumulates into the other O buffer.
-  struct Pending {
-    bool on = false;
-    float l;
-    int64_t out_off;  // element offset of this thread's 64 outputs
-    bool row_valid;
-    uint32_t ob, ul;  // O buffer, last step
-  } pend;
-  auto epilogue = [&]() -> bool {
-    bool good = true;
-    // the partner's partial sum, 16 bits at a time
-    const uint32_t lb = __float_as_uint(pend.l);
-    const uint32_t lo_hi = exchange(static_cast<uint16_t>(lb >> 16), good);
-    if (!good) return false;
-    const uint32_t lo_lo = exchange(static_cast<uint16_t>(lb & 0xffffu), good);
-    if (!good) return false;
-    const float inv_l = 1.f / (pend.l + __uint_as_float((lo_hi << 16) | lo_lo));
-    if (!wait_warp(&bar.pv_done[pend.ul & 1], (pend.ul >> 1) & 1, abortp)) return false;
-    release_v_upto(pend.ul);
-    tc_fence_after();
-    uint4* orow = reinterpret_cast<uint4*>(out + pend.out_off);
-    const uint32_t tO = lane_addr + kColO + pend.ob * kD + hw * 64;
-#pragma unroll 1
-    for (int c = 0; c < 2; ++c) {
-      uint32_t o[32];
-      tmem_ld32(tO + c * 32, o);
-      tmem_wait_ld();
-      if (pend.row_valid) {
-#pragma unroll
-        for (int v = 0; v < 4; ++v) {
-          uint4 pk;
-          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
-          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
-          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
-          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
-          orow[c * 4 + v] = pk;
-        }
-      }
-    }
-    // the O buffer may now be overwritten by the item two later
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive_remote(rm.o_free + 8 * pend.ob);
-    pend.on = false;
-    return true;
-  };
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
     Item2 w;
@@ -684,7 +625,6 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     __syncwarp();
     if (lane == 0) mbar_arrive_cluster(rm.item_empty + 8 * (k & 1));
     if (it < 0) break;
-    const uint32_t ob = k & 1;  // this item's O buffer
     const int tok = w.tok0 + r / geo.G;
     const bool row_valid = tok < w.n;
     const int kmax = row_valid ? w.P + tok : w.T - 1;  // last visible key
@@ -692,9 +632,8 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     const float sl2 = geo.scale_log2;
     for (int j = 0; j < w.nt; ++j, ++u) {
       const uint32_t sb = u & 1;
-      const uint32_t tS = lane_addr + kColS + sb * kKeys + hw * 64;
-      // this thread's 128-byte row of P: row r of 64-key column block hw
-      uint8_t* prow = smem_p + sb * kPBytes + hw * (kRows * 128) + r * 128;
+      const uint32_t tS = lane_addr + kColS + sb * 128 + hw * 64;
+      const uint32_t tP = lane_addr + kColP + sb * 64 + hw * 32;
       ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
       if (!ok) break;
       if (rel) mbar_arrive(&bar.k_empty[u % kRing]);
@@ -703,7 +642,7 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
       tmem_ld32(tS, sr[0]);
       tmem_ld32(tS + 32, sr[1]);
       tmem_wait_ld();
-      // S buffer sb is free for S(u+2)
+      // S buffer free for S(u+2)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(rm.s_free + 8 * sb);
@@ -742,9 +681,9 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
         const float m_new = fmaxf(m_run, mt);
         const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
 #pragma unroll 1
-        for (int c = 0; c < 2; ++c) {  // this half's 64 columns of the item's O
+        for (int c = 0; c < 2; ++c) {
           uint32_t o[32];
-          const uint32_t tO = lane_addr + kColO + ob * kD + hw * 64 + c * 32;
+          const uint32_t tO = lane_addr + kColO + hw * 64 + c * 32;
           tmem_ld32(tO, o);
           tmem_wait_ld();
 #pragma unroll
@@ -777,34 +716,59 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
             acc[e & 3] = f2_add(acc[e & 3], f2_pack(p0, p1));
             pk[e] = pack_bf16x2(p0, p1);
           }
-          // 16-byte chunks 4c..4c+3 of the row, 128-byte swizzled (chunk q
-          // of row r sits at chunk q ^ (r & 7))
-#pragma unroll
-          for (int q = 0; q < 4; ++q)
-            *reinterpret_cast<uint4*>(prow + (((4 * c + q) ^ (r & 7)) << 4)) =
-                make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+          tmem_st16(tP + c * 16, pk);
         }
         float s0, s1, s2, s3;
         f2_unpack(f2_add(acc[0], acc[1]), s0, s1);
         f2_unpack(f2_add(acc[2], acc[3]), s2, s3);
         l += (s0 + s2) + (s1 + s3);
       }
-      // publish this half of P(u): the tensor core reads it through the async proxy
-      fence_proxy_async_smem();
+      // publish this half of P(u)
+      tmem_wait_st();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(rm.p_full + 8 * sb);
-      // the previous item's epilogue, now that this item's pipeline is going
-      if (j == 0 && pend.on && !(ok = epilogue())) break;
     }
     if (!ok) break;
-    pend.on = true;
-    pend.l = l;
-    pend.out_off = (static_cast<int64_t>(w.cu + tok) * geo.Hq + w.g * geo.G + r % geo.G) * kD + hw * 64;
-    pend.row_valid = row_valid;
-    pend.ob = ob;
-    pend.ul = u - 1;
+    // ---- epilogue: O / l -> bf16 (this half's 64 columns), once the item's last PV is done
+    // the partner's partial sum, 16 bits at a time
+    const uint32_t lb = __float_as_uint(l);
+    const uint32_t lo_hi = exchange(static_cast<uint16_t>(lb >> 16), ok);
+    if (!ok) break;
+    const uint32_t lo_lo = exchange(static_cast<uint16_t>(lb & 0xffffu), ok);
+    if (!ok) break;
+    const float l_row = l + __uint_as_float((lo_hi << 16) | lo_lo);
+    const uint32_t ul = u - 1;
+    ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
+    if (!ok) break;
+    release_v_upto(ul);
+    tc_fence_after();
+    const int h = w.g * geo.G + r % geo.G;
+    const float inv_l = 1.f / l_row;
+    uint4* orow = reinterpret_cast<uint4*>(
+        out + (static_cast<int64_t>(w.cu + tok) * geo.Hq + h) * kD + hw * 64);
+#pragma unroll 1
+    for (int c = 0; c < 2; ++c) {
+      uint32_t o[32];
+      tmem_ld32(lane_addr + kColO + hw * 64 + c * 32, o);
+      tmem_wait_ld();
+      if (row_valid) {
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          uint4 pk;
+          pk.x = pack_bf16x2(__uint_as_float(o[8 * v + 0]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+          pk.y = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+          pk.z = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+          pk.w = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+          orow[c * 4 + v] = pk;
+        }
+      }
+    }
+    // O may now be overwritten by the next item's first PV
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive_remote(rm.o_free);
   }
-  if (ok && pend.on) epilogue();
 }
 
 // ------------------------------------------------------------------- kernel
@@ -820,9 +784,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint8_t* smem_p = base;                         // P, 2 x 32 KB
-  uint8_t* smem_q = smem_p + 2 * kPBytes;         // Q, kQBuf x 32 KB
-  uint8_t* smem_k = smem_q + kQBuf * kQBytes;     // K ring, kRing x 16 KB
+  uint8_t* smem_q = base;                     // 2 x 32 KB
+  uint8_t* smem_k = base + 2 * kQBytes;       // K ring, kRing x 16 KB
   uint8_t* smem_v = smem_k + kRing * kSlotBytes;  // V ring
   Bars2& bar = *reinterpret_cast<Bars2*>(smem_v + kRing * kSlotBytes);
   int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
@@ -834,11 +797,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&bar.s_full[i], 1);
-      mbar_init(&bar.s_free[i], 2 * kSoftmaxWarps);
       mbar_init(&bar.q_landed[i], 1);
       mbar_init(&bar.q_full[i], 2);
       mbar_init(&bar.q_empty[i], 1);
+      mbar_init(&bar.s_full[i], 1);
+      mbar_init(&bar.s_free[i], 2 * kSoftmaxWarps);
       mbar_init(&bar.p_full[i], 2 * kSoftmaxWarps);
       mbar_init(&bar.pv_done[i], 1);
       mbar_init(&bar.item_full[i], 1);
@@ -852,7 +815,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.v_full[s], 2);
       mbar_init(&bar.v_empty[s], 1);
     }
-    for (int i = 0; i < 2; ++i) mbar_init(&bar.o_free[i], 2 * kSoftmaxWarps);
+    mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
     mbar_init(&bar.drain, 2);
     for (int q = 0; q < 8; ++q) bar.xseq[q >> 2][q & 3] = 0;
     bar.abort_flag = 0;
@@ -913,7 +876,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     rm.v_full = mapa(smem_addr(&bar.v_full[0]), lead);
     rm.s_free = mapa(smem_addr(&bar.s_free[0]), lead);
     rm.p_full = mapa(smem_addr(&bar.p_full[0]), lead);
-    rm.o_free = mapa(smem_addr(&bar.o_free[0]), lead);
+    rm.o_free = mapa(smem_addr(&bar.o_free), lead);
     rm.item_empty = mapa(smem_addr(&bar.item_empty[0]), lead);
     rm.item_full = mapa(smem_addr(&bar.item_full[0]), peer);
     rm.item_msg = mapa(smem_addr(&bar.item_msg[0][0]), peer);
@@ -934,14 +897,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (rank == 0 && lane == 0) s_issuer2(smem_q, smem_k, bar, rm, tmem, geo);
     __syncwarp();
   } else if (warp == 2) {
-    if (rank == 0 && lane == 0) pv_issuer2(smem_p, smem_v, bar, rm, tmem, geo);
+    if (rank == 0 && lane == 0) pv_issuer2(smem_v, bar, rm, tmem, geo);
     __syncwarp();
   } else if (warp == 3) {
     producer2<false>(rank, smem_q, smem_v, bar, rm, item_start, total_items, geo, &map_q,
                      &map_v, block_table, prefix_lens, new_lens, cu_new_lens, status,
                      work_counter);
   } else if (warp >= 4) {
-    softmax2h(rank, bar, rm, tmem, smem_p, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
+    softmax2h(rank, bar, rm, tmem, xch, item_start, geo, prefix_lens, new_lens, cu_new_lens,
               out);
   }
   // a CTA that gave up tells its peer, so that the peer's roles leave their
@@ -973,8 +936,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn2() {
 }
 
 size_t smem_bytes2(int batch) {
-  return 1024 + 2 * kPBytes + kQBuf * kQBytes + static_cast<size_t>(2 * kRing) * kSlotBytes +
-         sizeof(Bars2) +
+  return 1024 + 2 * kQBytes + static_cast<size_t>(2 * kRing) * kSlotBytes + sizeof(Bars2) +
          (static_cast<size_t>(batch) + 1) * sizeof(int) +
          (batch <= kSortMax ? kSortMax * sizeof(int16_t) : 0) + 2 * 2 * kRows * sizeof(uint16_t);
 }

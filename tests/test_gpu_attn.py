@@ -348,3 +348,99 @@ def test_work_item_bound_refused_before_launch():
     assert "work items" in gcb.gc_last_error()
     assert pool.check() == gcb.GC_OK
     pool.close()
+
+
+# ------------------------------------------------------- the CTA-pair kernel
+# head_dim 128 prefill runs on the CTA-pair kernel when the block table can
+# describe contexts of 65536 tokens or more (the long-document configs do);
+# widening a block table with unused (-1) columns routes any workload there.
+PAIR_KEYS = 65536
+
+
+def on_pair_kernel(w):
+    cols = -(-PAIR_KEYS // w.ps)
+    if w.max_blocks < cols:
+        w.block_table = np.pad(w.block_table, ((0, 0), (0, cols - w.max_blocks)),
+                               constant_values=-1).astype(np.int32)
+    return w
+
+
+@pytest.mark.parametrize("make", [
+    lambda: wl.llama3_8b_layer(seed=0),
+    lambda: wl.custom("pair-g1", 4, 2, 2, 128, 16, [0, 77, 300, 129], [200, 1, 45, 130], seed=31),
+    lambda: wl.custom("pair-g8p64", 4, 16, 2, 128, 64, [0, 77, 300, 129], [200, 1, 45, 130], seed=32),
+    lambda: wl.custom("pair-g16p128", 4, 32, 2, 128, 128, [0, 77, 300, 129], [200, 1, 45, 130],
+                      seed=33),
+    lambda: wl.custom("pair-g4p32", 4, 8, 2, 128, 32, [0, 77, 300, 129], [200, 1, 45, 130], seed=34),
+    lambda: wl.custom("pair-ragged", 7, 16, 2, 128, 16, [0, 5, 17, 128, 255, 0, 1000],
+                      [3, 0, 1, 129, 17, 1, 0], seed=35),
+], ids=["8b", "g1p16", "g8p64", "g16p128", "g4p32", "ragged"])
+def test_pair_kernel_parity(make):
+    full_parity(on_pair_kernel(make()))
+
+
+def test_pair_kernel_70b_sampled():
+    sampled_parity(on_pair_kernel(wl.llama3_70b_layer(seed=2)), n_random=384)
+
+
+def test_pair_kernel_single_key_row_returns_v_bit_exact():
+    import torch
+    w = on_pair_kernel(wl.custom("pair-single", 3, 8, 2, 128, 16, [0, 0, 0], [1, 5, 130], seed=36))
+    db = DeviceBatch(w)
+    db.run()
+    assert db.check() == gcb.GC_OK
+    cu = w.cu_new_lens
+    _, v = w.kv_new()
+    for b in range(w.B):
+        row = db.out[cu[b]].view(torch.int16).cpu().numpy().view(np.uint16)
+        for h in range(w.Hq):
+            assert np.array_equal(row[h], v[cu[b], h // w.G])
+    db.close()
+
+
+def test_pair_kernel_large_score_jumps():
+    w = on_pair_kernel(wl.custom("pair-jumps", 1, 8, 1, 128, 16, [512], [64], seed=12))
+    src = wl.bf16_bits_to_f32(w.host_src())
+    keys = src[:, 0, 0, 0].reshape(-1, 128)
+    keys[192:256] *= 256.0
+    keys[256:320] *= 1024.0
+    src[:, 0, 0, 0] = keys.reshape(-1, 16, 128)
+    w._cache["src"] = wl.f32_to_bf16_bits(src)
+    full_parity(w)
+
+
+def test_pair_kernel_deterministic_and_page_permutation_invariant():
+    import torch
+    w = on_pair_kernel(wl.custom("pair-perm", 3, 16, 2, 128, 16, [100, 0, 260], [90, 33, 64],
+                                 seed=37))
+    a = DeviceBatch(w)
+    a.run()
+    first = a.out.clone()
+    a.out.fill_(0)
+    a.attn()
+    assert torch.equal(a.out.view(torch.int16), first.view(torch.int16))
+    w2 = on_pair_kernel(wl.custom("pair-perm", 3, 16, 2, 128, 16, [100, 0, 260], [90, 33, 64],
+                                  seed=37))
+    perm = np.random.default_rng(1).permutation(w2.num_pages).astype(np.int32)
+    w2.block_table = np.where(w2.block_table >= 0, perm[np.maximum(w2.block_table, 0)],
+                              -1).astype(np.int32)
+    w2._cache = dict(w._cache)
+    b = DeviceBatch(w2)
+    b.run()
+    assert a.check() == gcb.GC_OK and b.check() == gcb.GC_OK
+    assert torch.equal(first.view(torch.int16), b.out.view(torch.int16))
+    a.close()
+    b.close()
+
+
+def test_pair_kernel_bad_block_table_entry_is_reported_not_faulted():
+    w = on_pair_kernel(wl.custom("pair-badbt", 2, 8, 1, 128, 16, [40, 8], [30, 9], seed=38))
+    db = DeviceBatch(w)
+    db.run()
+    assert db.check() == gcb.GC_OK
+    bt = w.block_table.copy()
+    bt[1, 0] = -5
+    db.block_table = _i32(bt, "cuda")
+    db.attn()
+    assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
+    db.close()
