@@ -472,9 +472,11 @@ def run_ours(args):
             raise RuntimeError("device status after the end-to-end loop")
 
     # ---- restore of the full 80-layer KV of one 8192-token prefix
-    restore80 = ttft80 = decode = configs = None
+    restore80 = ttft80 = decode = configs = attn_q8 = None
     if not args.no_decode and rank == 0:
         decode = bench_decode(args, pk)
+    if not args.no_q8_attn and rank == 0:
+        attn_q8 = bench_attn_q8(args, pk)
     if not args.no_configs and rank == 0:
         configs = bench_configs(args, pk)
     if not args.no_restore80 and rank == 0:
@@ -509,7 +511,7 @@ def run_ours(args):
         "breakdown_ms": {"restore": restore_ms, "append": append_ms, "attention": attn_ms},
         "attn_tflops": attn_tflops, "restore_gbs": restore_gbs,
         "e2e": e2e, "restore_80layer": restore80, "prefill_80layer": ttft80, "decode": decode,
-        "configs": configs,
+        "configs": configs, "attn_q8": attn_q8,
         "clocks": clocks,
         "gpu_launches": 3 * args.steps,
     }
@@ -887,6 +889,92 @@ def bench_decode(args, pk):
     return res
 
 
+def bench_attn_q8(args, pk):
+    """Prefill attention over cached pages kept in the 8-bit tier
+    (gc_prefix_prefill_attn_q8) on the 70B-shaped layer and the conversation
+    mix: every full cached page is read from an INT8 image in device memory
+    (made with gc_kv_save_q8) and dequantised in the kernel; partly filled
+    last pages, which the new tokens are appended into, stay in the pool.
+    Next to it: the pool-only kernel, and the two-step path it replaces
+    (gc_kv_restore_q8 of the same pages into the pool, then attention).
+    Algorithmic HBM bytes of the cached K/V per step, counting one read
+    pass: two-step = image I + pool write B + pool read B; one-step = I, so
+    the one-step path moves 2B fewer bytes."""
+    import torch
+
+    from paper_2505_23970_gb300 import binding as gcb
+    from paper_2505_23970_gb300 import workloads as wl
+    from paper_2505_23970_gb300.harness import DeviceBatch, _i32
+
+    res = {}
+    stream = torch.cuda.current_stream()
+    for w in (wl.llama3_70b_layer(seed=args.seed), wl.conversation_mix(seed=args.seed)):
+        db = DeviceBatch(w)
+        db.restore()
+        db.append()
+        table = np.full((w.B, w.max_blocks), -1, dtype=np.int32)
+        ids = []
+        for b in range(w.B):
+            full = int(w.prefix_lens[b]) // w.ps
+            table[b, :full] = np.arange(len(ids), len(ids) + full)
+            ids.extend(w.block_table[b, :full].tolist())
+        n = len(ids)
+        ids_d = _i32(np.asarray(ids, dtype=np.int32), db.q.device)
+        table_d = _i32(table, db.q.device)
+        chunk8 = gcb.gc_kv_q8_chunk_bytes(db.pool.cfg)
+        img = torch.empty(max(n, 1) * w.L * 2 * chunk8, dtype=torch.uint8, device=db.q.device)
+        gcb.gc_kv_save_q8(db.pool.handle, img, ids_d, n, 0, w.L, stream, None,
+                          gcb.GC_SAVE_DST_DEVICE)
+        out_q8 = torch.empty_like(db.out)
+
+        def attn_q8():
+            gcb.gc_prefix_prefill_attn_q8(db.q, db.pool.handle, db.block_table, db.prefix_lens,
+                                          db.new_lens, out_q8, stream, 0, db.cu_new_lens, w.B,
+                                          w.max_blocks, w.Hq, w.scale, w.T_new, img, table_d,
+                                          n, 0)
+
+        def two_step():
+            gcb.gc_kv_restore_q8(db.pool.handle, img, ids_d, n, 0, w.L, stream, None,
+                                 gcb.GC_RESTORE_SRC_DEVICE)
+            db.attn(stream)
+
+        def timed(fn, reps=10):
+            for _ in range(3):
+                fn()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(reps):
+                fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            return a.elapsed_time(b) / reps
+
+        ms_pool = timed(lambda: db.attn(stream))
+        ms_q8 = timed(attn_q8)
+        ms_two = timed(two_step)
+        same = bool(torch.equal(out_q8.view(torch.int16), db.out.view(torch.int16)))
+        ok = db.check(stream) == gcb.GC_OK
+        flops = w.attn_flops()
+        B_bytes = n * w.L * 2 * w.Hkv * w.ps * w.d * 2
+        I_bytes = n * w.L * 2 * chunk8
+        tf = flops / (ms_q8 / 1e3) / 1e12
+        res[w.name] = {
+            "image_pages": n, "image_bytes": I_bytes, "cached_kv_bf16_bytes": B_bytes,
+            "hbm_bytes_saved_per_step": 2 * B_bytes,
+            "ms": {"attn_q8": ms_q8, "attn_pool": ms_pool, "restore_q8_then_attn": ms_two},
+            "attn_q8_tflops": tf, "attn_q8_frac_of_measured_peak": tf / pk["bf16_tflops"],
+            "attn_pool_tflops": flops / (ms_pool / 1e3) / 1e12,
+            "speedup_vs_two_step": ms_two / ms_q8,
+            "bit_identical_to_two_step": same, "device_status_ok": ok,
+            "l2": "not flushed between launches (image and pool pages exceed L2 on the 70B "
+                  "layer; the mix's 64 requests fit partly)"}
+        del img, out_q8
+        db.close()
+        torch.cuda.empty_cache()
+    return res
+
+
 def bench_ttft80(args, image=None):
     """All 80 layers of one request with an 8192-token cached prefix and
     1024 new tokens: restore of each layer's cached pages (pinned host ->
@@ -1010,6 +1098,8 @@ def main():
     ap.add_argument("--no-restore80", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-q8-attn", action="store_true",
+                    help="skip attention over 8-bit pages")
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the per-configuration measurements of every workload")
     ap.add_argument("--config-steps", type=int, default=10,
@@ -1018,7 +1108,7 @@ def main():
     ap.add_argument("--ref-step-seconds", type=float, default=None,
                     help="oracle seconds per step of --impl reference (default: sized so "
                          "the whole run takes about 2.5 minutes)")
-    ap.add_argument("--only", choices=["decode", "restore80", "prefill80", "configs"],
+    ap.add_argument("--only", choices=["decode", "restore80", "prefill80", "configs", "q8attn"],
                     default=None,
                     help="run one secondary measurement alone and print it (for profilers)")
     ap.add_argument("--profile", action="store_true",
@@ -1036,6 +1126,8 @@ def main():
         pk = peaks()
         if args.only == "decode":
             print(json.dumps({"decode": bench_decode(args, pk)}), flush=True)
+        elif args.only == "q8attn":
+            print(json.dumps({"attn_q8": bench_attn_q8(args, pk)}), flush=True)
         elif args.only == "configs":
             print(json.dumps({"configs": bench_configs(args, pk)}), flush=True)
         elif args.only == "restore80":

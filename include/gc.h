@@ -388,6 +388,43 @@ GC_API gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool*
                                                 int32_t max_blocks_per_seq, int32_t num_q_heads,
                                                 float softmax_scale, int32_t total_new_tokens);
 
+/* Prefill over a context whose cached pages stay in the 8-bit cache tier
+ * (Sec. 6.1: the 70B runs keep the KV in INT8; Sec. 3.2: an 8-bit tier
+ * halves what storage holds and what a restore moves).  The result is
+ * exactly that of gc_kv_restore_q8 of the 8-bit pages into the pool
+ * followed by gc_prefix_prefill_attn, but the pages are never written to
+ * the pool: the kernel dequantises each one (x' = bf16_rne(c * s), the
+ * restore's rounding) into the tile it would have loaded.
+ * Arguments as gc_prefix_prefill_attn, plus:
+ *   q8_image   device memory, 16-byte aligned: the 8-bit image
+ *              [n_image_blocks][L][2][gc_kv_q8_chunk_bytes], or with
+ *              GC_RESTORE_LAYER_MAJOR in flags [L][n_image_blocks][2][...],
+ *              as gc_kv_save_q8 writes it (e.g. staged by
+ *              gc_kv_stage_layers with GC_STAGE_Q8).  Only the chunks of
+ *              `layer` are read.
+ *   q8_table   int32 [batch][max_blocks_per_seq], device: for page j of
+ *              request b, an image block in [0, n_image_blocks) to read it
+ *              from, or -1 to read pool page block_table[b][j] as
+ *              gc_prefix_prefill_attn does (new tokens' pages, or pages
+ *              already resident).  An entry >= n_image_blocks is skipped
+ *              (its keys read as zeros) and recorded as GC_ERR_OUT_OF_RANGE.
+ *   n_image_blocks  blocks in the image (>= 0).
+ *   flags      0 or GC_RESTORE_LAYER_MAJOR.
+ * Both head sizes run on the one-SM kernel (one warp of each SM converts
+ * the 8-bit pages while the TMA unit loads the pool pages).
+ * Errors: as gc_prefix_prefill_attn; GC_ERR_INVALID_ARG also for unknown
+ * flags, a NULL q8_table (or q8_image with n_image_blocks > 0), a
+ * misaligned q8_image. */
+GC_API gc_status gc_prefix_prefill_attn_q8(const void* q, const gc_kv_pool* pool,
+                                           const int32_t* block_table, const int32_t* prefix_lens,
+                                           const int32_t* new_lens, void* out,
+                                           cudaStream_t stream, int32_t layer,
+                                           const int32_t* cu_new_lens, int32_t batch,
+                                           int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                           float softmax_scale, int32_t total_new_tokens,
+                                           const void* q8_image, const int32_t* q8_table,
+                                           int32_t n_image_blocks, uint32_t flags);
+
 /* Same operation and arguments as gc_prefix_prefill_attn, computed by a
  * plain CUDA-core kernel (one warp per row, fp32 throughout, no tensor
  * cores).  Slow; kept as an independent GPU cross-check of the indexing. */

@@ -41,6 +41,7 @@ EXPORTED = (
     "gc_kv_restore_q8",
     "gc_kv_append", "gc_prefix_prefill_attn",
     "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc",
+    "gc_prefix_prefill_attn_q8",
     "gc_paged_decode_workspace_bytes", "gc_paged_decode_attn", "gc_selftest_wait_timeout",
     "gc_last_error",
     "gc_status_string",
@@ -95,6 +96,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_prefix_prefill_attn.argtypes = attn
         lib.gc_prefix_prefill_attn_simt.argtypes = attn
         lib.gc_prefix_prefill_attn_noalloc.argtypes = attn
+        lib.gc_prefix_prefill_attn_q8.argtypes = attn + [vp, vp, i32, u32]
         lib.gc_selftest_wait_timeout.argtypes = [vp, vp]
         lib.gc_selftest_wait_timeout.restype = ctypes.c_int
         lib.gc_paged_decode_workspace_bytes.argtypes = [vp, i32, i32, i32]
@@ -106,7 +108,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                   "gc_kv_save_layers", "gc_kv_stage_layers", "gc_kv_save_q8", "gc_kv_restore_q8",
                   "gc_kv_append",
                   "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt",
-                  "gc_prefix_prefill_attn_noalloc", "gc_paged_decode_attn"):
+                  "gc_prefix_prefill_attn_noalloc", "gc_prefix_prefill_attn_q8",
+                  "gc_paged_decode_attn"):
             getattr(lib, f).restype = ctypes.c_int
         lib.gc_last_error.argtypes = []
         lib.gc_last_error.restype = ctypes.c_char_p
@@ -277,6 +280,21 @@ def gc_prefix_prefill_attn_noalloc(q, pool, block_table, prefix_lens, new_lens, 
                                                  batch, max_blocks_per_seq, num_q_heads,
                                                  softmax_scale, total_new_tokens),
            "gc_prefix_prefill_attn_noalloc")
+
+
+def gc_prefix_prefill_attn_q8(q, pool, block_table, prefix_lens, new_lens, out, stream,
+                              layer: int, cu_new_lens, batch: int, max_blocks_per_seq: int,
+                              num_q_heads: int, softmax_scale: float, total_new_tokens: int,
+                              q8_image, q8_table, n_image_blocks: int, flags: int = 0) -> None:
+    """gc_prefix_prefill_attn with the pages that q8_table maps (>= 0) read
+    from the 8-bit image q8_image instead of the pool."""
+    _check(load().gc_prefix_prefill_attn_q8(_addr(q), pool, _addr(block_table),
+                                            _addr(prefix_lens), _addr(new_lens), _addr(out),
+                                            _stream(stream), layer, _addr(cu_new_lens), batch,
+                                            max_blocks_per_seq, num_q_heads, softmax_scale,
+                                            total_new_tokens, _addr(q8_image), _addr(q8_table),
+                                            n_image_blocks, flags),
+           "gc_prefix_prefill_attn_q8")
 
 
 @dataclass

@@ -97,6 +97,12 @@ struct Geom {
   int32_t decode, split_tiles, max_splits;
   const int32_t* seq_lens;
   float* ws;
+  // pages read from an 8-bit image (the cache tier's layout): q8_table[b][j]
+  // >= 0 names the image block holding page j of request b
+  const uint8_t* q8_image;
+  const int32_t* q8_table;
+  int32_t q8_n_blocks, q8_layer_major, L;
+  uint32_t q8_hdr, q8_chunk;  // scale header and whole chunk (one block, layer, plane), bytes
 };
 
 struct Barriers {
@@ -209,7 +215,7 @@ __device__ __forceinline__ int read_item(Barriers& bar, uint32_t k, volatile int
 }
 
 // ------------------------------------------------------------------ roles
-template <int D>
+template <int D, bool kQ8>
 __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const int* item_start,
                          int total_items, const Geom& geo, const CUtensorMap* map_q,
                          const CUtensorMap* map_kv, const int32_t* __restrict__ block_table,
@@ -262,9 +268,12 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
       const int nkeys = min(kTileN, w.T - key0);
       const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
       const int blk0 = key0 >> geo.ps_shift;
-      int pg_id = -2;  // -2: no page in this lane
-      if (j < w.nt && lane < npages)
+      int pg_id = -2;  // -2: no page in this lane; -3: a page of the 8-bit image
+      if (j < w.nt && lane < npages) {
         pg_id = blk0 + lane < geo.max_blocks ? __ldg(block_table + bt_row + blk0 + lane) : -1;
+        if (kQ8 && blk0 + lane < geo.max_blocks && __ldg(geo.q8_table + bt_row + blk0 + lane) >= 0)
+          pg_id = -3;  // the converter warp fills it
+      }
       return pg_id;
     };
     int page_next = lookup(w.j0);
@@ -273,11 +282,11 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
       const int nkeys = min(kTileN, w.T - key0);
       int page = page_next;
       page_next = lookup(j + 1);
-      if (page != -2 && (page < 0 || page >= geo.num_pages)) {
+      if (page != -2 && page != -3 && (page < 0 || page >= geo.num_pages)) {
         record_error(status, GC_ERR_OUT_OF_RANGE);
         page = -1;
       }
-      if (page == -2) page = -1;
+      if (page == -2 || page == -3) page = -1;
       const int good = __popc(__ballot_sync(0xffffffffu, page >= 0));
       const int my_page = __shfl_sync(0xffffffffu, page, pg < 32 ? pg : 0);
       const bool issues = pg < kTileN / 16 && my_page >= 0;
@@ -330,6 +339,109 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
     if (armed_vfix >= 0) mbar_wait(&bar.vfix, armed_vfix, &no_abort);
     for (int s = 0; s < C::kStages; ++s)
       if (armed & (1u << s)) mbar_wait(&bar.kv_full[s], (armed_par >> s) & 1u, &no_abort);
+  }
+}
+
+// Converter (warp 3, attention over 8-bit pages only).  It follows the same
+// work items and ring slots as the producer and fills the pages the producer
+// leaves out (those the q8 table maps to the 8-bit image): each 16 codes of
+// a page are one 16-byte load, dequantised exactly as the 8-bit restore does
+// (c * s in binary32, rounded to bf16) and stored at the positions the TMA
+// box would have written (rows of 128 bytes, 16-byte chunks swizzled by row
+// within 8-row groups).  The slot's full barrier then counts the producer's
+// copies and this warp's arrival.
+template <int D>
+__device__ void converter(uint8_t* smem_kv, Barriers& bar, const int* item_start,
+                          const Geom& geo, const int32_t* __restrict__ prefix_lens,
+                          const int32_t* __restrict__ new_lens,
+                          const int32_t* __restrict__ cu_new_lens, int32_t* status) {
+  using C = Cfg<D>;
+  const int lane = threadIdx.x & 31;
+  volatile int* abortp = &bar.abort_flag;
+  uint32_t kv_count = 0;
+  bool ok = true;
+  constexpr int kUnitsPerRow = D / 16;  // 16-code units in a row of the page
+  for (uint32_t k = 0; ok; ++k) {
+    const int it = read_item(bar, k, abortp, ok);
+    ok = __all_sync(0xffffffffu, ok);
+    if (!ok) break;
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&bar.item_empty[k & 1]);
+    if (it < 0) break;
+    Item w;
+    decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
+    const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
+    for (int j = w.j0; ok && j < w.nt; ++j) {
+      const int key0 = j * kTileN;
+      const int nkeys = min(kTileN, w.T - key0);
+      const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
+      const int blk0 = key0 >> geo.ps_shift;
+      int ib = -1;  // image block of page `lane` of the tile
+      if (lane < npages && blk0 + lane < geo.max_blocks) {
+        ib = __ldg(geo.q8_table + bt_row + blk0 + lane);
+        if (ib >= geo.q8_n_blocks) {
+          record_error(status, GC_ERR_OUT_OF_RANGE);
+          ib = -1;
+        }
+      }
+      const uint32_t mine = __ballot_sync(0xffffffffu, ib >= 0);
+#pragma unroll 1
+      for (int kv = 0; kv < 2; ++kv) {
+        const int slot = kv_count % C::kStages;
+        ok = mbar_wait(&bar.kv_empty[slot], ((kv_count / C::kStages) & 1) ^ 1, abortp);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        uint8_t* dst = smem_kv + slot * C::kTileBytes;
+        // V rows past the sequence end are zeroed by the producer; leave them
+        const int rows_end = kv ? nkeys : kTileN;
+        for (uint32_t m = mine; m; m &= m - 1) {
+          const int p = __ffs(m) - 1;
+          const int blk = __shfl_sync(0xffffffffu, ib, p);
+          const uint64_t il = geo.q8_layer_major
+                                  ? static_cast<uint64_t>(geo.layer) * geo.q8_n_blocks + blk
+                                  : static_cast<uint64_t>(blk) * geo.L + geo.layer;
+          const uint8_t* chunk = geo.q8_image + (il * 2 + kv) * geo.q8_chunk;
+          const float sc = __ldg(reinterpret_cast<const float*>(chunk) + w.g);
+          const uint4* codes = reinterpret_cast<const uint4*>(
+              chunk + geo.q8_hdr + static_cast<uint64_t>(w.g) * geo.ps * D);
+          const int units = geo.ps * kUnitsPerRow;
+          for (int u0 = 0; u0 < units; u0 += 128) {
+            uint4 v[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int u = u0 + q * 32 + lane;
+              v[q] = u < units ? __ldg(codes + u) : make_uint4(0, 0, 0, 0);
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int u = u0 + q * 32 + lane;
+              if (u >= units) continue;
+              const int r = p * geo.ps + u / kUnitsPerRow;  // row of the tile
+              if (r >= rows_end) continue;
+              const int c0 = (u % kUnitsPerRow) * 16;       // first column
+              uint8_t* row = dst + (c0 >> 6) * C::kHalfBytes + r * 128;
+              const int q0 = (c0 & 63) >> 3;                 // first 16-byte chunk
+              uint4 lo, hi;
+              lo.x = q8_dequant2(v[q].x, 0, sc);
+              lo.y = q8_dequant2(v[q].x, 1, sc);
+              lo.z = q8_dequant2(v[q].y, 0, sc);
+              lo.w = q8_dequant2(v[q].y, 1, sc);
+              hi.x = q8_dequant2(v[q].z, 0, sc);
+              hi.y = q8_dequant2(v[q].z, 1, sc);
+              hi.z = q8_dequant2(v[q].w, 0, sc);
+              hi.w = q8_dequant2(v[q].w, 1, sc);
+              *reinterpret_cast<uint4*>(row + ((q0 ^ (r & 7)) << 4)) = lo;
+              *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ (r & 7)) << 4)) = hi;
+            }
+          }
+        }
+        // the tensor core reads the slot through the async proxy
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar.kv_full[slot]);
+        ++kv_count;
+      }
+    }
   }
 }
 
@@ -640,7 +752,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
   }
 }
 
-template <int D>
+template <int D, bool kQ8>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                    const __grid_constant__ CUtensorMap map_kv,
@@ -665,7 +777,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bar.vfix, 1);
     mbar_init(&bar.drain, 2);
     for (int s = 0; s < C::kStages; ++s) {
-      mbar_init(&bar.kv_full[s], 1);
+      mbar_init(&bar.kv_full[s], kQ8 ? 2 : 1);  // + the converter's arrival
       mbar_init(&bar.kv_empty[s], 2);
     }
     for (int i = 0; i < 2; ++i) {
@@ -675,7 +787,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&bar.item_full[s], 1);
-      mbar_init(&bar.item_empty[s], kItemConsumers);
+      mbar_init(&bar.item_empty[s], kItemConsumers + (kQ8 ? 1 : 0));
     }
     bar.abort_flag = 0;
     bar.p0_steps = 0;
@@ -748,13 +860,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp < 4) {
     regs_dec<kRegsProducer>();
     if (warp == 0) {
-      producer<D>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv,
+      producer<D, kQ8>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv,
                   block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
     } else if (warp == 1 || warp == 2) {
       if (lane == 0)
         mma_issuer<D>(warp - 1, smem_q, smem_kv, bar, tmem, item_start, total_items, geo,
                       prefix_lens, new_lens, cu_new_lens);
       __syncwarp();
+    } else if (kQ8) {
+      converter<D>(smem_kv, bar, item_start, geo, prefix_lens, new_lens, cu_new_lens, status);
     }
   } else {
     regs_inc<kRegsSoftmax>();
@@ -824,7 +938,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 template <int D>
 gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
-                 int* work_counter, const DecodeMode* dm = nullptr) {
+                 int* work_counter, const DecodeMode* dm = nullptr,
+                 const Q8Pages* q8 = nullptr) {
   using C = Cfg<D>;
   gc_status bound = check_item_bound(pool, a, dm, pool->num_sms);
   if (bound != GC_OK) return bound;
@@ -850,6 +965,15 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   geo.max_splits = dm ? dm->max_splits : 0;
   geo.seq_lens = dm ? dm->seq_lens : nullptr;
   geo.ws = dm ? dm->ws : nullptr;
+  geo.L = cfg.num_layers;
+  geo.q8_image = q8 ? q8->image : nullptr;
+  geo.q8_table = q8 ? q8->table : nullptr;
+  geo.q8_n_blocks = q8 ? q8->n_blocks : 0;
+  geo.q8_layer_major = q8 && q8->layer_major ? 1 : 0;
+  // image chunk of one (block, layer, plane): Hkv fp32 scales padded to 16
+  // bytes, then Hkv groups of ps*d codes
+  geo.q8_hdr = static_cast<uint32_t>(q8_header_bytes(cfg));
+  geo.q8_chunk = static_cast<uint32_t>(q8_chunk_bytes(cfg));
 
   const uint64_t pool_rows = static_cast<uint64_t>(cfg.num_layers) * 2 * cfg.num_pages *
                              cfg.num_kv_heads * cfg.page_size;
@@ -884,14 +1008,14 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   const size_t smem = 1024 + 2 * C::kTileBytes + C::kStages * C::kTileBytes + sizeof(Barriers) +
                       (static_cast<size_t>(a.batch) + 1) * sizeof(int) +
                       kSortMax * sizeof(int16_t);
-  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+  auto kernel = q8 ? attn_tc_kernel<D, true> : attn_tc_kernel<D, false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: smem attribute");
   // the work items are claimed from a counter in the pool's control block
   e = cudaMemsetAsync(work_counter, 0, sizeof(int), stream);
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: clearing the work counter");
-  attn_tc_kernel<D><<<pool->num_sms, kThreads, smem, stream>>>(
+  kernel<<<pool->num_sms, kThreads, smem, stream>>>(
       map_q, map_kv, a.block_table, a.prefix_lens, a.new_lens, a.cu_new_lens,
       static_cast<__nv_bfloat16*>(a.out), geo, pool->status, work_counter);
   e = cudaGetLastError();
@@ -918,6 +1042,15 @@ gc_status launch_d128(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t st
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream) {
   if (pool->cfg.head_dim == 128) return launch_d128(pool, a, stream, pool->work_counter);
   return launch<64>(pool, a, stream, pool->work_counter);
+}
+
+// Pages read from the 8-bit image run on the single-SM kernel at either head
+// size: its converter warp dequantises them into the same shared-memory
+// tiles the tensor map fills for pool pages.
+gc_status launch_attn_tc_q8(const gc_kv_pool* pool, const AttnArgs& a, const Q8Pages& q8,
+                            cudaStream_t stream) {
+  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter, nullptr, &q8);
+  return launch<64>(pool, a, stream, pool->work_counter, nullptr, &q8);
 }
 
 gc_status launch_attn_tc_decode(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode& dm,

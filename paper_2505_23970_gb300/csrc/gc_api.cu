@@ -583,6 +583,36 @@ gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool* pool,
   return gc::launch_attn_tc_noalloc(pool, a, stream);
 }
 
+gc_status gc_prefix_prefill_attn_q8(const void* q, const gc_kv_pool* pool,
+                                    const int32_t* block_table, const int32_t* prefix_lens,
+                                    const int32_t* new_lens, void* out, cudaStream_t stream,
+                                    int32_t layer, const int32_t* cu_new_lens, int32_t batch,
+                                    int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                    float softmax_scale, int32_t total_new_tokens,
+                                    const void* q8_image, const int32_t* q8_table,
+                                    int32_t n_image_blocks, uint32_t flags) {
+  Range range_("gc_prefix_prefill_attn_q8");
+  g_msg[0] = 0;
+  gc::AttnArgs a;
+  bool noop;
+  gc_status s = attn_common("gc_prefix_prefill_attn_q8", q, pool, block_table, prefix_lens,
+                            new_lens, out, layer, cu_new_lens, batch, max_blocks_per_seq,
+                            num_q_heads, softmax_scale, total_new_tokens, &a, &noop);
+  if (s != GC_OK) return s;
+  if (flags & ~GC_RESTORE_LAYER_MAJOR)
+    return fail(GC_ERR_INVALID_ARG, "gc_prefix_prefill_attn_q8: unknown flags 0x%x", flags);
+  if (n_image_blocks < 0)
+    return fail(GC_ERR_INVALID_ARG, "gc_prefix_prefill_attn_q8: negative n_image_blocks");
+  if (noop) return GC_OK;
+  if (!q8_table || (n_image_blocks > 0 && !q8_image))
+    return fail(GC_ERR_INVALID_ARG, "gc_prefix_prefill_attn_q8: NULL q8_image / q8_table");
+  if (reinterpret_cast<uintptr_t>(q8_image) % 16)
+    return fail(GC_ERR_INVALID_ARG, "gc_prefix_prefill_attn_q8: q8_image not 16-byte aligned");
+  const gc::Q8Pages q8{static_cast<const uint8_t*>(q8_image), q8_table, n_image_blocks,
+                       (flags & GC_RESTORE_LAYER_MAJOR) != 0};
+  return gc::launch_attn_tc_q8(pool, a, q8, stream);
+}
+
 gc_status gc_prefix_prefill_attn_simt(const void* q, const gc_kv_pool* pool,
                                       const int32_t* block_table, const int32_t* prefix_lens,
                                       const int32_t* new_lens, void* out, cudaStream_t stream,

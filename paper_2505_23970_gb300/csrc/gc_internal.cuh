@@ -38,6 +38,17 @@ __device__ __forceinline__ void record_error(int32_t* status, int32_t code) {
   atomicCAS(status, 0, code);
 }
 
+// One 8-bit code pair -> a bf16 pair: codes k*2 and k*2+1 (bytes) of the
+// 32-bit word, each c * s in binary32 rounded to bf16 (nearest even).  The
+// 8-bit restore and the attention over 8-bit pages both dequantise with it,
+// so they produce the same bf16 values.
+__device__ __forceinline__ uint32_t q8_dequant2(uint32_t codes, int k, float s) {
+  const float a = static_cast<float>(static_cast<int8_t>((codes >> (16 * k)) & 0xffu)) * s;
+  const float b = static_cast<float>(static_cast<int8_t>((codes >> (16 * k + 8)) & 0xffu)) * s;
+  const __nv_bfloat162 p = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&p);
+}
+
 // ---------------------------------------------------------------- launchers
 // Each returns GC_OK or a status with the message already set.
 // Page copies between a staging image [n_blocks][L][2][chunk] (or, with
@@ -81,6 +92,17 @@ struct AttnArgs {
 gc_status launch_attn_simt(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
 gc_status launch_attn_tc_noalloc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream);
+// Prefill attention with some pages read from a device 8-bit image (the
+// cache tier's layout) instead of the pool: q8_table [batch][max_blocks]
+// gives, per page of a request, an image block (>= 0) or -1 (pool page).
+struct Q8Pages {
+  const uint8_t* image;
+  const int32_t* table;
+  int32_t n_blocks;   // blocks in the image
+  bool layer_major;   // image [L][n][2][chunk] instead of [n][L][2][chunk]
+};
+gc_status launch_attn_tc_q8(const gc_kv_pool* pool, const AttnArgs& a, const Q8Pages& q8,
+                            cudaStream_t stream);
 // head_dim 128 prefill on CTA pairs (attn_tc2.cu), work items claimed from
 // `work_counter` (zeroed by the launch).
 gc_status launch_attn_tc2(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,

@@ -198,10 +198,7 @@ __global__ void __launch_bounds__(256) save_q8_kernel(uint8_t* __restrict__ imag
 }
 
 __device__ __forceinline__ uint32_t dequant2(uint32_t codes, int k, float s) {
-  const float a = static_cast<float>(static_cast<int8_t>((codes >> (16 * k)) & 0xffu)) * s;
-  const float b = static_cast<float>(static_cast<int8_t>((codes >> (16 * k + 8)) & 0xffu)) * s;
-  const __nv_bfloat162 p = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<const uint32_t*>(&p);
+  return q8_dequant2(codes, k, s);
 }
 
 // Each thread dequantises 16 codes (one 16-byte load) into 16 bf16 values

@@ -1,0 +1,251 @@
+"""Prefill over pages kept in the 8-bit cache tier (gc_prefix_prefill_attn_q8).
+
+The operation is defined as the 8-bit restore (Sec. 6.1 keeps the 70B KV in
+INT8) followed by prefix-reuse attention (Sec. 2.2), so the oracle is
+oracle.kv_restore_q8 of every cached page, oracle.kv_append and
+oracle.prefix_attn.  The GPU path never writes the 8-bit pages into the
+pool; it is checked bit for bit against the library's own two-step path
+(gc_kv_restore_q8 of every page, then gc_prefix_prefill_attn on the same
+one-SM kernel) and within the attention tolerance against the oracle."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2505_23970_gb300 import binding as gcb
+from paper_2505_23970_gb300 import workloads as wl
+from paper_2505_23970_gb300.harness import DeviceBatch, _i32
+
+from ._util import assert_attn_close, gather_rows, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2505_23970_gb300 import build
+    build.build()
+
+
+class Q8Case:
+    """The 8-bit image of a workload's cached pages (made by the oracle's
+    quantiser), the q8 table mapping each request's FULL prefix pages to it,
+    and the partly cached last pages: those also receive the new tokens
+    (gc_kv_append writes into them), so they are dequantised into the pool
+    first, as a serving loop does before appending to a page."""
+
+    def __init__(self, w, frac_in_image=1.0, seed=0):
+        self.w = w
+        self.ids = w.prefix_blocks()
+        src_pool = w.empty_pool()
+        if self.ids.size:
+            oracle.kv_restore(src_pool, w.host_src(), self.ids)
+        self.img = oracle.kv_save_q8(src_pool, self.ids)       # [n][L][2][chunk]
+        self.table = np.full((w.B, w.max_blocks), -1, dtype=np.int32)
+        rng = np.random.default_rng(seed)
+        to_pool, off = [], 0
+        for b in range(w.B):
+            P = int(w.prefix_lens[b])
+            nb, full = -(-P // w.ps), P // w.ps
+            for j in range(nb):
+                if j < full and rng.random() < frac_in_image:
+                    self.table[b, j] = off + j
+                else:
+                    to_pool.append(off + j)   # image index of a page restored to the pool
+            off += nb
+        self.to_pool = np.asarray(to_pool, dtype=np.int64)
+
+    def oracle_pool(self):
+        w = self.w
+        pool = w.empty_pool()
+        if self.ids.size:
+            oracle.kv_restore_q8(pool, self.img, self.ids)
+        k, v = w.kv_new()
+        for l in range(w.L):
+            oracle.kv_append(pool, l, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
+        return pool
+
+
+def _dev_image(img, layer_major):
+    import torch
+    if layer_major:
+        img = np.ascontiguousarray(img.swapaxes(0, 1))
+    return torch.from_numpy(img).cuda()
+
+
+def run_q8(case, layer=0, layer_major=False, table=None):
+    """Restore the pool-side pages, append, attention over the q8 table."""
+    import torch
+    w = case.w
+    db = DeviceBatch(w, with_restore=False)
+    if case.to_pool.size:
+        part = torch.from_numpy(np.ascontiguousarray(case.img[case.to_pool])).cuda()
+        gcb.gc_kv_restore_q8(db.pool.handle, part, _i32(case.ids[case.to_pool], "cuda"),
+                             int(case.to_pool.size), 0, w.L, None, None,
+                             gcb.GC_RESTORE_SRC_DEVICE)
+    for l in range(w.L):
+        db.append(layer=l)
+    dimg = _dev_image(case.img, layer_major)
+    flags = gcb.GC_RESTORE_LAYER_MAJOR if layer_major else 0
+    gcb.gc_prefix_prefill_attn_q8(db.q, db.pool.handle, db.block_table, db.prefix_lens,
+                                  db.new_lens, db.out, None, layer, db.cu_new_lens, w.B,
+                                  w.max_blocks, w.Hq, w.scale, w.T_new, dimg,
+                                  _i32(case.table if table is None else table, "cuda"),
+                                  int(case.ids.size), flags)
+    status = db.check()
+    out = db.out.clone()
+    pool = db.pool_bits()
+    db.close()
+    return status, out, pool
+
+
+def run_restore_then_attn(case, layer=0):
+    """The two-step path: every cached page dequantised into the pool."""
+    import torch
+    w = case.w
+    db = DeviceBatch(w, with_restore=False)
+    if case.ids.size:
+        gcb.gc_kv_restore_q8(db.pool.handle, torch.from_numpy(case.img).cuda(),
+                             _i32(case.ids, "cuda"), int(case.ids.size), 0, w.L, None, None,
+                             gcb.GC_RESTORE_SRC_DEVICE)
+    for l in range(w.L):
+        db.append(layer=l)
+    db.attn(layer=layer)
+    assert db.check() == gcb.GC_OK
+    out = db.out.clone()
+    db.close()
+    return out
+
+
+def _bits_equal(a, b):
+    import torch
+    return torch.equal(a.view(torch.int16), b.view(torch.int16))
+
+
+def full_q8_parity(w, **kw):
+    case = Q8Case(w, **kw)
+    status, out, _ = run_q8(case)
+    assert status == gcb.GC_OK
+    assert _bits_equal(out, run_restore_then_attn(case)), f"{w.name}: differs from restore + attn"
+    import torch
+    ref = oracle.prefix_attn(w.q(), case.oracle_pool(), 0, w.block_table, w.prefix_lens,
+                             w.cu_new_lens, w.scale)
+    return assert_attn_close(out.to(torch.float64).cpu().numpy(), ref, f"{w.name} [q8]")
+
+
+def sampled_q8_parity(w, n_random=512, bit_exact=True):
+    import torch
+    case = Q8Case(w)
+    status, out, _ = run_q8(case)
+    assert status == gcb.GC_OK
+    if bit_exact:
+        assert _bits_equal(out, run_restore_then_attn(case)), f"{w.name}: differs"
+    rows = sample_rows(w, n_random)
+    ref = oracle.prefix_attn_rows(w.q(), case.oracle_pool(), 0, w.block_table, w.prefix_lens,
+                                  w.cu_new_lens, w.scale, rows)
+    got = gather_rows(out.to(torch.float64).cpu().numpy(), w, rows)
+    return assert_attn_close(got, ref, f"{w.name} sampled [q8]")
+
+
+# ---------------------------------------------------------------- shapes
+@pytest.mark.parametrize("G,d,ps", [(8, 128, 16), (4, 64, 16), (1, 128, 32), (16, 64, 64),
+                                    (2, 128, 128)])
+def test_q8_shapes_ragged(G, d, ps):
+    """Head groupings, both head sizes and every page size, with prefixes
+    that end inside a page, a request without prefix and one without new
+    tokens: bit-exact against restore + attention, within tolerance of the
+    oracle."""
+    Hkv = 2
+    w = wl.custom(f"q8-G{G}-d{d}-ps{ps}", 5, G * Hkv, Hkv, d, ps, [300, 0, 1000, 17, 640],
+                  [70, 45, 0, 260, 129], seed=G * 7 + d + ps)
+    full_q8_parity(w)
+
+
+def test_q8_tiny():
+    full_q8_parity(wl.tiny())
+
+
+def test_q8_mixed_pool_and_image_pages():
+    """Half of the full prefix pages read from the image, the other half
+    already in the pool: the kernel takes each page from where the table
+    says, with the same result as the all-pool path."""
+    w = wl.custom("q8-mixed", 3, 16, 2, 128, 16, [2000, 700, 129], [200, 64, 300], seed=31)
+    full_q8_parity(w, frac_in_image=0.5, seed=3)
+
+
+def test_q8_llama3_70b_layer_sampled():
+    """The 70B-shaped layer (8 x (8192 cached + 1024 new), 64/8 heads)."""
+    sampled_q8_parity(wl.llama3_70b_layer())
+
+
+def test_q8_conversation_mix_sampled():
+    """The multi-turn mix (64 requests, lognormal lengths, every prefix hit)."""
+    sampled_q8_parity(wl.conversation_mix(hit_p=1.0))
+
+
+def test_q8_long_document_sampled():
+    """131072 cached tokens in 64-token pages.  The all-pool path runs this
+    block table on SM pairs, so only the oracle comparison applies."""
+    sampled_q8_parity(wl.long_document(B=1), n_random=128, bit_exact=False)
+
+
+@pytest.mark.parametrize("layer_major", [False, True])
+def test_q8_layer_of_a_multilayer_image(layer_major):
+    """An image of three layers, attention of layer 1, in both image
+    layouts: only layer 1's chunks are read."""
+    w = wl.custom("q8-layers", 2, 16, 2, 128, 16, [520, 47], [40, 129], seed=15)
+    w.L = 3
+    case = Q8Case(w)
+    status, out, _ = run_q8(case, layer=1, layer_major=layer_major)
+    assert status == gcb.GC_OK
+    assert _bits_equal(out, run_restore_then_attn(case, layer=1))
+    import torch
+    ref = oracle.prefix_attn(w.q(), case.oracle_pool(), 1, w.block_table, w.prefix_lens,
+                             w.cu_new_lens, w.scale)
+    assert_attn_close(out.to(torch.float64).cpu().numpy(), ref, "layer 1 [q8]")
+
+
+def test_q8_pool_pages_of_image_pages_are_not_read():
+    """Pool pages behind image-mapped table entries keep their NaN fill
+    (nothing restores them) and the pool is not written by the call."""
+    w = wl.custom("q8-untouched", 2, 16, 2, 128, 16, [640, 300], [64, 20], seed=9)
+    case = Q8Case(w)
+    status, out, pool = run_q8(case)
+    assert status == gcb.GC_OK
+    import torch
+    assert torch.isfinite(out.float()).all()
+    for b in range(w.B):
+        for j in range(w.max_blocks):
+            if case.table[b, j] >= 0:
+                page = w.block_table[b, j]
+                assert np.all(pool[0, :, page] == 0x7FC0)
+
+
+def test_q8_bad_table_entry_is_reported_not_faulted():
+    """An image block >= n_image_blocks is skipped and recorded as
+    GC_ERR_OUT_OF_RANGE in the status word."""
+    w = wl.custom("q8-bad", 2, 16, 2, 128, 16, [640, 300], [64, 20], seed=10)
+    case = Q8Case(w)
+    bad = case.table.copy()
+    bad[1, 2] = case.ids.size + 5
+    status, _, _ = run_q8(case, table=bad)
+    assert status == gcb.GC_ERR_OUT_OF_RANGE
+
+
+def test_q8_host_checks():
+    """Unknown flags, a NULL table and a misaligned image fail before any
+    launch with GC_ERR_INVALID_ARG."""
+    import torch
+    w = wl.custom("q8-args", 1, 16, 2, 128, 16, [64], [16], seed=11)
+    case = Q8Case(w)
+    db = DeviceBatch(w, with_restore=False)
+    dimg = _dev_image(case.img, False)
+    tab = _i32(case.table, "cuda")
+    args = (db.q, db.pool.handle, db.block_table, db.prefix_lens, db.new_lens, db.out, None, 0,
+            db.cu_new_lens, w.B, w.max_blocks, w.Hq, w.scale, w.T_new)
+    for image, table, flags in ((dimg, tab, 0x10), (dimg, None, 0),
+                                (dimg.data_ptr() + 4, tab, 0)):
+        with pytest.raises(gcb.GcError) as e:
+            gcb.gc_prefix_prefill_attn_q8(*args, image, table, int(case.ids.size), flags)
+        assert e.value.status == gcb.GC_ERR_INVALID_ARG
+    torch.cuda.synchronize()
+    db.close()
