@@ -457,3 +457,40 @@ def test_q8_image_layout_and_layer_range():
     ref = np.zeros_like(pool)
     oracle.kv_restore_q8(ref, full, ids)
     assert np.array_equal(out[2], ref[2]) and np.all(out[[0, 1, 3]] == 0)
+
+
+def test_q8_attention_on_exact_codes_equals_bf16_attention():
+    """Attention over 8-bit pages is defined as the 8-bit restore followed by
+    prefix attention.  Pages whose values are integers in [-127, 127] times
+    2^-e, with +-127 in every (page, plane, head) group, have scale 2^-e and
+    codes equal to those integers exactly, so the 8-bit path must give the
+    bf16 path's result bit for bit (stale NaN slots past a prefix included)."""
+    w = wl.custom("q8-exact", 3, 8, 2, 16, 4, [13, 8, 0], [5, 6, 3], seed=23)
+    src = w.host_src()
+    rng = np.random.default_rng(29)
+    n = src.shape[0]
+    codes = rng.integers(-127, 128, size=src.shape)
+    codes[..., 0, 0] = np.where(rng.random(codes.shape[:-2]) < 0.5, 127, -127)
+    e = rng.integers(2, 9, size=src.shape[:-2])[..., None, None]
+    exact = codes.astype(np.float32) * np.float32(2.0) ** -e.astype(np.float32)
+    stale = np.isnan(wl.bf16_bits_to_f32(src))
+    w._cache["src"] = np.where(stale, src, wl.f32_to_bf16_bits(exact))
+    ids = w.prefix_blocks()
+    bf = _fill_pool(w)
+    out_bf = oracle.prefix_attn(w.q(), bf, 0, w.block_table, w.prefix_lens, w.cu_new_lens,
+                                w.scale)
+    cached = w.empty_pool()
+    oracle.kv_restore(cached, w.host_src(), ids)                # before the append
+    img = oracle.kv_save_q8(cached, ids)
+    scales, got = oracle.q8_split(img, w.Hkv, w.ps, w.d)       # [n][L][2][Hkv](...)
+    want = np.where(stale, 0, codes)
+    assert np.array_equal(got.astype(np.int64), want)
+    assert np.array_equal(scales.astype(np.float64), 2.0 ** -e[..., 0, 0].astype(np.float64))
+    q8 = w.empty_pool()
+    oracle.kv_restore_q8(q8, img, ids)
+    k, v = w.kv_new()
+    oracle.kv_append(q8, 0, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
+    out_q8 = oracle.prefix_attn(w.q(), q8, 0, w.block_table, w.prefix_lens, w.cu_new_lens,
+                                w.scale)
+    assert n == ids.size and np.all(np.isfinite(out_q8))
+    assert np.array_equal(out_q8, out_bf)
