@@ -407,11 +407,15 @@ GC_API gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool*
  *              from, or -1 to read pool page block_table[b][j] as
  *              gc_prefix_prefill_attn does (new tokens' pages, or pages
  *              already resident).  An entry >= n_image_blocks is skipped
- *              (its keys read as zeros) and recorded as GC_ERR_OUT_OF_RANGE.
+ *              (the output of that request is then unspecified) and
+ *              recorded as GC_ERR_OUT_OF_RANGE.
  *   n_image_blocks  blocks in the image (>= 0).
  *   flags      0 or GC_RESTORE_LAYER_MAJOR.
- * Both head sizes run on the one-SM kernel (one warp of each SM converts
- * the 8-bit pages while the TMA unit loads the pool pages).
+ * Both head sizes run on a 16-warp variant of the one-SM kernel: the
+ * producer bulk-copies each image page's codes into the K/V ring and a
+ * fourth warpgroup dequantises them there, while the TMA unit loads the
+ * pool pages.  Shared memory limits batch to 8192 as for
+ * gc_prefix_prefill_attn.
  * Errors: as gc_prefix_prefill_attn; GC_ERR_INVALID_ARG also for unknown
  * flags, a NULL q8_table (or q8_image with n_image_blocks > 0), a
  * misaligned q8_image. */

@@ -45,6 +45,10 @@
 //  * Decode mode (one new token per request): items are (request, kv head,
 //    range of K/V tiles); a request cut into several ranges writes fp32
 //    partials that a separate kernel merges.
+//  * Pages in the 8-bit cache tier (gc_prefix_prefill_attn_q8): a 16-warp
+//    variant whose producer bulk-copies an image page's codes into the
+//    page's rows of the ring slot and whose fourth warpgroup dequantises
+//    them there (see "pages of the 8-bit image" below).
 //  * Every mbarrier wait and spin is bounded; a timeout raises the CTA's
 //    abort flag, all roles leave their loops, in-flight copies and MMAs are
 //    drained, TMEM is freed and GC_ERR_TIMEOUT is recorded in the pool
@@ -61,6 +65,8 @@ namespace {
 using namespace ptx;
 
 constexpr int kThreads = 384;
+// With pages read from an 8-bit image a fourth warpgroup converts them.
+constexpr int kThreadsQ8 = 512;
 // Batches up to this size are numbered longest request first (ranked in
 // shared memory by every CTA); larger batches keep the given order.
 constexpr int kSortMax = 512;
@@ -68,6 +74,10 @@ constexpr int kRegsProducer = 88;   // warps 0-3 after setmaxnreg.dec
 constexpr int kRegsSoftmax = 208;   // warps 4-11 after setmaxnreg.inc
 static_assert(128 * kRegsProducer + 256 * kRegsSoftmax <= kThreads * 168,
               "register split exceeds the launch allocation");
+constexpr int kRegsProducerQ8 = 64;  // warps 0-3 of the 8-bit variant
+constexpr int kRegsConverter = 32;   // warps 12-15 of the 8-bit variant
+static_assert(128 * (kRegsProducerQ8 + kRegsConverter) + 256 * kRegsSoftmax <= kThreadsQ8 * 128,
+              "register split of the 8-bit variant exceeds the launch allocation");
 constexpr int kTileM = 128;     // rows per Q tile
 constexpr int kTileN = 128;     // keys per K/V tile
 // The running row max is only recomputed when a tile's probabilities, taken
@@ -214,11 +224,137 @@ __device__ __forceinline__ int read_item(Barriers& bar, uint32_t k, volatile int
   return ok ? *reinterpret_cast<volatile int*>(&bar.item_slot[k & 1]) : -1;
 }
 
+// ------------------------------------------------- pages of the 8-bit image
+// With an 8-bit image (the cache tier's layout, one fp32 scale per (block,
+// layer, plane, kv head)), pages that the q8 table maps to the image reach
+// the ring in two stages.  The producer bulk-copies a page's ps*d codes into
+// the page's own rows of the ring slot (d = 128: code row r in the first
+// 128 bytes of tile row r; d = 64: code row k at byte ps*64 + 64k of the
+// page's rows) and looks the page's scale up one tile ahead; the converter
+// warpgroup (warps 12-15) then turns the codes into bf16 in place, with
+// the rounding of the 8-bit restore (bf16_rne(c * s)), at the positions the
+// tensor map's 128-byte swizzle gives pool pages, and adds its arrivals to
+// the slot's full barrier.  The pool is never written.
+constexpr int kConvWarps = 4;
+constexpr int kMaxPages = kTileN / 16;  // pages per K/V tile (ps >= 16)
+
+struct Q8State {
+  uint64_t codes_full[8];    // per ring slot: the codes have landed (tx bytes)
+  uint32_t mask[8];          // per slot: bit p = page p of the tile is an image page
+  int32_t rows_end[8];       // per slot: rows below this are keys; -1 ends the work
+  float scale[8][kMaxPages];  // per slot and page
+};
+
+__device__ __forceinline__ uint64_t q8_chunk_index(const Geom& geo, int blk, int kv) {
+  const uint64_t il = geo.q8_layer_major
+                          ? static_cast<uint64_t>(geo.layer) * geo.q8_n_blocks + blk
+                          : static_cast<uint64_t>(blk) * geo.L + geo.layer;
+  return il * 2 + kv;
+}
+
+// 16 codes (one 16-byte word) -> 16 bf16 values as two 16-byte words.
+__device__ __forceinline__ void dequant16(const uint4& v, float s, uint4& lo, uint4& hi) {
+  lo.x = q8_dequant2(v.x, 0, s);
+  lo.y = q8_dequant2(v.x, 1, s);
+  lo.z = q8_dequant2(v.y, 0, s);
+  lo.w = q8_dequant2(v.y, 1, s);
+  hi.x = q8_dequant2(v.z, 0, s);
+  hi.y = q8_dequant2(v.z, 1, s);
+  hi.z = q8_dequant2(v.w, 0, s);
+  hi.w = q8_dequant2(v.w, 1, s);
+}
+
+// Converter warp c of the warpgroup.  d = 128: tile rows [32c, 32c+32), in
+// batches of 8 rows (a batch lies in one page).  Each batch is read whole
+// (code row r sits under output row r's first 128 bytes) before any of it
+// is written.  d = 64: pages p = c, c+4, ..., each in ascending batches of
+// 8 rows; a batch's output rows only cover code rows of this or earlier
+// batches of the same page, which are already in registers or converted.
+// Rows at or past rows_end (V rows past the sequence end) are written as
+// zeros: their probabilities are zero, and 0 * NaN would poison the product.
+template <int D>
+__device__ void converter(uint8_t* smem_kv, Barriers& bar, Q8State& q8, const Geom& geo) {
+  using C = Cfg<D>;
+  const int lane = threadIdx.x & 31;
+  const int c = (threadIdx.x >> 5) - kThreads / 32;
+  volatile int* abortp = &bar.abort_flag;
+  for (uint32_t step = 0;; ++step) {
+    const int slot = step % C::kStages;
+    bool ok = mbar_wait(&q8.codes_full[slot], (step / C::kStages) & 1, abortp);
+    if (!__all_sync(0xffffffffu, ok)) break;
+    const int rows_end = *reinterpret_cast<volatile int32_t*>(&q8.rows_end[slot]);
+    if (rows_end < 0) break;
+    const uint32_t mask = *reinterpret_cast<volatile uint32_t*>(&q8.mask[slot]);
+    uint8_t* tile = smem_kv + slot * C::kTileBytes;
+    if (D == 128) {
+#pragma unroll 1
+      for (int a = 32 * c; a < 32 * c + 32; a += 8) {
+        const int p = a >> geo.ps_shift;
+        if (!((mask >> p) & 1u)) continue;
+        const float sc = q8.scale[slot][p];
+        uint4 v[2];
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const int r = a + q * 4 + (lane >> 3), u = lane & 7;
+          v[q] = r < rows_end ? *reinterpret_cast<const uint4*>(tile + r * 128 + u * 16)
+                              : make_uint4(0, 0, 0, 0);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const int r = a + q * 4 + (lane >> 3), u = lane & 7;
+          uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
+          if (r < rows_end) dequant16(v[q], sc, lo, hi);
+          const int h = u >> 2, q0 = (u & 3) * 2, sw = r & 7;
+          uint8_t* row = tile + h * C::kHalfBytes + r * 128;
+          // the two halves store their chunk pairs in opposite order, so the
+          // 8 lanes of a row hit 8 distinct bank groups in each store
+          if (h == 0) {
+            *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
+            *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
+          } else {
+            *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
+            *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
+          }
+        }
+        __syncwarp();
+      }
+    } else {
+#pragma unroll 1
+      for (int p = c; p < (kTileN >> geo.ps_shift); p += kConvWarps) {
+        if (!((mask >> p) & 1u)) continue;
+        const float sc = q8.scale[slot][p];
+        const int r0 = p << geo.ps_shift;
+        const uint8_t* codes = tile + r0 * 128 + geo.ps * 64;
+#pragma unroll 1
+        for (int a = 0; a < geo.ps; a += 8) {
+          const int k = a + (lane >> 2), u = lane & 3, r = r0 + k;
+          const uint4 v = r < rows_end ? *reinterpret_cast<const uint4*>(codes + k * 64 + u * 16)
+                                       : make_uint4(0, 0, 0, 0);
+          __syncwarp();
+          uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
+          if (r < rows_end) dequant16(v, sc, lo, hi);
+          const int sw = r & 7;
+          uint8_t* row = tile + r * 128;
+          *reinterpret_cast<uint4*>(row + (((2 * u) ^ sw) << 4)) = lo;
+          *reinterpret_cast<uint4*>(row + (((2 * u + 1) ^ sw) << 4)) = hi;
+          __syncwarp();
+        }
+      }
+    }
+    // the tensor core reads the slot through the async proxy
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&bar.kv_full[slot]);
+  }
+}
+
 // ------------------------------------------------------------------ roles
 template <int D, bool kQ8>
-__device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const int* item_start,
-                         int total_items, const Geom& geo, const CUtensorMap* map_q,
-                         const CUtensorMap* map_kv, const int32_t* __restrict__ block_table,
+__device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, Q8State* q8,
+                         const int* item_start, int total_items, const Geom& geo,
+                         const CUtensorMap* map_q, const CUtensorMap* map_kv,
+                         const int32_t* __restrict__ block_table,
                          const int32_t* __restrict__ prefix_lens,
                          const int32_t* __restrict__ new_lens,
                          const int32_t* __restrict__ cu_new_lens, int32_t* status,
@@ -228,9 +364,11 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
   volatile int* abortp = &bar.abort_flag;
   uint32_t q_count = 0, kv_count = 0, vfix_count = 0;
   uint32_t armed = 0, armed_par = 0;  // per slot: a load in flight, and its phase parity
+  uint32_t armed8 = 0, armed8_par = 0;  // the same for the code copies of image pages
   int armed_q = -1, armed_vfix = -1;
   bool ok = true;
   const uint32_t box_bytes = static_cast<uint32_t>(geo.ps) * 128;  // one page, one column block
+  const uint32_t page_codes = static_cast<uint32_t>(geo.ps) * D;   // one page of 8-bit codes
 
   for (uint32_t k = 0; ok; ++k) {
     const int it = claim_item(bar, k, work_counter, total_items, abortp, ok);
@@ -261,33 +399,55 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
     // every box of a 16-row-page tile could not keep up with the MMAs.
     const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
     const int pg = lane / C::kHalves, hh = lane % C::kHalves;
-    // lane p (< pages of the tile) looks up page p of a tile; tile j+1's
-    // lookup is issued before tile j's copies so its latency is hidden
-    auto lookup = [&](int j) -> int {
+    // lane p (< pages of the tile) looks up page p of a tile: its pool page,
+    // or its image block and K and V scales; tile j+1's lookup is issued
+    // before tile j's copies so its latency is hidden
+    struct Lookup {
+      int page;        // pool page, -1 none (or bad), -2 no page in this lane
+      int blk;         // image block, or -1
+      float sk, sv;    // the image page's scales
+    };
+    auto lookup = [&](int j) -> Lookup {
+      Lookup l{-2, -1, 0.f, 0.f};
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
       const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
       const int blk0 = key0 >> geo.ps_shift;
-      int pg_id = -2;  // -2: no page in this lane; -3: a page of the 8-bit image
       if (j < w.nt && lane < npages) {
-        pg_id = blk0 + lane < geo.max_blocks ? __ldg(block_table + bt_row + blk0 + lane) : -1;
-        if (kQ8 && blk0 + lane < geo.max_blocks && __ldg(geo.q8_table + bt_row + blk0 + lane) >= 0)
-          pg_id = -3;  // the converter warp fills it
+        if (blk0 + lane >= geo.max_blocks) {
+          l.page = -1;
+        } else {
+          const int32_t ib = kQ8 ? __ldg(geo.q8_table + bt_row + blk0 + lane) : -1;
+          if (ib < 0) {
+            l.page = __ldg(block_table + bt_row + blk0 + lane);
+          } else if (ib >= geo.q8_n_blocks) {
+            l.page = -1;
+            l.blk = -2;  // out of range, reported below
+          } else {
+            l.blk = ib;
+            const uint8_t* ck = geo.q8_image + q8_chunk_index(geo, ib, 0) * geo.q8_chunk;
+            l.sk = __ldg(reinterpret_cast<const float*>(ck) + w.g);
+            l.sv = __ldg(reinterpret_cast<const float*>(ck + geo.q8_chunk) + w.g);
+          }
+        }
       }
-      return pg_id;
+      return l;
     };
-    int page_next = lookup(w.j0);
+    Lookup next = lookup(w.j0);
     for (int j = w.j0; ok && j < w.nt; ++j) {
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
-      int page = page_next;
-      page_next = lookup(j + 1);
-      if (page != -2 && page != -3 && (page < 0 || page >= geo.num_pages)) {
+      Lookup cur = next;
+      next = lookup(j + 1);
+      int page = cur.page;
+      if (cur.blk == -2 || (page != -2 && cur.blk < 0 && (page < 0 || page >= geo.num_pages))) {
         record_error(status, GC_ERR_OUT_OF_RANGE);
         page = -1;
+        cur.blk = -1;
       }
-      if (page == -2 || page == -3) page = -1;
+      if (page == -2) page = -1;
       const int good = __popc(__ballot_sync(0xffffffffu, page >= 0));
+      const uint32_t img_mask = kQ8 ? __ballot_sync(0xffffffffu, cur.blk >= 0) : 0u;
       const int my_page = __shfl_sync(0xffffffffu, page, pg < 32 ? pg : 0);
       const bool issues = pg < kTileN / 16 && my_page >= 0;
 #pragma unroll 1
@@ -298,6 +458,25 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
         uint8_t* dst = smem_kv + slot * C::kTileBytes;
         const bool fix = kv == 1 && nkeys < kTileN;
         uint64_t* full = fix ? &bar.vfix : &bar.kv_full[slot];
+        if (kQ8) {
+          // codes of the image pages, converted by the converter warpgroup
+          if (cur.blk >= 0) q8->scale[slot][lane] = kv ? cur.sv : cur.sk;
+          __syncwarp();
+          if (lane == 0) {
+            q8->mask[slot] = img_mask;
+            q8->rows_end[slot] = fix ? nkeys : kTileN;
+            mbar_arrive_expect_tx(&q8->codes_full[slot], __popc(img_mask) * page_codes);
+          }
+          __syncwarp();
+          if (cur.blk >= 0) {
+            const uint8_t* src = geo.q8_image + q8_chunk_index(geo, cur.blk, kv) * geo.q8_chunk +
+                                 geo.q8_hdr + static_cast<uint64_t>(w.g) * page_codes;
+            uint8_t* cdst = dst + lane * box_bytes + (D == 128 ? 0 : geo.ps * 64);
+            bulk_load(cdst, src, page_codes, &q8->codes_full[slot]);
+          }
+          armed8 |= 1u << slot;
+          armed8_par = (armed8_par & ~(1u << slot)) | (((kv_count / C::kStages) & 1u) << slot);
+        }
         if (lane == 0)
           mbar_arrive_expect_tx(full, static_cast<uint32_t>(good) * box_bytes * C::kHalves);
         __syncwarp();
@@ -308,7 +487,8 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
         }
         if (fix) {
           // V rows past the end of the sequence must be zero, not stale or NaN:
-          // their P is zero but 0 * NaN would poison the PV product.
+          // their P is zero but 0 * NaN would poison the PV product.  Rows of
+          // image pages are zeroed by the converters (they hold codes here).
           ok = mbar_wait(&bar.vfix, vfix_count & 1, abortp);
           if (!ok) {
             armed &= ~(1u << slot);
@@ -319,7 +499,9 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
           const int zrows = kTileN - nkeys;
           for (int h = 0; h < C::kHalves; ++h) {
             uint4* z = reinterpret_cast<uint4*>(dst + h * C::kHalfBytes + nkeys * 128);
-            for (int k = lane; k < zrows * 8; k += 32) z[k] = make_uint4(0, 0, 0, 0);
+            for (int k = lane; k < zrows * 8; k += 32)
+              if (!kQ8 || !((img_mask >> ((nkeys + (k >> 3)) >> geo.ps_shift)) & 1u))
+                z[k] = make_uint4(0, 0, 0, 0);
           }
           fence_proxy_async_smem();
           __syncwarp();
@@ -332,115 +514,25 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, const
       }
     }
   }
+  if (kQ8 && ok) {
+    // tell the converters that the work is done (the slot's previous
+    // conversion has been consumed once the slot is free again)
+    const int slot = kv_count % C::kStages;
+    ok = mbar_wait(&bar.kv_empty[slot], ((kv_count / C::kStages) & 1) ^ 1, abortp);
+    if (ok && lane == 0) {
+      q8->rows_end[slot] = -1;
+      mbar_arrive(&q8->codes_full[slot]);
+    }
+  }
   if (!ok && lane == 0) {
     // drain copies still in flight before the CTA exits (bounded, ignores abort)
     int no_abort = 0;
     if (armed_q >= 0) mbar_wait(&bar.q_full, armed_q, &no_abort);
     if (armed_vfix >= 0) mbar_wait(&bar.vfix, armed_vfix, &no_abort);
-    for (int s = 0; s < C::kStages; ++s)
+    for (int s = 0; s < C::kStages; ++s) {
       if (armed & (1u << s)) mbar_wait(&bar.kv_full[s], (armed_par >> s) & 1u, &no_abort);
-  }
-}
-
-// Converter (warp 3, attention over 8-bit pages only).  It follows the same
-// work items and ring slots as the producer and fills the pages the producer
-// leaves out (those the q8 table maps to the 8-bit image): each 16 codes of
-// a page are one 16-byte load, dequantised exactly as the 8-bit restore does
-// (c * s in binary32, rounded to bf16) and stored at the positions the TMA
-// box would have written (rows of 128 bytes, 16-byte chunks swizzled by row
-// within 8-row groups).  The slot's full barrier then counts the producer's
-// copies and this warp's arrival.
-template <int D>
-__device__ void converter(uint8_t* smem_kv, Barriers& bar, const int* item_start,
-                          const Geom& geo, const int32_t* __restrict__ prefix_lens,
-                          const int32_t* __restrict__ new_lens,
-                          const int32_t* __restrict__ cu_new_lens, int32_t* status) {
-  using C = Cfg<D>;
-  const int lane = threadIdx.x & 31;
-  volatile int* abortp = &bar.abort_flag;
-  uint32_t kv_count = 0;
-  bool ok = true;
-  constexpr int kUnitsPerRow = D / 16;  // 16-code units in a row of the page
-  for (uint32_t k = 0; ok; ++k) {
-    const int it = read_item(bar, k, abortp, ok);
-    ok = __all_sync(0xffffffffu, ok);
-    if (!ok) break;
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&bar.item_empty[k & 1]);
-    if (it < 0) break;
-    Item w;
-    decode_item(it, item_start, geo, prefix_lens, new_lens, cu_new_lens, w);
-    const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
-    for (int j = w.j0; ok && j < w.nt; ++j) {
-      const int key0 = j * kTileN;
-      const int nkeys = min(kTileN, w.T - key0);
-      const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
-      const int blk0 = key0 >> geo.ps_shift;
-      int ib = -1;  // image block of page `lane` of the tile
-      if (lane < npages && blk0 + lane < geo.max_blocks) {
-        ib = __ldg(geo.q8_table + bt_row + blk0 + lane);
-        if (ib >= geo.q8_n_blocks) {
-          record_error(status, GC_ERR_OUT_OF_RANGE);
-          ib = -1;
-        }
-      }
-      const uint32_t mine = __ballot_sync(0xffffffffu, ib >= 0);
-#pragma unroll 1
-      for (int kv = 0; kv < 2; ++kv) {
-        const int slot = kv_count % C::kStages;
-        ok = mbar_wait(&bar.kv_empty[slot], ((kv_count / C::kStages) & 1) ^ 1, abortp);
-        ok = __all_sync(0xffffffffu, ok);
-        if (!ok) break;
-        uint8_t* dst = smem_kv + slot * C::kTileBytes;
-        // V rows past the sequence end are zeroed by the producer; leave them
-        const int rows_end = kv ? nkeys : kTileN;
-        for (uint32_t m = mine; m; m &= m - 1) {
-          const int p = __ffs(m) - 1;
-          const int blk = __shfl_sync(0xffffffffu, ib, p);
-          const uint64_t il = geo.q8_layer_major
-                                  ? static_cast<uint64_t>(geo.layer) * geo.q8_n_blocks + blk
-                                  : static_cast<uint64_t>(blk) * geo.L + geo.layer;
-          const uint8_t* chunk = geo.q8_image + (il * 2 + kv) * geo.q8_chunk;
-          const float sc = __ldg(reinterpret_cast<const float*>(chunk) + w.g);
-          const uint4* codes = reinterpret_cast<const uint4*>(
-              chunk + geo.q8_hdr + static_cast<uint64_t>(w.g) * geo.ps * D);
-          const int units = geo.ps * kUnitsPerRow;
-          for (int u0 = 0; u0 < units; u0 += 128) {
-            uint4 v[4];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const int u = u0 + q * 32 + lane;
-              v[q] = u < units ? __ldg(codes + u) : make_uint4(0, 0, 0, 0);
-            }
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const int u = u0 + q * 32 + lane;
-              if (u >= units) continue;
-              const int r = p * geo.ps + u / kUnitsPerRow;  // row of the tile
-              if (r >= rows_end) continue;
-              const int c0 = (u % kUnitsPerRow) * 16;       // first column
-              uint8_t* row = dst + (c0 >> 6) * C::kHalfBytes + r * 128;
-              const int q0 = (c0 & 63) >> 3;                 // first 16-byte chunk
-              uint4 lo, hi;
-              lo.x = q8_dequant2(v[q].x, 0, sc);
-              lo.y = q8_dequant2(v[q].x, 1, sc);
-              lo.z = q8_dequant2(v[q].y, 0, sc);
-              lo.w = q8_dequant2(v[q].y, 1, sc);
-              hi.x = q8_dequant2(v[q].z, 0, sc);
-              hi.y = q8_dequant2(v[q].z, 1, sc);
-              hi.z = q8_dequant2(v[q].w, 0, sc);
-              hi.w = q8_dequant2(v[q].w, 1, sc);
-              *reinterpret_cast<uint4*>(row + ((q0 ^ (r & 7)) << 4)) = lo;
-              *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ (r & 7)) << 4)) = hi;
-            }
-          }
-        }
-        // the tensor core reads the slot through the async proxy
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bar.kv_full[slot]);
-        ++kv_count;
-      }
+      if (kQ8 && (armed8 & (1u << s)))
+        mbar_wait(&q8->codes_full[s], (armed8_par >> s) & 1u, &no_abort);
     }
   }
 }
@@ -753,7 +845,7 @@ __device__ void softmax_wg(Barriers& bar, uint32_t tmem, const int* item_start,
 }
 
 template <int D, bool kQ8>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kQ8 ? kThreadsQ8 : kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                    const __grid_constant__ CUtensorMap map_kv,
                    const int32_t* __restrict__ block_table, const int32_t* __restrict__ prefix_lens,
@@ -769,6 +861,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   Barriers& bar = *reinterpret_cast<Barriers*>(smem_kv + C::kStages * C::kTileBytes);
   int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
   int16_t* order = reinterpret_cast<int16_t*>(item_start + geo.batch + 1);  // [min(batch, kSortMax)]
+  Q8State* q8 = kQ8 ? reinterpret_cast<Q8State*>(
+                          (reinterpret_cast<uintptr_t>(order + kSortMax) + 7) & ~uintptr_t(7))
+                    : nullptr;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
@@ -777,8 +872,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(&bar.vfix, 1);
     mbar_init(&bar.drain, 2);
     for (int s = 0; s < C::kStages; ++s) {
-      mbar_init(&bar.kv_full[s], kQ8 ? 2 : 1);  // + the converter's arrival
+      mbar_init(&bar.kv_full[s], kQ8 ? 1 + kConvWarps : 1);  // + one arrival per converter warp
       mbar_init(&bar.kv_empty[s], 2);
+      if (kQ8) mbar_init(&q8->codes_full[s], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&bar.s_full[i], 1);
@@ -787,7 +883,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(&bar.item_full[s], 1);
-      mbar_init(&bar.item_empty[s], kItemConsumers + (kQ8 ? 1 : 0));
+      mbar_init(&bar.item_empty[s], kItemConsumers);
     }
     bar.abort_flag = 0;
     bar.p0_steps = 0;
@@ -806,7 +902,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto total_len = [&](int b) {
       return geo.decode ? __ldg(geo.seq_lens + b) : __ldg(prefix_lens + b) + __ldg(new_lens + b);
     };
-    for (int b = threadIdx.x; b < geo.batch; b += kThreads) {
+    for (int b = threadIdx.x; b < geo.batch; b += blockDim.x) {
       const int tb = total_len(b);
       int rank = 0;
       for (int o = 0; o < geo.batch; ++o) {
@@ -858,18 +954,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int total_items = item_start[geo.batch];
 
   if (warp < 4) {
-    regs_dec<kRegsProducer>();
+    regs_dec<kQ8 ? kRegsProducerQ8 : kRegsProducer>();
     if (warp == 0) {
-      producer<D, kQ8>(smem_q, smem_kv, bar, item_start, total_items, geo, &map_q, &map_kv,
-                  block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
+      producer<D, kQ8>(smem_q, smem_kv, bar, q8, item_start, total_items, geo, &map_q, &map_kv,
+                       block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
     } else if (warp == 1 || warp == 2) {
       if (lane == 0)
         mma_issuer<D>(warp - 1, smem_q, smem_kv, bar, tmem, item_start, total_items, geo,
                       prefix_lens, new_lens, cu_new_lens);
       __syncwarp();
-    } else if (kQ8) {
-      converter<D>(smem_kv, bar, item_start, geo, prefix_lens, new_lens, cu_new_lens, status);
     }
+  } else if (kQ8 && warp >= kThreads / 32) {
+    regs_dec<kRegsConverter>();
+    converter<D>(smem_kv, bar, *q8, geo);
   } else {
     regs_inc<kRegsSoftmax>();
     if (warp < 8)
@@ -1007,7 +1104,7 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   }
   const size_t smem = 1024 + 2 * C::kTileBytes + C::kStages * C::kTileBytes + sizeof(Barriers) +
                       (static_cast<size_t>(a.batch) + 1) * sizeof(int) +
-                      kSortMax * sizeof(int16_t);
+                      kSortMax * sizeof(int16_t) + (q8 ? sizeof(Q8State) + 8 : 0);
   auto kernel = q8 ? attn_tc_kernel<D, true> : attn_tc_kernel<D, false>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
@@ -1015,7 +1112,7 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   // the work items are claimed from a counter in the pool's control block
   e = cudaMemsetAsync(work_counter, 0, sizeof(int), stream);
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: clearing the work counter");
-  kernel<<<pool->num_sms, kThreads, smem, stream>>>(
+  kernel<<<pool->num_sms, q8 ? kThreadsQ8 : kThreads, smem, stream>>>(
       map_q, map_kv, a.block_table, a.prefix_lens, a.new_lens, a.cu_new_lens,
       static_cast<__nv_bfloat16*>(a.out), geo, pool->status, work_counter);
   e = cudaGetLastError();
