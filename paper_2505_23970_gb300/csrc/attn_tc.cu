@@ -252,18 +252,6 @@ __device__ __forceinline__ uint64_t q8_chunk_index(const Geom& geo, int blk, int
   return il * 2 + kv;
 }
 
-// 16 codes (one 16-byte word) -> 16 bf16 values as two 16-byte words.
-__device__ __forceinline__ void dequant16(const uint4& v, float s, uint4& lo, uint4& hi) {
-  lo.x = q8_dequant2(v.x, 0, s);
-  lo.y = q8_dequant2(v.x, 1, s);
-  lo.z = q8_dequant2(v.y, 0, s);
-  lo.w = q8_dequant2(v.y, 1, s);
-  hi.x = q8_dequant2(v.z, 0, s);
-  hi.y = q8_dequant2(v.z, 1, s);
-  hi.z = q8_dequant2(v.w, 0, s);
-  hi.w = q8_dequant2(v.w, 1, s);
-}
-
 // Converter warp c of the warpgroup.  d = 128: tile rows [32c, 32c+32), in
 // batches of 8 rows (a batch lies in one page).  Each batch is read whole
 // (code row r sits under output row r's first 128 bytes) before any of it
@@ -304,7 +292,7 @@ __device__ void converter(uint8_t* smem_kv, Barriers& bar, Q8State& q8, const Ge
         for (int q = 0; q < 2; ++q) {
           const int r = a + q * 4 + (lane >> 3), u = lane & 7;
           uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
-          if (r < rows_end) dequant16(v[q], sc, lo, hi);
+          if (r < rows_end) q8_dequant16(v[q], sc, lo, hi);
           const int h = u >> 2, q0 = (u & 3) * 2, sw = r & 7;
           uint8_t* row = tile + h * C::kHalfBytes + r * 128;
           // the two halves store their chunk pairs in opposite order, so the
@@ -333,7 +321,7 @@ __device__ void converter(uint8_t* smem_kv, Barriers& bar, Q8State& q8, const Ge
                                        : make_uint4(0, 0, 0, 0);
           __syncwarp();
           uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
-          if (r < rows_end) dequant16(v, sc, lo, hi);
+          if (r < rows_end) q8_dequant16(v, sc, lo, hi);
           const int sw = r & 7;
           uint8_t* row = tile + r * 128;
           *reinterpret_cast<uint4*>(row + (((2 * u) ^ sw) << 4)) = lo;
@@ -1141,9 +1129,9 @@ gc_status launch_attn_tc(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t
   return launch<64>(pool, a, stream, pool->work_counter);
 }
 
-// Pages read from the 8-bit image run on the single-SM kernel at either head
-// size: its converter warp dequantises them into the same shared-memory
-// tiles the tensor map fills for pool pages.
+// Pages read from the 8-bit image run on the 16-warp variant of the
+// single-SM kernel at either head size: its converter warpgroup dequantises
+// them into the same shared-memory tiles the tensor map fills for pool pages.
 gc_status launch_attn_tc_q8(const gc_kv_pool* pool, const AttnArgs& a, const Q8Pages& q8,
                             cudaStream_t stream) {
   if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter, nullptr, &q8);

@@ -38,15 +38,42 @@ __device__ __forceinline__ void record_error(int32_t* status, int32_t code) {
   atomicCAS(status, 0, code);
 }
 
-// One 8-bit code pair -> a bf16 pair: codes k*2 and k*2+1 (bytes) of the
-// 32-bit word, each c * s in binary32 rounded to bf16 (nearest even).  The
-// 8-bit restore and the attention over 8-bit pages both dequantise with it,
-// so they produce the same bf16 values.
-__device__ __forceinline__ uint32_t q8_dequant2(uint32_t codes, int k, float s) {
-  const float a = static_cast<float>(static_cast<int8_t>((codes >> (16 * k)) & 0xffu)) * s;
-  const float b = static_cast<float>(static_cast<int8_t>((codes >> (16 * k + 8)) & 0xffu)) * s;
-  const __nv_bfloat162 p = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<const uint32_t*>(&p);
+// 16 8-bit codes (one 16-byte word, byte i = code i) -> 16 bf16 values
+// (lo: codes 0-7, hi: codes 8-15, in order), each c * s in binary32 rounded
+// to bf16 (nearest even).  The 8-bit restore and the attention over 8-bit
+// pages both dequantise with it, so they produce the same bf16 values.
+// float(c) is formed without a conversion instruction: the byte c + 128
+// (c xor 0x80) placed in the low mantissa bits of 2^23 is the float
+// 2^23 + 128 + c, from which subtracting 2^23 + 128 is exact; the
+// subtraction and the product (one rounding, as c * s) run as paired fp32
+// operations, two codes at a time.
+__device__ __forceinline__ uint32_t q8_pair(uint32_t biased, uint32_t sel, uint64_t s2) {
+  const uint32_t a = __byte_perm(biased, 0x4B000000u, 0x7540u + sel);
+  const uint32_t b = __byte_perm(biased, 0x4B000000u, 0x7540u + sel + 1);
+  uint32_t r;
+  asm("{\n\t.reg .b64 t;\n\t.reg .f32 x, y;\n\t"
+      "mov.b64 t, {%1, %2};\n\t"
+      "add.rn.f32x2 t, t, %3;\n\t"
+      "mul.rn.f32x2 t, t, %4;\n\t"
+      "mov.b64 {x, y}, t;\n\t"
+      "cvt.rn.bf16x2.f32 %0, y, x;\n\t}"
+      : "=r"(r)
+      : "r"(a), "r"(b), "l"(0xCB000080CB000080ull), "l"(s2));  // -(2^23 + 128), twice
+  return r;
+}
+
+__device__ __forceinline__ void q8_dequant16(const uint4& v, float s, uint4& lo, uint4& hi) {
+  const uint64_t s2 = (static_cast<uint64_t>(__float_as_uint(s)) << 32) | __float_as_uint(s);
+  const uint32_t x = v.x ^ 0x80808080u, y = v.y ^ 0x80808080u;
+  const uint32_t z = v.z ^ 0x80808080u, w = v.w ^ 0x80808080u;
+  lo.x = q8_pair(x, 0, s2);
+  lo.y = q8_pair(x, 2, s2);
+  lo.z = q8_pair(y, 0, s2);
+  lo.w = q8_pair(y, 2, s2);
+  hi.x = q8_pair(z, 0, s2);
+  hi.y = q8_pair(z, 2, s2);
+  hi.z = q8_pair(w, 0, s2);
+  hi.w = q8_pair(w, 2, s2);
 }
 
 // ---------------------------------------------------------------- launchers

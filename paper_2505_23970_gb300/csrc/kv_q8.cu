@@ -197,10 +197,6 @@ __global__ void __launch_bounds__(256) save_q8_kernel(uint8_t* __restrict__ imag
   }
 }
 
-__device__ __forceinline__ uint32_t dequant2(uint32_t codes, int k, float s) {
-  return q8_dequant2(codes, k, s);
-}
-
 // Each thread dequantises 16 codes (one 16-byte load) into 16 bf16 values
 // (two 16-byte stores; a warp's pair of stores covers 1 KB contiguously).
 __global__ void __launch_bounds__(256) restore_q8_kernel(const uint8_t* __restrict__ image,
@@ -245,14 +241,7 @@ __global__ void __launch_bounds__(256) restore_q8_kernel(const uint8_t* __restri
     for (int k = 0; k < U; ++k) {
       if (!dst[k]) continue;
       uint4 lo, hi;
-      lo.x = dequant2(v[k].x, 0, s[k]);
-      lo.y = dequant2(v[k].x, 1, s[k]);
-      lo.z = dequant2(v[k].y, 0, s[k]);
-      lo.w = dequant2(v[k].y, 1, s[k]);
-      hi.x = dequant2(v[k].z, 0, s[k]);
-      hi.y = dequant2(v[k].z, 1, s[k]);
-      hi.z = dequant2(v[k].w, 0, s[k]);
-      hi.w = dequant2(v[k].w, 1, s[k]);
+      q8_dequant16(v[k], s[k], lo, hi);
       dst[k][0] = lo;
       dst[k][1] = hi;
     }
