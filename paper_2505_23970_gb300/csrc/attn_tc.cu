@@ -74,9 +74,11 @@ constexpr int kRegsProducer = 88;   // warps 0-3 after setmaxnreg.dec
 constexpr int kRegsSoftmax = 208;   // warps 4-11 after setmaxnreg.inc
 static_assert(128 * kRegsProducer + 256 * kRegsSoftmax <= kThreads * 168,
               "register split exceeds the launch allocation");
-constexpr int kRegsProducerQ8 = 64;  // warps 0-3 of the 8-bit variant
-constexpr int kRegsConverter = 32;   // warps 12-15 of the 8-bit variant
-static_assert(128 * (kRegsProducerQ8 + kRegsConverter) + 256 * kRegsSoftmax <= kThreadsQ8 * 128,
+constexpr int kRegsProducerQ8 = 72;  // warps 0-3 of the 8-bit variant
+constexpr int kRegsConverter = 40;   // warps 12-15 of the 8-bit variant
+constexpr int kRegsSoftmaxQ8 = 200;  // warps 4-11 of the 8-bit variant
+static_assert(128 * (kRegsProducerQ8 + kRegsConverter) + 256 * kRegsSoftmaxQ8 <=
+                  kThreadsQ8 * 128,
               "register split of the 8-bit variant exceeds the launch allocation");
 constexpr int kTileM = 128;     // rows per Q tile
 constexpr int kTileN = 128;     // keys per K/V tile
@@ -387,46 +389,56 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, Q8Sta
     // every box of a 16-row-page tile could not keep up with the MMAs.
     const int64_t bt_row = static_cast<int64_t>(w.b) * geo.max_blocks;
     const int pg = lane / C::kHalves, hh = lane % C::kHalves;
-    // lane p (< pages of the tile) looks up page p of a tile: its pool page,
-    // or its image block and K and V scales; tile j+1's lookup is issued
-    // before tile j's copies so its latency is hidden
+    // lane p (< pages of the tile) looks up page p of a tile in two stages:
+    // its block-table (and q8-table) entries are loaded two tiles ahead, an
+    // image page's K and V scales one tile ahead, so no load is waited for
+    // while the current tile's copies are issued
+    struct Raw {
+      int page;  // block-table entry, -1 past max_blocks, -2 no page in this lane
+      int ib;    // q8-table entry, or -1
+    };
     struct Lookup {
       int page;        // pool page, -1 none (or bad), -2 no page in this lane
-      int blk;         // image block, or -1
+      int blk;         // image block, -1 none, -2 out of range
       float sk, sv;    // the image page's scales
     };
-    auto lookup = [&](int j) -> Lookup {
-      Lookup l{-2, -1, 0.f, 0.f};
+    auto load_raw = [&](int j) -> Raw {
+      Raw r{-2, -1};
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
       const int npages = (nkeys + geo.ps - 1) >> geo.ps_shift;
       const int blk0 = key0 >> geo.ps_shift;
       if (j < w.nt && lane < npages) {
-        if (blk0 + lane >= geo.max_blocks) {
+        const bool in = blk0 + lane < geo.max_blocks;
+        r.page = in ? __ldg(block_table + bt_row + blk0 + lane) : -1;
+        if (kQ8 && in) r.ib = __ldg(geo.q8_table + bt_row + blk0 + lane);
+      }
+      return r;
+    };
+    auto resolve = [&](const Raw& r) -> Lookup {
+      Lookup l{r.page, -1, 0.f, 0.f};
+      if (kQ8 && r.ib >= 0) {
+        l.page = -2;
+        if (r.ib >= geo.q8_n_blocks) {
           l.page = -1;
+          l.blk = -2;  // reported when the tile is issued
         } else {
-          const int32_t ib = kQ8 ? __ldg(geo.q8_table + bt_row + blk0 + lane) : -1;
-          if (ib < 0) {
-            l.page = __ldg(block_table + bt_row + blk0 + lane);
-          } else if (ib >= geo.q8_n_blocks) {
-            l.page = -1;
-            l.blk = -2;  // out of range, reported below
-          } else {
-            l.blk = ib;
-            const uint8_t* ck = geo.q8_image + q8_chunk_index(geo, ib, 0) * geo.q8_chunk;
-            l.sk = __ldg(reinterpret_cast<const float*>(ck) + w.g);
-            l.sv = __ldg(reinterpret_cast<const float*>(ck + geo.q8_chunk) + w.g);
-          }
+          l.blk = r.ib;
+          const uint8_t* ck = geo.q8_image + q8_chunk_index(geo, r.ib, 0) * geo.q8_chunk;
+          l.sk = __ldg(reinterpret_cast<const float*>(ck) + w.g);
+          l.sv = __ldg(reinterpret_cast<const float*>(ck + geo.q8_chunk) + w.g);
         }
       }
       return l;
     };
-    Lookup next = lookup(w.j0);
+    Lookup next = resolve(load_raw(w.j0));
+    Raw raw2 = load_raw(w.j0 + 1);
     for (int j = w.j0; ok && j < w.nt; ++j) {
       const int key0 = j * kTileN;
       const int nkeys = min(kTileN, w.T - key0);
       Lookup cur = next;
-      next = lookup(j + 1);
+      next = resolve(raw2);
+      raw2 = load_raw(j + 2);
       int page = cur.page;
       if (cur.blk == -2 || (page != -2 && cur.blk < 0 && (page < 0 || page >= geo.num_pages))) {
         record_error(status, GC_ERR_OUT_OF_RANGE);
@@ -956,7 +968,7 @@ __global__ void __launch_bounds__(kQ8 ? kThreadsQ8 : kThreads, 1)
     regs_dec<kRegsConverter>();
     converter<D>(smem_kv, bar, *q8, geo);
   } else {
-    regs_inc<kRegsSoftmax>();
+    regs_inc<kQ8 ? kRegsSoftmaxQ8 : kRegsSoftmax>();
     if (warp < 8)
       softmax_wg<D, 0>(bar, tmem, item_start, total_items, geo, prefix_lens, new_lens,
                        cu_new_lens, out);
