@@ -412,7 +412,7 @@ GC_API gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool*
  *   n_image_blocks  blocks in the image (>= 0).
  *   flags      0 or GC_RESTORE_LAYER_MAJOR.
  * Both head sizes run on a 16-warp variant of the one-SM kernel: the
- * producer bulk-copies each image page's codes into the K/V ring and a
+ * producer loads each image page's codes into the K/V ring (TMA) and a
  * fourth warpgroup dequantises them there, while the TMA unit loads the
  * pool pages.  Shared memory limits batch to 8192 as for
  * gc_prefix_prefill_attn.

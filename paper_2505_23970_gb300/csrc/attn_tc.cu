@@ -46,7 +46,7 @@
 //    range of K/V tiles); a request cut into several ranges writes fp32
 //    partials that a separate kernel merges.
 //  * Pages in the 8-bit cache tier (gc_prefix_prefill_attn_q8): a 16-warp
-//    variant whose producer bulk-copies an image page's codes into the
+//    variant whose producer loads an image page's codes (TMA) into the
 //    page's rows of the ring slot and whose fourth warpgroup dequantises
 //    them there (see "pages of the 8-bit image" below).
 //  * Every mbarrier wait and spin is bounded; a timeout raises the CTA's
@@ -75,8 +75,8 @@ constexpr int kRegsSoftmax = 208;   // warps 4-11 after setmaxnreg.inc
 static_assert(128 * kRegsProducer + 256 * kRegsSoftmax <= kThreads * 168,
               "register split exceeds the launch allocation");
 constexpr int kRegsProducerQ8 = 72;  // warps 0-3 of the 8-bit variant
-constexpr int kRegsConverter = 40;   // warps 12-15 of the 8-bit variant
-constexpr int kRegsSoftmaxQ8 = 200;  // warps 4-11 of the 8-bit variant
+constexpr int kRegsConverter = 56;   // warps 12-15 of the 8-bit variant
+constexpr int kRegsSoftmaxQ8 = 192;  // warps 4-11 of the 8-bit variant
 static_assert(128 * (kRegsProducerQ8 + kRegsConverter) + 256 * kRegsSoftmaxQ8 <=
                   kThreadsQ8 * 128,
               "register split of the 8-bit variant exceeds the launch allocation");
@@ -229,7 +229,8 @@ __device__ __forceinline__ int read_item(Barriers& bar, uint32_t k, volatile int
 // ------------------------------------------------- pages of the 8-bit image
 // With an 8-bit image (the cache tier's layout, one fp32 scale per (block,
 // layer, plane, kv head)), pages that the q8 table maps to the image reach
-// the ring in two stages.  The producer bulk-copies a page's ps*d codes into
+// the ring in two stages.  The producer loads a page's ps*d codes (one box of
+// a 3-D tensor map over the image's d-byte code rows) into
 // the page's own rows of the ring slot (d = 128: code row r in the first
 // 128 bytes of tile row r; d = 64: code row k at byte ps*64 + 64k of the
 // page's rows) and looks the page's scale up one tile ahead; the converter
@@ -255,13 +256,51 @@ __device__ __forceinline__ uint64_t q8_chunk_index(const Geom& geo, int blk, int
 }
 
 // Converter warp c of the warpgroup.  d = 128: tile rows [32c, 32c+32), in
-// batches of 8 rows (a batch lies in one page).  Each batch is read whole
+// batches of 16 rows (a batch lies in one page).  Each batch is read whole
 // (code row r sits under output row r's first 128 bytes) before any of it
 // is written.  d = 64: pages p = c, c+4, ..., each in ascending batches of
-// 8 rows; a batch's output rows only cover code rows of this or earlier
+// 16 rows; a batch's output rows only cover code rows of this or earlier
 // batches of the same page, which are already in registers or converted.
 // Rows at or past rows_end (V rows past the sequence end) are written as
 // zeros: their probabilities are zero, and 0 * NaN would poison the product.
+template <int D>
+__device__ __forceinline__ void convert_batch(uint8_t* tile, const uint8_t* codes, int r0,
+                                              int code_row0, float sc, int rows_end, int lane) {
+  using C = Cfg<D>;
+  constexpr int kWords = D / 16;        // 16-byte words of codes per row
+  constexpr int kLanesPerRow = kWords;  // one word per lane and row
+  constexpr int kRowsPerPass = 32 / kLanesPerRow;
+  constexpr int kPasses = 16 / kRowsPerPass;  // 16 rows per batch
+  const int u = lane % kLanesPerRow;
+  uint4 v[kPasses];
+#pragma unroll
+  for (int q = 0; q < kPasses; ++q) {
+    const int k = q * kRowsPerPass + lane / kLanesPerRow;  // row of the batch
+    v[q] = r0 + k < rows_end
+               ? *reinterpret_cast<const uint4*>(codes + (code_row0 + k) * D + u * 16)
+               : make_uint4(0, 0, 0, 0);
+  }
+  __syncwarp();
+#pragma unroll
+  for (int q = 0; q < kPasses; ++q) {
+    const int r = r0 + q * kRowsPerPass + lane / kLanesPerRow;
+    uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
+    if (r < rows_end) q8_dequant16(v[q], sc, lo, hi);
+    const int h = u >> 2, q0 = (u & 3) * 2, sw = r & 7;
+    uint8_t* row = tile + h * C::kHalfBytes + r * 128;
+    // at d = 128 the two halves store their chunk pairs in opposite order, so
+    // the 8 lanes of a row hit 8 distinct bank groups in each store
+    if (h == 0) {
+      *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
+      *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
+    } else {
+      *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
+      *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
+    }
+  }
+  __syncwarp();
+}
+
 template <int D>
 __device__ void converter(uint8_t* smem_kv, Barriers& bar, Q8State& q8, const Geom& geo) {
   using C = Cfg<D>;
@@ -278,58 +317,19 @@ __device__ void converter(uint8_t* smem_kv, Barriers& bar, Q8State& q8, const Ge
     uint8_t* tile = smem_kv + slot * C::kTileBytes;
     if (D == 128) {
 #pragma unroll 1
-      for (int a = 32 * c; a < 32 * c + 32; a += 8) {
+      for (int a = 32 * c; a < 32 * c + 32; a += 16) {
         const int p = a >> geo.ps_shift;
-        if (!((mask >> p) & 1u)) continue;
-        const float sc = q8.scale[slot][p];
-        uint4 v[2];
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const int r = a + q * 4 + (lane >> 3), u = lane & 7;
-          v[q] = r < rows_end ? *reinterpret_cast<const uint4*>(tile + r * 128 + u * 16)
-                              : make_uint4(0, 0, 0, 0);
-        }
-        __syncwarp();
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-          const int r = a + q * 4 + (lane >> 3), u = lane & 7;
-          uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
-          if (r < rows_end) q8_dequant16(v[q], sc, lo, hi);
-          const int h = u >> 2, q0 = (u & 3) * 2, sw = r & 7;
-          uint8_t* row = tile + h * C::kHalfBytes + r * 128;
-          // the two halves store their chunk pairs in opposite order, so the
-          // 8 lanes of a row hit 8 distinct bank groups in each store
-          if (h == 0) {
-            *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
-            *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
-          } else {
-            *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
-            *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
-          }
-        }
-        __syncwarp();
+        if ((mask >> p) & 1u) convert_batch<D>(tile, tile, a, a, q8.scale[slot][p], rows_end, lane);
       }
     } else {
 #pragma unroll 1
       for (int p = c; p < (kTileN >> geo.ps_shift); p += kConvWarps) {
         if (!((mask >> p) & 1u)) continue;
-        const float sc = q8.scale[slot][p];
         const int r0 = p << geo.ps_shift;
         const uint8_t* codes = tile + r0 * 128 + geo.ps * 64;
 #pragma unroll 1
-        for (int a = 0; a < geo.ps; a += 8) {
-          const int k = a + (lane >> 2), u = lane & 3, r = r0 + k;
-          const uint4 v = r < rows_end ? *reinterpret_cast<const uint4*>(codes + k * 64 + u * 16)
-                                       : make_uint4(0, 0, 0, 0);
-          __syncwarp();
-          uint4 lo = make_uint4(0, 0, 0, 0), hi = lo;
-          if (r < rows_end) q8_dequant16(v, sc, lo, hi);
-          const int sw = r & 7;
-          uint8_t* row = tile + r * 128;
-          *reinterpret_cast<uint4*>(row + (((2 * u) ^ sw) << 4)) = lo;
-          *reinterpret_cast<uint4*>(row + (((2 * u + 1) ^ sw) << 4)) = hi;
-          __syncwarp();
-        }
+        for (int a = 0; a < geo.ps; a += 16)
+          convert_batch<D>(tile, codes, r0 + a, a, q8.scale[slot][p], rows_end, lane);
       }
     }
     // the tensor core reads the slot through the async proxy
@@ -344,6 +344,7 @@ template <int D, bool kQ8>
 __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, Q8State* q8,
                          const int* item_start, int total_items, const Geom& geo,
                          const CUtensorMap* map_q, const CUtensorMap* map_kv,
+                         const CUtensorMap* map_q8,
                          const int32_t* __restrict__ block_table,
                          const int32_t* __restrict__ prefix_lens,
                          const int32_t* __restrict__ new_lens,
@@ -469,10 +470,10 @@ __device__ void producer(uint8_t* smem_q, uint8_t* smem_kv, Barriers& bar, Q8Sta
           }
           __syncwarp();
           if (cur.blk >= 0) {
-            const uint8_t* src = geo.q8_image + q8_chunk_index(geo, cur.blk, kv) * geo.q8_chunk +
-                                 geo.q8_hdr + static_cast<uint64_t>(w.g) * page_codes;
+            // rows [g*ps, (g+1)*ps) of the chunk's code rows (d bytes each)
             uint8_t* cdst = dst + lane * box_bytes + (D == 128 ? 0 : geo.ps * 64);
-            bulk_load(cdst, src, page_codes, &q8->codes_full[slot]);
+            tma_load_3d(cdst, map_q8, &q8->codes_full[slot], 0, w.g * geo.ps,
+                        static_cast<int32_t>(q8_chunk_index(geo, cur.blk, kv)));
           }
           armed8 |= 1u << slot;
           armed8_par = (armed8_par & ~(1u << slot)) | (((kv_count / C::kStages) & 1u) << slot);
@@ -848,6 +849,7 @@ template <int D, bool kQ8>
 __global__ void __launch_bounds__(kQ8 ? kThreadsQ8 : kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                    const __grid_constant__ CUtensorMap map_kv,
+                   const __grid_constant__ CUtensorMap map_q8,
                    const int32_t* __restrict__ block_table, const int32_t* __restrict__ prefix_lens,
                    const int32_t* __restrict__ new_lens, const int32_t* __restrict__ cu_new_lens,
                    __nv_bfloat16* __restrict__ out, Geom geo, int32_t* status,
@@ -892,6 +894,7 @@ __global__ void __launch_bounds__(kQ8 ? kThreadsQ8 : kThreads, 1)
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&map_q);
     prefetch_tensormap(&map_kv);
+    if (kQ8) prefetch_tensormap(&map_q8);
   }
   if (warp == 1) {
     tmem_alloc(&bar.tmem_base, 512);
@@ -957,7 +960,7 @@ __global__ void __launch_bounds__(kQ8 ? kThreadsQ8 : kThreads, 1)
     regs_dec<kQ8 ? kRegsProducerQ8 : kRegsProducer>();
     if (warp == 0) {
       producer<D, kQ8>(smem_q, smem_kv, bar, q8, item_start, total_items, geo, &map_q, &map_kv,
-                       block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
+                       &map_q8, block_table, prefix_lens, new_lens, cu_new_lens, status, work_counter);
     } else if (warp == 1 || warp == 2) {
       if (lane == 0)
         mma_issuer<D>(warp - 1, smem_q, smem_kv, bar, tmem, item_start, total_items, geo,
@@ -1102,6 +1105,28 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
     if (r != CUDA_SUCCESS)
       return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn: pool tensor map (CUresult %d)", (int)r);
   }
+  // 8-bit image: its code rows (d bytes each; Hkv*ps rows per chunk after the
+  // scale header) as a 3-D map, box = one page of one kv head
+  CUtensorMap map_q8 = map_kv;  // unused by the bf16 kernel
+  if (q8) {
+    const uint64_t chunks = static_cast<uint64_t>(q8->n_blocks) * cfg.num_layers * 2;
+    if (chunks >= (1ull << 31))
+      return fail(GC_ERR_UNSUPPORTED, "gc_prefix_prefill_attn_q8: image of %llu chunks (limit 2^31)",
+                  static_cast<unsigned long long>(chunks));
+    // an empty image is never read; the map then points at the pool
+    const void* base = chunks ? static_cast<const void*>(q8->image + geo.q8_hdr) : pool->data;
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(D),
+                          static_cast<cuuint64_t>(cfg.num_kv_heads) * cfg.page_size,
+                          chunks ? chunks : 1};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(geo.q8_chunk)};
+    cuuint32_t box[3] = {static_cast<cuuint32_t>(D), static_cast<cuuint32_t>(cfg.page_size), 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUresult r = enc(&map_q8, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void*>(base), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(GC_ERR_CUDA, "gc_prefix_prefill_attn_q8: image tensor map (CUresult %d)", (int)r);
+  }
   const size_t smem = 1024 + 2 * C::kTileBytes + C::kStages * C::kTileBytes + sizeof(Barriers) +
                       (static_cast<size_t>(a.batch) + 1) * sizeof(int) +
                       kSortMax * sizeof(int16_t) + (q8 ? sizeof(Q8State) + 8 : 0);
@@ -1113,7 +1138,7 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   e = cudaMemsetAsync(work_counter, 0, sizeof(int), stream);
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: clearing the work counter");
   kernel<<<pool->num_sms, q8 ? kThreadsQ8 : kThreads, smem, stream>>>(
-      map_q, map_kv, a.block_table, a.prefix_lens, a.new_lens, a.cu_new_lens,
+      map_q, map_kv, map_q8, a.block_table, a.prefix_lens, a.new_lens, a.cu_new_lens,
       static_cast<__nv_bfloat16*>(a.out), geo, pool->status, work_counter);
   e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "gc_prefix_prefill_attn: launch");
