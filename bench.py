@@ -513,7 +513,7 @@ def run_ours(args):
         "roofline": {"bound": "tensor", "achieved": attn_tflops, "peak": peak_t,
                      "unit": "TFLOP/s", "frac": attn_tflops / peak_t,
                      "traffic": traffic_record("attn_tc", WORKLOAD),
-                     "kernel": "attn_tc_kernel<128>", "peak_source": pk["source"] + " burst",
+                     "kernel": "attn_tc_kernel<128, 0>", "peak_source": pk["source"] + " burst",
                      "frac_of_sustained": (attn_tflops / pk["bf16_tflops_sustained"]
                                            if pk.get("bf16_tflops_sustained") else None),
                      "flops_per_launch": flops, "ms_per_launch": attn_ms},
