@@ -878,6 +878,61 @@ def bench_configs(args, pk):
     return res
 
 
+def decode_q8_entry(w, db, stream, pk, reps):
+    """The same decode step with every full cached page read from an 8-bit
+    image (gc_paged_decode_attn_q8); the page holding the new token stays in
+    the pool.  Algorithmic bytes: the image pages' codes and scales, the pool
+    pages' K and V rows, q and out."""
+    import torch
+
+    from paper_2505_23970_gb300 import binding as gcb
+    from paper_2505_23970_gb300.harness import _i32
+
+    table = np.full((w.B, w.max_blocks), -1, dtype=np.int32)
+    ids = []
+    for b in range(w.B):
+        full = int(w.prefix_lens[b]) // w.ps
+        table[b, :full] = np.arange(len(ids), len(ids) + full)
+        ids.extend(w.block_table[b, :full].tolist())
+    n = len(ids)
+    chunk8 = gcb.gc_kv_q8_chunk_bytes(db.pool.cfg)
+    img = torch.empty(max(n, 1) * w.L * 2 * chunk8, dtype=torch.uint8, device=db.q.device)
+    gcb.gc_kv_save_q8(db.pool.handle, img, _i32(np.asarray(ids, np.int32), db.q.device), n, 0,
+                      w.L, stream, None, gcb.GC_SAVE_DST_DEVICE)
+    table_d = _i32(table, db.q.device)
+    seq = _i32(w.total_lens, db.q.device)
+    need = gcb.gc_paged_decode_workspace_bytes(db.pool.handle, w.B, w.max_blocks, w.Hq)
+    wsb = torch.empty(max(need, 16), dtype=torch.uint8, device=db.q.device)
+    out = torch.empty_like(db.out)
+
+    def f():
+        gcb.gc_paged_decode_attn_q8(db.q, db.pool.handle, db.block_table, seq, out, stream, 0,
+                                    w.B, w.max_blocks, w.Hq, w.scale, wsb, need, img, table_d,
+                                    n, 0)
+
+    for _ in range(3):
+        f()
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        f()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / reps
+    ok = db.check(stream) == gcb.GC_OK
+    img_keys = n * w.ps
+    pool_keys = int(w.total_lens.sum()) - img_keys
+    byts = (n * 2 * chunk8 + pool_keys * w.Hkv * w.d * 2 * 2 +
+            2 * w.B * w.Hq * w.d * 2)
+    gbs = byts / (ms / 1e3) / 1e9
+    del img, wsb, out
+    return {"us_per_step": ms * 1e3, "bytes_per_step": byts, "gbs": gbs,
+            "frac_hbm": gbs / pk["hbm_gbs"], "tok_per_s": w.B / (ms / 1e3),
+            "image_pages": n, "device_status_ok": ok}
+
+
 def bench_decode(args, pk):
     """Paged decode attention (one new token per request) on two contexts
     mixes: 8 x 9216 tokens (the 70B prefill config, continued) and the 64
@@ -917,6 +972,7 @@ def bench_decode(args, pk):
                        "us_per_step": ms * 1e3, "bytes_per_step": kv + qo, "gbs": gbs,
                        "frac_hbm": gbs / pk["hbm_gbs"], "tok_per_s": w.B / (ms / 1e3),
                        "workspace_bytes": ws, "device_status_ok": ok}
+        res[w.name]["q8"] = decode_q8_entry(w, db, stream, pk, reps)
         db.close()
     return res
 

@@ -481,7 +481,30 @@ GC_API gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool,
                                       int32_t num_q_heads, float softmax_scale, void* workspace,
                                       size_t workspace_bytes);
 
-/* Message of the last failing call on this thread ("" if none). */
+/* Paged decode attention with the cached pages read from the 8-bit cache
+ * tier (Sec. 6.1: the 70B runs keep the KV in INT8; Sec. 2.1: decode is
+ * bound by memory, and an 8-bit page is half the bytes).  The result is
+ * exactly that of gc_kv_restore_q8 of the image pages into the pool followed
+ * by gc_paged_decode_attn: the kernel dequantises each image page
+ * (x' = bf16_rne(c * s), the restore's rounding) into the tile it would have
+ * loaded, and the pool is never written.
+ * Arguments as gc_paged_decode_attn, plus q8_image, q8_table, n_image_blocks
+ * and flags as gc_prefix_prefill_attn_q8 (q8_table [batch][max_blocks_per_seq]:
+ * an image block >= 0, or -1 for a pool page, e.g. the page the new token
+ * was appended to).  head_dim 128 only (the transposed decode kernel, with a
+ * converter warpgroup).
+ * Errors: as gc_paged_decode_attn; GC_ERR_UNSUPPORTED for head_dim 64;
+ * GC_ERR_INVALID_ARG for unknown flags, a NULL q8_table (or q8_image with
+ * n_image_blocks > 0), a misaligned q8_image. */
+GC_API gc_status gc_paged_decode_attn_q8(const void* q, const gc_kv_pool* pool,
+                                         const int32_t* block_table, const int32_t* seq_lens,
+                                         void* out, cudaStream_t stream, int32_t layer,
+                                         int32_t batch, int32_t max_blocks_per_seq,
+                                         int32_t num_q_heads, float softmax_scale,
+                                         void* workspace, size_t workspace_bytes,
+                                         const void* q8_image, const int32_t* q8_table,
+                                         int32_t n_image_blocks, uint32_t flags);
+
 /* Test hook, not part of the method (the paper has no counterpart): launches
  * one thread that waits on a device barrier nobody arrives at, with the same
  * bounded wait every libgc kernel uses.  After its limit (about 1.5 s) the
@@ -490,6 +513,7 @@ GC_API gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool,
  * exercised without hanging the GPU.  Errors: GC_ERR_INVALID_ARG, GC_ERR_CUDA. */
 GC_API gc_status gc_selftest_wait_timeout(gc_kv_pool* pool, cudaStream_t stream);
 
+/* Message of the last failing call on this thread ("" if none). */
 GC_API const char* gc_last_error(void);
 
 /* Static name of a status code. */

@@ -41,7 +41,7 @@ EXPORTED = (
     "gc_kv_restore_q8",
     "gc_kv_append", "gc_prefix_prefill_attn",
     "gc_prefix_prefill_attn_simt", "gc_prefix_prefill_attn_noalloc",
-    "gc_prefix_prefill_attn_q8",
+    "gc_prefix_prefill_attn_q8", "gc_paged_decode_attn_q8",
     "gc_paged_decode_workspace_bytes", "gc_paged_decode_attn", "gc_selftest_wait_timeout",
     "gc_last_error",
     "gc_status_string",
@@ -103,13 +103,15 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         lib.gc_paged_decode_workspace_bytes.restype = ctypes.c_size_t
         lib.gc_paged_decode_attn.argtypes = [vp, vp, vp, vp, vp, vp, i32, i32, i32, i32,
                                              ctypes.c_float, vp, ctypes.c_size_t]
+        lib.gc_paged_decode_attn_q8.argtypes = lib.gc_paged_decode_attn.argtypes + [vp, vp, i32,
+                                                                                  u32]
         for f in ("gc_kv_pool_create", "gc_kv_pool_destroy", "gc_kv_pool_data",
                   "gc_kv_pool_check", "gc_kv_restore", "gc_kv_save", "gc_kv_restore_layers",
                   "gc_kv_save_layers", "gc_kv_stage_layers", "gc_kv_save_q8", "gc_kv_restore_q8",
                   "gc_kv_append",
                   "gc_prefix_prefill_attn", "gc_prefix_prefill_attn_simt",
                   "gc_prefix_prefill_attn_noalloc", "gc_prefix_prefill_attn_q8",
-                  "gc_paged_decode_attn"):
+                  "gc_paged_decode_attn", "gc_paged_decode_attn_q8"):
             getattr(lib, f).restype = ctypes.c_int
         lib.gc_last_error.argtypes = []
         lib.gc_last_error.restype = ctypes.c_char_p
@@ -358,6 +360,20 @@ def gc_paged_decode_attn(q, pool, block_table, seq_lens, out, stream, layer: int
                                        max_blocks_per_seq, num_q_heads, softmax_scale,
                                        _addr(workspace), workspace_bytes),
            "gc_paged_decode_attn")
+
+
+def gc_paged_decode_attn_q8(q, pool, block_table, seq_lens, out, stream, layer: int, batch: int,
+                            max_blocks_per_seq: int, num_q_heads: int, softmax_scale: float,
+                            workspace, workspace_bytes: int, q8_image, q8_table,
+                            n_image_blocks: int, flags: int = 0) -> None:
+    """gc_paged_decode_attn with the pages that q8_table maps (>= 0) read from
+    the 8-bit image q8_image instead of the pool."""
+    _check(load().gc_paged_decode_attn_q8(_addr(q), pool, _addr(block_table), _addr(seq_lens),
+                                          _addr(out), _stream(stream), layer, batch,
+                                          max_blocks_per_seq, num_q_heads, softmax_scale,
+                                          _addr(workspace), workspace_bytes, _addr(q8_image),
+                                          _addr(q8_table), n_image_blocks, flags),
+           "gc_paged_decode_attn_q8")
 
 
 def gc_selftest_wait_timeout(pool, stream=None) -> None:

@@ -65,7 +65,49 @@ constexpr int kMaxStages = 6;
 struct DGeom {
   int32_t batch, Hq, Hkv, G, ps, ps_shift, num_pages, max_blocks, layer;
   float scale_log2;
+  // pages read from an 8-bit image (the cache tier's layout): q8_table[b][j]
+  // >= 0 names the image block holding page j of request b
+  const uint8_t* q8_image;
+  const int32_t* q8_table;
+  int32_t q8_n_blocks, q8_layer_major, L;
+  uint32_t q8_chunk;  // bytes of one (block, layer, plane) chunk
 };
+
+// ---------------------------------------------------- the 8-bit variant
+// Pages of an 8-bit image reach the K/V ring in two stages: the producer
+// loads a page's ps x 128 codes (one box of a 3-D tensor map over the
+// image's 128-byte code rows) into a ring of 16 KB code slots, code row n of
+// the tile at byte 128 n, and its K and V scales (plain loads, a tile
+// ahead); a converter warpgroup (warps 8-11) turns them into bf16, with the
+// rounding of the 8-bit restore, at the grouped, swizzled positions the
+// pool's 4-D boxes give pool pages, once the MMA has freed the tile's slot,
+// and adds its four arrivals to the slot's full barrier.  The pool is never
+// written.
+constexpr int kConvWarpsD = 4;
+constexpr int kConvWarp0 = 8;
+constexpr int kThreadsQ8 = kThreads + 32 * kConvWarpsD;
+constexpr int kCodeStages = 4;
+constexpr int kCodeSlotBytes = kKeys * kD;  // 16 KB
+constexpr int kMaxPagesD = kKeys / 16;
+constexpr int kRegsRolesQ8 = 152;    // warps 0-3 of the 8-bit variant
+constexpr int kRegsSoftmaxQ8 = 208;  // warps 4-7
+constexpr int kRegsConvQ8 = 128;     // warps 8-11
+static_assert(128 * (kRegsRolesQ8 + kRegsSoftmaxQ8 + kRegsConvQ8) <= kThreadsQ8 * 168,
+              "register split of the 8-bit variant exceeds the launch allocation");
+
+struct D8State {
+  uint64_t code_full[kCodeStages], code_empty[kCodeStages];
+  uint32_t mask[kCodeStages];  // bit p: page p of the step's tile is an image page
+  int32_t end[kCodeStages];    // 1: no more steps
+  float scale[kCodeStages][kMaxPagesD];
+};
+
+__device__ __forceinline__ uint64_t d_chunk_index(const DGeom& geo, int blk, int kv) {
+  const uint64_t il = geo.q8_layer_major
+                          ? static_cast<uint64_t>(geo.layer) * geo.q8_n_blocks + blk
+                          : static_cast<uint64_t>(blk) * geo.L + geo.layer;
+  return il * 2 + kv;
+}
 
 struct DBar {
   uint64_t q_full[2], q_empty[2], drain;
@@ -219,6 +261,235 @@ __device__ void d_producer(uint8_t* smem_q, uint8_t* smem_kv, DBar& bar, const i
       if (armed_q & (1u << s)) mbar_wait(&bar.q_full[s], (armed_q_par >> s) & 1u, &no_abort);
     for (int s = 0; s < kStages; ++s)
       if (armed & (1u << s)) mbar_wait(&bar.kv_full[s], (armed_par >> s) & 1u, &no_abort);
+  }
+}
+
+// The producer of the 8-bit variant: Q^T as above; per K/V step the codes
+// of the tile's image pages into the next code slot, then the pool pages
+// into the ring slot.  Lane p handles page p; a tile's table entries are
+// loaded two tiles ahead and an image page's scales one tile ahead (within a
+// piece; the first tile of a piece waits for its lookups).
+template <int kStages>
+__device__ void d_producer_q8(uint8_t* smem_q, uint8_t* smem_kv, uint8_t* smem_code, DBar& bar,
+                              D8State& q8, const int* unit_start, int u0, int u1,
+                              const DGeom& geo, const CUtensorMap* map_q,
+                              const CUtensorMap* map_kv, const CUtensorMap* map_q8,
+                              const int32_t* __restrict__ block_table,
+                              const int32_t* __restrict__ seq_lens, int32_t* status) {
+  const int lane = threadIdx.x & 31;
+  volatile int* abortp = &bar.abort_flag;
+  uint32_t q_count = 0, step = 0;
+  uint32_t armed = 0, armed_par = 0, armed_q = 0, armed_q_par = 0, armed8 = 0, armed8_par = 0;
+  bool ok = true;
+  const uint32_t box_bytes = static_cast<uint32_t>(geo.ps) * kD * 2;  // one pool page
+  const uint32_t code_bytes = static_cast<uint32_t>(geo.ps) * kD;    // one image page
+
+  struct Raw {
+    int page, ib;  // block-table and q8-table entries (-2: no page in this lane)
+  };
+  struct Look {
+    int page;      // pool page, -1 none or bad, -2 no page in this lane
+    int blk;       // image block, -1 none, -2 out of range
+    float sk, sv;  // the image page's scales
+  };
+  auto raw_load = [&](const Piece& pc, int jt) -> Raw {
+    Raw r{-2, -1};
+    const int key0 = jt * kKeys;
+    const int np = (min(kKeys, pc.T - key0) + geo.ps - 1) >> geo.ps_shift;
+    const int blk = (key0 >> geo.ps_shift) + lane;
+    if (lane < np) {
+      if (blk < geo.max_blocks) {
+        const int64_t e = static_cast<int64_t>(pc.b) * geo.max_blocks + blk;
+        r.page = __ldg(block_table + e);
+        r.ib = __ldg(geo.q8_table + e);
+      } else {
+        r.page = -1;
+      }
+    }
+    return r;
+  };
+  auto resolve = [&](const Piece& pc, const Raw& r) -> Look {
+    Look l{r.page, -1, 0.f, 0.f};
+    if (r.ib >= 0) {
+      l.page = -2;
+      if (r.ib >= geo.q8_n_blocks) {
+        l.page = -1;
+        l.blk = -2;
+      } else {
+        l.blk = r.ib;
+        const uint8_t* ck = geo.q8_image + d_chunk_index(geo, r.ib, 0) * geo.q8_chunk;
+        l.sk = __ldg(reinterpret_cast<const float*>(ck) + pc.g);
+        l.sv = __ldg(reinterpret_cast<const float*>(ck + geo.q8_chunk) + pc.g);
+      }
+    }
+    return l;
+  };
+  int u = u0;
+  Piece w, wn;
+  bool have = u < u1;
+  Look next{-2, -1, 0.f, 0.f};
+  Raw raw2{-2, -1};
+  if (have) {
+    next_piece(u, u1, u0, unit_start, geo, seq_lens, w);
+    next = resolve(w, raw_load(w, w.j0));
+    if (w.j0 + 1 < w.j1) raw2 = raw_load(w, w.j0 + 1);
+  }
+  while (ok && have) {
+    // ---- Q^T: the 16 q rows from head g*G of token b (rows past the end read 0)
+    const int qs = q_count & 1;
+    ok = mbar_wait(&bar.q_empty[qs], ((q_count >> 1) & 1) ^ 1, abortp);
+    if (!ok) break;
+    if (lane == 0) {
+      mbar_arrive_expect_tx(&bar.q_full[qs], kSmallBytes);
+      const int row = w.b * geo.Hq + w.g * geo.G;
+      uint8_t* dst = smem_q + qs * kSmallBytes;
+      tma_load_2d(dst, map_q, &bar.q_full[qs], 0, row);
+      tma_load_2d(dst + kSmallHalf, map_q, &bar.q_full[qs], 64, row);
+    }
+    armed_q |= 1u << qs;
+    armed_q_par = (armed_q_par & ~(1u << qs)) | (((q_count >> 1) & 1u) << qs);
+    ++q_count;
+    have = false;
+    for (int j = w.j0; ok && j < w.j1; ++j) {
+      Look cur = next;
+      if (j + 1 < w.j1) {
+        next = resolve(w, raw2);
+        raw2 = j + 2 < w.j1 ? raw_load(w, j + 2) : Raw{-2, -1};
+      } else if (u < u1) {
+        next_piece(u, u1, u0, unit_start, geo, seq_lens, wn);
+        next = resolve(wn, raw_load(wn, wn.j0));
+        raw2 = wn.j0 + 1 < wn.j1 ? raw_load(wn, wn.j0 + 1) : Raw{-2, -1};
+        have = true;
+      }
+      int page = cur.page;
+      if (cur.blk == -2 || (cur.blk < 0 && page != -2 && (page < 0 || page >= geo.num_pages))) {
+        record_error(status, GC_ERR_OUT_OF_RANGE);
+        page = -1;
+        cur.blk = -1;
+      }
+      if (page == -2) page = -1;
+      const int good = __popc(__ballot_sync(0xffffffffu, page >= 0));
+      const uint32_t img = __ballot_sync(0xffffffffu, cur.blk >= 0);
+#pragma unroll 1
+      for (int kv = 0; kv < 2; ++kv) {
+        // codes of the image pages into the next code slot
+        const int cs = step % kCodeStages;
+        ok = mbar_wait(&q8.code_empty[cs], ((step / kCodeStages) & 1) ^ 1, abortp);
+        if (!ok) break;
+        if (cur.blk >= 0) q8.scale[cs][lane] = kv ? cur.sv : cur.sk;
+        __syncwarp();
+        if (lane == 0) {
+          q8.mask[cs] = img;
+          q8.end[cs] = 0;
+          mbar_arrive_expect_tx(&q8.code_full[cs], __popc(img) * code_bytes);
+        }
+        __syncwarp();
+        if (cur.blk >= 0)
+          tma_load_3d(smem_code + cs * kCodeSlotBytes + lane * code_bytes, map_q8,
+                      &q8.code_full[cs], 0, w.g * geo.ps,
+                      static_cast<int32_t>(d_chunk_index(geo, cur.blk, kv)));
+        armed8 |= 1u << cs;
+        armed8_par = (armed8_par & ~(1u << cs)) | (((step / kCodeStages) & 1u) << cs);
+        // pool pages into the ring slot
+        const int slot = step % kStages;
+        ok = mbar_wait(&bar.kv_empty[slot], ((step / kStages) & 1) ^ 1, abortp);
+        if (!ok) break;
+        uint8_t* dst = smem_kv + slot * kTileBytes;
+        if (lane == 0)
+          mbar_arrive_expect_tx(&bar.kv_full[slot], static_cast<uint32_t>(good) * box_bytes);
+        __syncwarp();
+        if (page >= 0) {
+          const int plane_row = (geo.layer * 2 + kv) * geo.num_pages;
+          const int row = (((plane_row + page) * geo.Hkv + w.g) << geo.ps_shift);
+          tma_load_4d(dst + lane * box_bytes, map_kv, &bar.kv_full[slot], 0, 0, 0, row >> 3);
+        }
+        armed |= 1u << slot;
+        armed_par = (armed_par & ~(1u << slot)) | (((step / kStages) & 1u) << slot);
+        ++step;
+      }
+    }
+    if (have) w = wn;
+  }
+  if (ok) {
+    // no more steps: tell the converters through the next code slot
+    const int cs = step % kCodeStages;
+    ok = mbar_wait(&q8.code_empty[cs], ((step / kCodeStages) & 1) ^ 1, abortp);
+    if (ok && lane == 0) {
+      q8.end[cs] = 1;
+      mbar_arrive(&q8.code_full[cs]);
+    }
+  }
+  if (!ok && lane == 0) {
+    // abort: wait (bounded, ignoring the flag) for the copies this warp armed
+    int no_abort = 0;
+    for (int s = 0; s < 2; ++s)
+      if (armed_q & (1u << s)) mbar_wait(&bar.q_full[s], (armed_q_par >> s) & 1u, &no_abort);
+    for (int s = 0; s < kCodeStages; ++s)
+      if (armed8 & (1u << s)) mbar_wait(&q8.code_full[s], (armed8_par >> s) & 1u, &no_abort);
+    for (int s = 0; s < kStages; ++s)
+      if (armed & (1u << s)) mbar_wait(&bar.kv_full[s], (armed_par >> s) & 1u, &no_abort);
+  }
+}
+
+// Converter warp c (warps 8-11) of the 8-bit variant: keys [32c, 32c+32) of
+// every step's tile, in batches of 16 keys (a batch lies in one page), for
+// the pages the step's mask marks.  Code row n sits at byte 128 n of the code
+// slot; key n, column half h lands at (n / 8) * 2048 + h * 1024 + (n % 8) * 128
+// with 16-byte chunk q at q ^ (n % 8), as the pool's boxes lay out pool pages.
+template <int kStages>
+__device__ void d_converter(uint8_t* smem_kv, const uint8_t* smem_code, DBar& bar, D8State& q8,
+                            const DGeom& geo) {
+  const int lane = threadIdx.x & 31;
+  const int c = (threadIdx.x >> 5) - kConvWarp0;
+  const int u = lane & 7;                  // 16-code word of a key's row
+  const int h = u >> 2, q0 = (u & 3) * 2;  // column half and first chunk it lands in
+  volatile int* abortp = &bar.abort_flag;
+  for (uint32_t step = 0;; ++step) {
+    const int cs = step % kCodeStages;
+    bool ok = mbar_wait(&q8.code_full[cs], (step / kCodeStages) & 1, abortp);
+    if (!__all_sync(0xffffffffu, ok)) break;
+    if (*reinterpret_cast<volatile int32_t*>(&q8.end[cs])) break;
+    const uint32_t mask = *reinterpret_cast<volatile uint32_t*>(&q8.mask[cs]);
+    const int slot = step % kStages;
+    // the ring slot is free once the MMAs of its previous use have completed
+    ok = mbar_wait(&bar.kv_empty[slot], ((step / kStages) & 1) ^ 1, abortp);
+    if (!__all_sync(0xffffffffu, ok)) break;
+    uint8_t* tile = smem_kv + slot * kTileBytes;
+    const uint8_t* codes = smem_code + cs * kCodeSlotBytes;
+#pragma unroll 1
+    for (int a = 32 * c; a < 32 * c + 32; a += 16) {
+      const int p = a >> geo.ps_shift;
+      if (!((mask >> p) & 1u)) continue;
+      const float sc = q8.scale[cs][p];
+      uint4 v[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        v[q] = *reinterpret_cast<const uint4*>(codes + (a + q * 4 + (lane >> 3)) * 128 + u * 16);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int n = a + q * 4 + (lane >> 3);
+        uint4 lo, hi;
+        q8_dequant16(v[q], sc, lo, hi);
+        const int sw = n & 7;
+        uint8_t* row = tile + (n >> 3) * kGroupBytes + h * kAtomBytes + sw * 128;
+        // the two halves store their chunk pairs in opposite order, so the 8
+        // lanes of a key hit 8 distinct bank groups in each store
+        if (h == 0) {
+          *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
+          *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
+        } else {
+          *reinterpret_cast<uint4*>(row + (((q0 + 1) ^ sw) << 4)) = hi;
+          *reinterpret_cast<uint4*>(row + ((q0 ^ sw) << 4)) = lo;
+        }
+      }
+    }
+    // the tensor core reads the slot through the async proxy
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      mbar_arrive(&bar.kv_full[slot]);
+      mbar_arrive(&q8.code_empty[cs]);
+    }
   }
 }
 
@@ -571,10 +842,11 @@ __device__ void d_softmax(uint8_t* smem_p, uint8_t* smem_kv, DBar& bar, float* x
   }
 }
 
-template <int kStages>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int kStages, bool kQ8>
+__global__ void __launch_bounds__(kQ8 ? kThreadsQ8 : kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap map_q,
                      const __grid_constant__ CUtensorMap map_kv,
+                     const __grid_constant__ CUtensorMap map_q8,
                      const int32_t* __restrict__ block_table, const int32_t* __restrict__ seq_lens,
                      __nv_bfloat16* __restrict__ out, void* ws_raw, DGeom geo,
                      int32_t* status, int* merge_counters) {
@@ -584,16 +856,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem_q = base;                      // Q^T x 2, 8 KB
   uint8_t* smem_p = base + 2 * kSmallBytes;    // P^T x 2, 8 KB
   uint8_t* smem_kv = base + 4 * kSmallBytes;   // ring, 1024-aligned
-  DBar& bar = *reinterpret_cast<DBar*>(smem_kv + kStages * kTileBytes);
+  uint8_t* smem_code = smem_kv + kStages * kTileBytes;  // 8-bit variant: code slots
+  DBar& bar = *reinterpret_cast<DBar*>(smem_code + (kQ8 ? kCodeStages * kCodeSlotBytes : 0));
   float* xbuf = reinterpret_cast<float*>(&bar + 1);             // [2][4][kN]
   int* unit_start = reinterpret_cast<int*>(xbuf + 2 * 4 * kN);  // [batch + 1]
+  D8State* q8 = reinterpret_cast<D8State*>(
+      (reinterpret_cast<uintptr_t>(unit_start + geo.batch + 1) + 7) & ~uintptr_t(7));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     mbar_init(&bar.drain, 1);
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&bar.kv_full[s], 1);
+      mbar_init(&bar.kv_full[s], kQ8 ? 1 + kConvWarpsD : 1);  // + one arrival per converter
       mbar_init(&bar.kv_empty[s], 1);
+    }
+    if (kQ8) {
+      for (int s = 0; s < kCodeStages; ++s) {
+        mbar_init(&q8->code_full[s], 1);
+        mbar_init(&q8->code_empty[s], kConvWarpsD);
+      }
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar.q_full[b], 1);
@@ -609,6 +890,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     prefetch_tensormap(&map_q);
     prefetch_tensormap(&map_kv);
+    if (kQ8) prefetch_tensormap(&map_q8);
   }
   if (warp == 1) {
     tmem_alloc(&bar.tmem_base, kTmemCols);
@@ -659,16 +941,28 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int u1 = min(total, u0 + per);
   const Workspace ws = carve(ws_raw, gridDim.x);
 
+  if (kQ8) {
+    // warpgroups: roles, softmax, converters
+    if (warp < 4) regs_dec<kRegsRolesQ8>();
+    else if (warp < 8) regs_inc<kRegsSoftmaxQ8>();
+    else regs_dec<kRegsConvQ8>();
+  }
   if (warp == 0) {
-    d_producer<kStages>(smem_q, smem_kv, bar, unit_start, u0, u1, geo, &map_q, &map_kv,
-                        block_table, seq_lens, status);
+    if (kQ8)
+      d_producer_q8<kStages>(smem_q, smem_kv, smem_code, bar, *q8, unit_start, u0, u1, geo,
+                             &map_q, &map_kv, &map_q8, block_table, seq_lens, status);
+    else
+      d_producer<kStages>(smem_q, smem_kv, bar, unit_start, u0, u1, geo, &map_q, &map_kv,
+                          block_table, seq_lens, status);
   } else if (warp == 1) {
     if (lane == 0)
       d_issuer<kStages>(smem_q, smem_p, smem_kv, bar, tmem, unit_start, u0, u1, geo, seq_lens);
     __syncwarp();
-  } else if (warp >= kSoftmaxWarp0) {
+  } else if (warp >= kSoftmaxWarp0 && warp < kSoftmaxWarp0 + 4) {
     d_softmax<kStages>(smem_p, smem_kv, bar, xbuf, tmem, unit_start, u0, u1, geo, seq_lens, out, ws, per,
                        merge_counters);
+  } else if (kQ8 && warp >= kConvWarp0) {
+    d_converter<kStages>(smem_kv, smem_code, bar, *q8, geo);
   }
   tc_fence_before();
   __syncthreads();
@@ -695,16 +989,18 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // One CTA per SM, at most one per merge counter of the pool's control block.
 int decode_grid(const gc_kv_pool* pool) { return min(pool->num_sms, kMergeCounters); }
 
-size_t smem_bytes(int stages, int batch) {
+size_t smem_bytes(int stages, int batch, bool q8 = false) {
   return 1024 + 4 * kSmallBytes + static_cast<size_t>(stages) * kTileBytes + sizeof(DBar) +
-         2 * 4 * kN * sizeof(float) + (static_cast<size_t>(batch) + 1) * sizeof(int);
+         2 * 4 * kN * sizeof(float) + (static_cast<size_t>(batch) + 1) * sizeof(int) +
+         (q8 ? kCodeStages * static_cast<size_t>(kCodeSlotBytes) + sizeof(D8State) + 8 : 0);
 }
 
-template <int kStages>
+template <int kStages, bool kQ8>
 gc_status launch_stages(const gc_kv_pool* pool, const DecodeArgs& a, const DGeom& geo,
-                        const CUtensorMap& map_q, const CUtensorMap& map_kv, cudaStream_t stream) {
-  const size_t smem = smem_bytes(kStages, a.batch);
-  cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStages>,
+                        const CUtensorMap& map_q, const CUtensorMap& map_kv,
+                        const CUtensorMap& map_q8, cudaStream_t stream) {
+  const size_t smem = smem_bytes(kStages, a.batch, kQ8);
+  cudaError_t e = cudaFuncSetAttribute(decode_tc_kernel<kStages, kQ8>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return cuda_fail(e, "gc_paged_decode_attn: smem attribute");
@@ -713,12 +1009,13 @@ gc_status launch_stages(const gc_kv_pool* pool, const DecodeArgs& a, const DGeom
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   lc.gridDim = dim3(decode_grid(pool));
-  lc.blockDim = dim3(kThreads);
+  lc.blockDim = dim3(kQ8 ? kThreadsQ8 : kThreads);
   lc.dynamicSmemBytes = smem;
   lc.stream = stream;
   lc.attrs = attr;
   lc.numAttrs = 1;
-  e = cudaLaunchKernelEx(&lc, decode_tc_kernel<kStages>, map_q, map_kv, a.block_table, a.seq_lens,
+  e = cudaLaunchKernelEx(&lc, decode_tc_kernel<kStages, kQ8>, map_q, map_kv, map_q8, a.block_table,
+                         a.seq_lens,
                          static_cast<__nv_bfloat16*>(a.out), a.workspace, geo, pool->status,
                          pool->merge_counters);
   if (e != cudaSuccess) return cuda_fail(e, "gc_paged_decode_attn: launch");
@@ -737,7 +1034,8 @@ size_t decode_tc_workspace_bytes(const gc_kv_pool* pool, int32_t) {
   return grid * 2 * kN * kD * sizeof(float) + grid * 2 * kN * sizeof(float2);
 }
 
-gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream) {
+gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream,
+                           const Q8Pages* q8) {
   const size_t need = decode_tc_workspace_bytes(pool, a.batch);
   if (a.workspace == nullptr || a.workspace_bytes < need)
     return fail(GC_ERR_INVALID_ARG,
@@ -766,6 +1064,12 @@ gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStre
   geo.max_blocks = a.max_blocks;
   geo.layer = a.layer;
   geo.scale_log2 = a.softmax_scale * 1.4426950408889634f;
+  geo.q8_image = q8 ? q8->image : nullptr;
+  geo.q8_table = q8 ? q8->table : nullptr;
+  geo.q8_n_blocks = q8 ? q8->n_blocks : 0;
+  geo.q8_layer_major = q8 && q8->layer_major ? 1 : 0;
+  geo.L = cfg.num_layers;
+  geo.q8_chunk = static_cast<uint32_t>(q8_chunk_bytes(cfg));
   const uint64_t pool_rows = static_cast<uint64_t>(cfg.num_layers) * 2 * cfg.num_pages *
                              cfg.num_kv_heads * cfg.page_size;
   if (pool_rows >= (1ull << 31))
@@ -800,11 +1104,38 @@ gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStre
     if (r != CUDA_SUCCESS)
       return fail(GC_ERR_CUDA, "gc_paged_decode_attn: pool tensor map (CUresult %d)", (int)r);
   }
-  // six ring slots unless the unit table of a large batch needs the room
   constexpr size_t kSmemLimit = 232448;
+  if (q8) {
+    // the image's code rows (128 bytes each; Hkv*ps rows per chunk after the
+    // scale header) as a 3-D map, box = one page of one kv head
+    const uint64_t chunks = static_cast<uint64_t>(q8->n_blocks) * cfg.num_layers * 2;
+    if (chunks >= (1ull << 31))
+      return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn_q8: image of %llu chunks (limit 2^31)",
+                  static_cast<unsigned long long>(chunks));
+    const void* base = chunks ? static_cast<const void*>(q8->image + q8_header_bytes(cfg))
+                              : pool->data;  // an empty image is never read
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(kD),
+                          static_cast<cuuint64_t>(cfg.num_kv_heads) * cfg.page_size,
+                          chunks ? chunks : 1};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(geo.q8_chunk)};
+    cuuint32_t box[3] = {static_cast<cuuint32_t>(kD), static_cast<cuuint32_t>(cfg.page_size), 1};
+    cuuint32_t es[3] = {1, 1, 1};
+    CUtensorMap map_q8;
+    CUresult r = enc(&map_q8, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void*>(base), dims,
+                     strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(GC_ERR_CUDA, "gc_paged_decode_attn_q8: image tensor map (CUresult %d)", (int)r);
+    // four ring slots and four code slots unless a large batch's unit table
+    // needs the room
+    return smem_bytes(4, a.batch, true) <= kSmemLimit
+               ? launch_stages<4, true>(pool, a, geo, map_q, map_kv, map_q8, stream)
+               : launch_stages<3, true>(pool, a, geo, map_q, map_kv, map_q8, stream);
+  }
+  // six ring slots unless the unit table of a large batch needs the room
   const gc_status st = smem_bytes(6, a.batch) <= kSmemLimit
-                           ? launch_stages<6>(pool, a, geo, map_q, map_kv, stream)
-                           : launch_stages<5>(pool, a, geo, map_q, map_kv, stream);
+                           ? launch_stages<6, false>(pool, a, geo, map_q, map_kv, map_kv, stream)
+                           : launch_stages<5, false>(pool, a, geo, map_q, map_kv, map_kv, stream);
   return st;
 }
 

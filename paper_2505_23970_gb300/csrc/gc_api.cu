@@ -670,6 +670,53 @@ gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool, const int3
   return gc::launch_decode(pool, a, stream);
 }
 
+gc_status gc_paged_decode_attn_q8(const void* q, const gc_kv_pool* pool,
+                                  const int32_t* block_table, const int32_t* seq_lens, void* out,
+                                  cudaStream_t stream, int32_t layer, int32_t batch,
+                                  int32_t max_blocks_per_seq, int32_t num_q_heads,
+                                  float softmax_scale, void* workspace, size_t workspace_bytes,
+                                  const void* q8_image, const int32_t* q8_table,
+                                  int32_t n_image_blocks, uint32_t flags) {
+  Range range_("gc_paged_decode_attn_q8");
+  g_msg[0] = 0;
+  const char* who = "gc_paged_decode_attn_q8";
+  if (!pool) return fail(GC_ERR_INVALID_ARG, "%s: pool is NULL", who);
+  if (batch < 0 || max_blocks_per_seq < 0 || n_image_blocks < 0)
+    return fail(GC_ERR_INVALID_ARG, "%s: negative size", who);
+  if (flags & ~GC_RESTORE_LAYER_MAJOR)
+    return fail(GC_ERR_INVALID_ARG, "%s: unknown flags 0x%x", who, flags);
+  if (layer < 0 || layer >= pool->cfg.num_layers)
+    return fail(GC_ERR_OUT_OF_RANGE, "%s: layer %d outside [0, %d)", who, layer,
+                pool->cfg.num_layers);
+  const int hkv = pool->cfg.num_kv_heads;
+  if (num_q_heads <= 0 || num_q_heads % hkv)
+    return fail(GC_ERR_INVALID_ARG, "%s: num_q_heads %d not a multiple of num_kv_heads %d", who,
+                num_q_heads, hkv);
+  const int G = num_q_heads / hkv;
+  if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16)
+    return fail(GC_ERR_UNSUPPORTED, "%s: q heads per kv head %d not in {1,2,4,8,16}", who, G);
+  if (!gc::decode_tc_supported(pool, num_q_heads))
+    return fail(GC_ERR_UNSUPPORTED, "%s: head_dim %d (only 128)", who, pool->cfg.head_dim);
+  if (!(softmax_scale > 0.0f) || softmax_scale == __builtin_inff())
+    return fail(GC_ERR_INVALID_ARG, "%s: softmax_scale must be positive and finite", who);
+  if (batch > 8192) return fail(GC_ERR_UNSUPPORTED, "%s: batch %d > 8192", who, batch);
+  if (batch == 0) return GC_OK;
+  if (!q || !out || !block_table || !seq_lens || !q8_table || (n_image_blocks > 0 && !q8_image))
+    return fail(GC_ERR_INVALID_ARG, "%s: NULL array argument", who);
+  if (max_blocks_per_seq == 0) return fail(GC_ERR_INVALID_ARG, "%s: max_blocks_per_seq is 0", who);
+  if (static_cast<int64_t>(max_blocks_per_seq) * pool->cfg.page_size > 2147483647LL)
+    return fail(GC_ERR_UNSUPPORTED, "%s: %lld-token block table", who,
+                static_cast<long long>(max_blocks_per_seq) * pool->cfg.page_size);
+  if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out) |
+       reinterpret_cast<uintptr_t>(workspace) | reinterpret_cast<uintptr_t>(q8_image)) % 16)
+    return fail(GC_ERR_INVALID_ARG, "%s: q / out / workspace / q8_image not 16-byte aligned", who);
+  const gc::DecodeArgs a{q, out, block_table, seq_lens, batch, max_blocks_per_seq, layer,
+                         num_q_heads, softmax_scale, workspace, workspace_bytes};
+  const gc::Q8Pages q8{static_cast<const uint8_t*>(q8_image), q8_table, n_image_blocks,
+                       (flags & GC_RESTORE_LAYER_MAJOR) != 0};
+  return gc::launch_decode_tc(pool, a, stream, &q8);
+}
+
 gc_status gc_selftest_wait_timeout(gc_kv_pool* pool, cudaStream_t stream) {
   g_msg[0] = 0;
   if (!pool) return fail(GC_ERR_INVALID_ARG, "gc_selftest_wait_timeout: pool is NULL");

@@ -171,7 +171,10 @@ gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_
 // at most 16 q heads per kv head.
 bool decode_tc_supported(const gc_kv_pool* pool, int32_t num_q_heads);
 size_t decode_tc_workspace_bytes(const gc_kv_pool* pool, int32_t batch);
-gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream);
+// With q8, the pages that q8->table maps (>= 0) are read from the 8-bit
+// image instead of the pool.
+gc_status launch_decode_tc(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream,
+                           const Q8Pages* q8 = nullptr);
 // Workspace bytes of a decode call on either path.
 size_t decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch, int32_t max_blocks,
                               int32_t num_q_heads);

@@ -71,6 +71,10 @@ def test_null_pool_is_rejected_before_any_launch(lib):
         gcb.gc_prefix_prefill_attn_q8(16, None, 16, 16, 16, 16, None, 0, 16, 1, 1, 8, 0.1, 1,
                                       16, 16, 1, 0)
     assert e.value.status == gcb.GC_ERR_INVALID_ARG
+    with pytest.raises(gcb.GcError) as e:
+        gcb.gc_paged_decode_attn_q8(16, None, 16, 16, 16, None, 0, 1, 1, 8, 0.1, 16, 1 << 20,
+                                    16, 16, 1, 0)
+    assert e.value.status == gcb.GC_ERR_INVALID_ARG
 
 
 def test_status_strings(lib):
