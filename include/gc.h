@@ -491,10 +491,11 @@ GC_API gc_status gc_paged_decode_attn(const void* q, const gc_kv_pool* pool,
  * Arguments as gc_paged_decode_attn, plus q8_image, q8_table, n_image_blocks
  * and flags as gc_prefix_prefill_attn_q8 (q8_table [batch][max_blocks_per_seq]:
  * an image block >= 0, or -1 for a pool page, e.g. the page the new token
- * was appended to).  head_dim 128 only (the transposed decode kernel, with a
- * converter warpgroup).
- * Errors: as gc_paged_decode_attn; GC_ERR_UNSUPPORTED for head_dim 64;
- * GC_ERR_INVALID_ARG for unknown flags, a NULL q8_table (or q8_image with
+ * was appended to).  Kernels: head_dim 128 runs the transposed decode kernel
+ * with a converter warpgroup, head_dim 64 the decode mode of the 8-bit
+ * prefill variant (gc_prefix_prefill_attn_q8); both dequantise with the
+ * restore's rounding.
+ * Errors: as gc_paged_decode_attn; GC_ERR_INVALID_ARG also for unknown flags, a NULL q8_table (or q8_image with
  * n_image_blocks > 0), a misaligned q8_image. */
 GC_API gc_status gc_paged_decode_attn_q8(const void* q, const gc_kv_pool* pool,
                                          const int32_t* block_table, const int32_t* seq_lens,

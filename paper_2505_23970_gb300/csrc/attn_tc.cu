@@ -1176,9 +1176,9 @@ gc_status launch_attn_tc_q8(const gc_kv_pool* pool, const AttnArgs& a, const Q8P
 }
 
 gc_status launch_attn_tc_decode(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode& dm,
-                                cudaStream_t stream) {
-  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter, &dm);
-  return launch<64>(pool, a, stream, pool->work_counter, &dm);
+                                cudaStream_t stream, const Q8Pages* q8) {
+  if (pool->cfg.head_dim == 128) return launch<128>(pool, a, stream, pool->work_counter, &dm, q8);
+  return launch<64>(pool, a, stream, pool->work_counter, &dm, q8);
 }
 
 }  // namespace gc

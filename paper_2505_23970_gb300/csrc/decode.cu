@@ -113,12 +113,13 @@ size_t decode_workspace_bytes(const gc_kv_pool* pool, int32_t batch, int32_t max
   return decode_split(pool, batch, max_blocks, num_q_heads).workspace_bytes;
 }
 
-gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream) {
+gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream,
+                        const Q8Pages* q8) {
   if (a.batch > 8192) return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: batch %d > 8192", a.batch);
   if (static_cast<int64_t>(a.max_blocks) * pool->cfg.page_size > 2147483647LL)
     return fail(GC_ERR_UNSUPPORTED, "gc_paged_decode_attn: %lld-token block table",
                 static_cast<long long>(a.max_blocks) * pool->cfg.page_size);
-  if (decode_tc_supported(pool, a.num_q_heads)) return launch_decode_tc(pool, a, stream);
+  if (decode_tc_supported(pool, a.num_q_heads)) return launch_decode_tc(pool, a, stream, q8);
   const DecodeSplit sp = decode_split(pool, a.batch, a.max_blocks, a.num_q_heads);
   if (sp.workspace_bytes > 0 && (a.workspace == nullptr || a.workspace_bytes < sp.workspace_bytes))
     return fail(GC_ERR_INVALID_ARG,
@@ -132,7 +133,7 @@ gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_
   AttnArgs args{a.q, a.out, a.block_table, nullptr, nullptr, nullptr, a.batch, a.max_blocks,
                 a.layer, a.num_q_heads, a.batch, a.softmax_scale};
   const DecodeMode dm{sp.split_tiles, sp.splits, a.seq_lens, static_cast<float*>(a.workspace)};
-  gc_status st = launch_attn_tc_decode(pool, args, dm, stream);
+  gc_status st = launch_attn_tc_decode(pool, args, dm, stream, q8);
   if (st != GC_OK || sp.splits <= 1) return st;
   const unsigned heads = static_cast<unsigned>(a.batch) * static_cast<unsigned>(a.num_q_heads);
   // programmatic dependent launch: the merge grid is set up while the

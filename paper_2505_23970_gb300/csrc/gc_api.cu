@@ -695,18 +695,12 @@ gc_status gc_paged_decode_attn_q8(const void* q, const gc_kv_pool* pool,
   const int G = num_q_heads / hkv;
   if (G != 1 && G != 2 && G != 4 && G != 8 && G != 16)
     return fail(GC_ERR_UNSUPPORTED, "%s: q heads per kv head %d not in {1,2,4,8,16}", who, G);
-  if (!gc::decode_tc_supported(pool, num_q_heads))
-    return fail(GC_ERR_UNSUPPORTED, "%s: head_dim %d (only 128)", who, pool->cfg.head_dim);
   if (!(softmax_scale > 0.0f) || softmax_scale == __builtin_inff())
     return fail(GC_ERR_INVALID_ARG, "%s: softmax_scale must be positive and finite", who);
-  if (batch > 8192) return fail(GC_ERR_UNSUPPORTED, "%s: batch %d > 8192", who, batch);
   if (batch == 0) return GC_OK;
   if (!q || !out || !block_table || !seq_lens || !q8_table || (n_image_blocks > 0 && !q8_image))
     return fail(GC_ERR_INVALID_ARG, "%s: NULL array argument", who);
   if (max_blocks_per_seq == 0) return fail(GC_ERR_INVALID_ARG, "%s: max_blocks_per_seq is 0", who);
-  if (static_cast<int64_t>(max_blocks_per_seq) * pool->cfg.page_size > 2147483647LL)
-    return fail(GC_ERR_UNSUPPORTED, "%s: %lld-token block table", who,
-                static_cast<long long>(max_blocks_per_seq) * pool->cfg.page_size);
   if ((reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(out) |
        reinterpret_cast<uintptr_t>(workspace) | reinterpret_cast<uintptr_t>(q8_image)) % 16)
     return fail(GC_ERR_INVALID_ARG, "%s: q / out / workspace / q8_image not 16-byte aligned", who);
@@ -714,7 +708,7 @@ gc_status gc_paged_decode_attn_q8(const void* q, const gc_kv_pool* pool,
                          num_q_heads, softmax_scale, workspace, workspace_bytes};
   const gc::Q8Pages q8{static_cast<const uint8_t*>(q8_image), q8_table, n_image_blocks,
                        (flags & GC_RESTORE_LAYER_MAJOR) != 0};
-  return gc::launch_decode_tc(pool, a, stream, &q8);
+  return gc::launch_decode(pool, a, stream, &q8);
 }
 
 gc_status gc_selftest_wait_timeout(gc_kv_pool* pool, cudaStream_t stream) {

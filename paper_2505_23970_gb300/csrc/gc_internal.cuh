@@ -142,7 +142,7 @@ struct DecodeMode {
   float* ws;
 };
 gc_status launch_attn_tc_decode(const gc_kv_pool* pool, const AttnArgs& a, const DecodeMode& dm,
-                                cudaStream_t stream);
+                                cudaStream_t stream, const Q8Pages* q8 = nullptr);
 // Host-side bound of the attention kernels' 32-bit work numbering (items and
 // q rows of one call, with a margin of two claims per CTA of `grid`):
 // GC_ERR_UNSUPPORTED before anything is launched when a call could pass it.
@@ -166,7 +166,10 @@ struct DecodeSplit {
 };
 DecodeSplit decode_split(const gc_kv_pool* pool, int32_t batch, int32_t max_blocks,
                          int32_t num_q_heads);
-gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream);
+// With q8, the pages that q8->table maps (>= 0) are read from the 8-bit
+// image instead of the pool.
+gc_status launch_decode(const gc_kv_pool* pool, const DecodeArgs& a, cudaStream_t stream,
+                        const Q8Pages* q8 = nullptr);
 // The transposed tensor-core decode kernel (decode_tc.cu): head_dim 128 and
 // at most 16 q heads per kv head.
 bool decode_tc_supported(const gc_kv_pool* pool, int32_t num_q_heads);

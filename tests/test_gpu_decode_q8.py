@@ -109,13 +109,15 @@ def test_q8_decode_mix():
     decode_q8_parity(wl.decode_mix(seed=1))
 
 
-@pytest.mark.parametrize("G,ps", [(1, 16), (4, 32), (16, 64), (8, 128)])
-def test_q8_decode_groupings_and_page_sizes(G, ps):
-    """Head groupings and page sizes, contexts that end inside a page and on
-    a page boundary, one of a single key."""
+@pytest.mark.parametrize("G,d,ps", [(1, 128, 16), (4, 128, 32), (16, 128, 64), (8, 128, 128),
+                                    (2, 64, 16), (8, 64, 64)])
+def test_q8_decode_groupings_and_page_sizes(G, d, ps):
+    """Head groupings, both head sizes (d 64 runs the decode mode of the 8-bit
+    prefill variant) and page sizes, contexts that end inside a page and on a
+    page boundary, one of a single key."""
     Hkv = 2
     ctx = [1, ps, ps + 1, 3 * ps - 1, 700, 129]
-    w = wl.custom(f"q8dec-G{G}-ps{ps}", len(ctx), G * Hkv, Hkv, 128, ps,
+    w = wl.custom(f"q8dec-G{G}-d{d}-ps{ps}", len(ctx), G * Hkv, Hkv, d, ps,
                   [c - 1 for c in ctx], [1] * len(ctx), seed=G + ps)
     decode_q8_parity(w)
 
@@ -165,20 +167,20 @@ def test_q8_decode_pool_untouched_and_bad_entry_reported():
     assert status == gcb.GC_ERR_OUT_OF_RANGE
 
 
+def test_q8_decode_d64_long_contexts_split_and_merged():
+    """d 64 with contexts long enough that requests are cut into key ranges
+    (fp32 partials merged by the merge kernel)."""
+    w = wl.custom("q8dec-d64-split", 3, 16, 4, 64, 16, [8191, 3000, 20], [1] * 3, seed=16)
+    decode_q8_parity(w)
+
+
 def test_q8_decode_host_checks():
     import torch
-    w = wl.custom("q8dec-args", 1, 8, 1, 64, 16, [63], [1], seed=13)
-    db = DeviceBatch(w, with_restore=False)
-    seq = _i32(w.total_lens, "cuda")
     img = torch.zeros(4096, dtype=torch.uint8, device="cuda")
-    tab = _i32(np.full((1, w.max_blocks), -1, np.int32), "cuda")
     ws = torch.empty(1 << 20, dtype=torch.uint8, device="cuda")
-    with pytest.raises(gcb.GcError) as e:  # head_dim 64
-        gcb.gc_paged_decode_attn_q8(db.q, db.pool.handle, db.block_table, seq, db.out, None, 0, 1,
-                                    w.max_blocks, w.Hq, w.scale, ws, ws.numel(), img, tab, 0, 0)
-    assert e.value.status == gcb.GC_ERR_UNSUPPORTED
-    db.close()
     w = wl.custom("q8dec-args2", 1, 8, 1, 128, 16, [63], [1], seed=13)
+    seq = _i32(w.total_lens, "cuda")
+    tab = _i32(np.full((1, w.max_blocks), -1, np.int32), "cuda")
     db = DeviceBatch(w, with_restore=False)
     for image, table, flags in ((img, tab, 0x10), (img, None, 0), (img.data_ptr() + 4, tab, 0)):
         with pytest.raises(gcb.GcError) as e:
