@@ -78,21 +78,22 @@ struct DGeom {
 // loads a page's ps x 128 codes (one box of a 3-D tensor map over the
 // image's 128-byte code rows) into a ring of 16 KB code slots, code row n of
 // the tile at byte 128 n, and its K and V scales (plain loads, a tile
-// ahead); a converter warpgroup (warps 8-11) turns them into bf16, with the
+// ahead); two converter warpgroups (warps 8-15) turn them into bf16, with the
 // rounding of the 8-bit restore, at the grouped, swizzled positions the
 // pool's 4-D boxes give pool pages, once the MMA has freed the tile's slot,
-// and adds its four arrivals to the slot's full barrier.  The pool is never
-// written.
-constexpr int kConvWarpsD = 4;
+// and add their eight arrivals to the slot's full barrier.  The pool is
+// never written.
+constexpr int kConvWarpsD = 8;
 constexpr int kConvWarp0 = 8;
 constexpr int kThreadsQ8 = kThreads + 32 * kConvWarpsD;
 constexpr int kCodeStages = 4;
 constexpr int kCodeSlotBytes = kKeys * kD;  // 16 KB
 constexpr int kMaxPagesD = kKeys / 16;
-constexpr int kRegsRolesQ8 = 152;    // warps 0-3 of the 8-bit variant
-constexpr int kRegsSoftmaxQ8 = 208;  // warps 4-7
-constexpr int kRegsConvQ8 = 128;     // warps 8-11
-static_assert(128 * (kRegsRolesQ8 + kRegsSoftmaxQ8 + kRegsConvQ8) <= kThreadsQ8 * 168,
+constexpr int kRegsRolesQ8 = 112;    // warps 0-3 of the 8-bit variant
+constexpr int kRegsSoftmaxQ8 = 192;  // warps 4-7
+constexpr int kRegsConvQ8 = 104;     // warps 8-15
+static_assert(128 * (kRegsRolesQ8 + kRegsSoftmaxQ8) + 32 * kConvWarpsD * kRegsConvQ8 <=
+                  kThreadsQ8 * 128,
               "register split of the 8-bit variant exceeds the launch allocation");
 
 struct D8State {
@@ -431,8 +432,8 @@ __device__ void d_producer_q8(uint8_t* smem_q, uint8_t* smem_kv, uint8_t* smem_c
   }
 }
 
-// Converter warp c (warps 8-11) of the 8-bit variant: keys [32c, 32c+32) of
-// every step's tile, in batches of 16 keys (a batch lies in one page), for
+// Converter warp c (warps 8-15) of the 8-bit variant: keys [16c, 16c+16) of
+// every step's tile, in batches of 8 keys (a batch lies in one page), for
 // the pages the step's mask marks.  Code row n sits at byte 128 n of the code
 // slot; key n, column half h lands at (n / 8) * 2048 + h * 1024 + (n % 8) * 128
 // with 16-byte chunk q at q ^ (n % 8), as the pool's boxes lay out pool pages.
@@ -457,16 +458,16 @@ __device__ void d_converter(uint8_t* smem_kv, const uint8_t* smem_code, DBar& ba
     uint8_t* tile = smem_kv + slot * kTileBytes;
     const uint8_t* codes = smem_code + cs * kCodeSlotBytes;
 #pragma unroll 1
-    for (int a = 32 * c; a < 32 * c + 32; a += 16) {
+    for (int a = 16 * c; a < 16 * c + 16; a += 8) {
       const int p = a >> geo.ps_shift;
       if (!((mask >> p) & 1u)) continue;
       const float sc = q8.scale[cs][p];
-      uint4 v[4];
+      uint4 v[2];
 #pragma unroll
-      for (int q = 0; q < 4; ++q)
+      for (int q = 0; q < 2; ++q)
         v[q] = *reinterpret_cast<const uint4*>(codes + (a + q * 4 + (lane >> 3)) * 128 + u * 16);
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
+      for (int q = 0; q < 2; ++q) {
         const int n = a + q * 4 + (lane >> 3);
         uint4 lo, hi;
         q8_dequant16(v[q], sc, lo, hi);
@@ -943,7 +944,7 @@ __global__ void __launch_bounds__(kQ8 ? kThreadsQ8 : kThreads, 1)
 
   if (kQ8) {
     // warpgroups: roles, softmax, converters
-    if (warp < 4) regs_dec<kRegsRolesQ8>();
+    if (warp < 4) regs_dec<kRegsRolesQ8>();  // (no change at a 128-register launch)
     else if (warp < 8) regs_inc<kRegsSoftmaxQ8>();
     else regs_dec<kRegsConvQ8>();
   }
