@@ -41,3 +41,25 @@ class Q8Case:
         for l in range(w.L):
             oracle.kv_append(pool, l, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
         return pool
+
+
+def all_pages_case(w):
+    """Every page of every request (the new tokens' too, the last one partly
+    filled) in the 8-bit image, made by the oracle from the pool after the
+    append; returns (image, block ids, q8 table, oracle pool)."""
+    pool = w.empty_pool()
+    if w.prefix_blocks().size:
+        oracle.kv_restore(pool, w.host_src(), w.prefix_blocks())
+    k, v = w.kv_new()
+    oracle.kv_append(pool, 0, k, v, w.block_table, w.prefix_lens, w.cu_new_lens)
+    table = np.full((w.B, w.max_blocks), -1, dtype=np.int32)
+    ids = []
+    for b in range(w.B):
+        nb = -(-int(w.total_lens[b]) // w.ps)
+        table[b, :nb] = np.arange(len(ids), len(ids) + nb)
+        ids.extend(w.block_table[b, :nb].tolist())
+    ids = np.asarray(ids, dtype=np.int32)
+    img = oracle.kv_save_q8(pool, ids)
+    ref_pool = w.empty_pool()
+    oracle.kv_restore_q8(ref_pool, img, ids)
+    return img, ids, table, ref_pool

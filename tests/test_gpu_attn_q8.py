@@ -15,7 +15,7 @@ from paper_2505_23970_gb300 import binding as gcb
 from paper_2505_23970_gb300 import workloads as wl
 from paper_2505_23970_gb300.harness import DeviceBatch, _i32
 
-from ._q8 import Q8Case
+from ._q8 import Q8Case, all_pages_case
 from ._util import assert_attn_close, gather_rows, sample_rows
 
 pytestmark = pytest.mark.gpu
@@ -211,3 +211,33 @@ def test_q8_host_checks():
         assert e.value.status == gcb.GC_ERR_INVALID_ARG
     torch.cuda.synchronize()
     db.close()
+
+
+@pytest.mark.parametrize("d", [128, 64])
+def test_q8_every_page_from_the_image(d):
+    """Sequences that end inside an image page: V rows past the end are
+    zeroed by the converters (the pool holds NaN everywhere), keys past the
+    end are masked; bit-exact against restore + attention."""
+    import torch
+    w = wl.custom(f"q8-allimg-d{d}", 4, 16, 2, d, 16, [300, 0, 77, 640], [70, 45, 3, 129],
+                  seed=17 + d)
+    img, ids, table, ref_pool = all_pages_case(w)
+    db = DeviceBatch(w, with_restore=False)
+    dimg = torch.from_numpy(img).cuda()
+    gcb.gc_prefix_prefill_attn_q8(db.q, db.pool.handle, db.block_table, db.prefix_lens,
+                                  db.new_lens, db.out, None, 0, db.cu_new_lens, w.B,
+                                  w.max_blocks, w.Hq, w.scale, w.T_new, dimg,
+                                  _i32(table, "cuda"), int(ids.size), 0)
+    assert db.check() == gcb.GC_OK
+    out = db.out.clone()
+    db.close()
+    db = DeviceBatch(w, with_restore=False)
+    gcb.gc_kv_restore_q8(db.pool.handle, dimg, _i32(ids, "cuda"), int(ids.size), 0, w.L, None,
+                         None, gcb.GC_RESTORE_SRC_DEVICE)
+    db.attn()
+    assert db.check() == gcb.GC_OK
+    assert _bits_equal(out, db.out)
+    db.close()
+    ref = oracle.prefix_attn(w.q(), ref_pool, 0, w.block_table, w.prefix_lens, w.cu_new_lens,
+                             w.scale)
+    assert_attn_close(out.to(torch.float64).cpu().numpy(), ref, f"{w.name} [q8, all pages]")

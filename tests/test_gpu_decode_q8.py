@@ -15,7 +15,7 @@ from paper_2505_23970_gb300 import binding as gcb
 from paper_2505_23970_gb300 import workloads as wl
 from paper_2505_23970_gb300.harness import DeviceBatch, _i32
 
-from ._q8 import Q8Case
+from ._q8 import Q8Case, all_pages_case
 from ._util import assert_attn_close
 
 pytestmark = pytest.mark.gpu
@@ -189,4 +189,26 @@ def test_q8_decode_host_checks():
                                         table, 1, flags)
         assert e.value.status == gcb.GC_ERR_INVALID_ARG
     torch.cuda.synchronize()
+    db.close()
+
+
+@pytest.mark.parametrize("d", [128, 64])
+def test_q8_decode_every_page_from_the_image(d):
+    """The page holding the new token also read from the image: the context
+    ends inside an image page (V rows past it zeroed, keys masked)."""
+    import torch
+    w = wl.custom(f"q8dec-allimg-d{d}", 4, 16, 2, d, 16, [300, 0, 76, 639], [1] * 4,
+                  seed=19 + d)
+    img, ids, table, ref_pool = all_pages_case(w)
+    db = DeviceBatch(w, with_restore=False)
+    seq = _i32(w.total_lens, "cuda")
+    ws, need = _workspace(db)
+    gcb.gc_paged_decode_attn_q8(db.q, db.pool.handle, db.block_table, seq, db.out, None, 0, w.B,
+                                w.max_blocks, w.Hq, w.scale, ws, need,
+                                torch.from_numpy(img).cuda(), _i32(table, "cuda"),
+                                int(ids.size), 0)
+    assert db.check() == gcb.GC_OK
+    ref = oracle.prefix_attn(w.q(), ref_pool, 0, w.block_table, w.prefix_lens, w.cu_new_lens,
+                             w.scale)
+    assert_attn_close(db.out.to(torch.float64).cpu().numpy(), ref, f"{w.name} [q8 decode]")
     db.close()
