@@ -744,6 +744,21 @@ def bench_configs(args, pk):
     peak_t, peak_h = pk["bf16_tflops"], pk["hbm_gbs"]
     res = {}
     flush_buf = torch.empty(512 * 2**20, dtype=torch.uint8, device=dev)
+    # the host link's reference rate: best of 3 pinned 256 MB host -> device
+    # cudaMemcpyAsync calls on the bench stream
+    link_h = torch.empty(256 * 2**20, dtype=torch.uint8).pin_memory()
+    link_d = torch.empty_like(link_h, device=dev)
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    link_ms = []
+    for _ in range(3):
+        a.record(stream)
+        memcpy_async(link_d, link_h, link_h.numel(), 1, stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        link_ms.append(a.elapsed_time(b))
+    link_gbs = link_h.numel() / (min(link_ms) / 1e3) / 1e9
+    del link_h, link_d
     for name in CONFIG_SET:
         t_cfg = time.perf_counter()
         w = make_workload(name, args.seed)
@@ -870,6 +885,10 @@ def bench_configs(args, pk):
             "e2e_tok_per_s": w.T_new / (e2e_ms / 1e3), "e2e_ms_per_step": e2e_ms,
             "e2e_h2d_bytes_per_step": int((q.numel() + 2 * k_new.numel()) * 2 + payload),
             "e2e_d2h_bytes_per_step": int(out.numel() * 2),
+            "e2e_h2d_gbs": ((q.numel() + 2 * k_new.numel()) * 2 + payload) / (e2e_ms / 1e3) / 1e9,
+            "e2e_h2d_frac_link": (((q.numel() + 2 * k_new.numel()) * 2 + payload) /
+                                  (e2e_ms / 1e3) / 1e9 / link_gbs),
+            "link_h2d_gbs": link_gbs,
             "l2": "flushed between steps" if flush else "inputs larger than L2",
             "device_status_ok": ok, "wall_s": time.perf_counter() - t_cfg}
         del q_h, k_h, v_h, img_h, out_h, q, k_new, v_new, img, out
@@ -1087,16 +1106,19 @@ def bench_ttft80(args, image=None):
     reps = 5
 
     def timed(fn):
+        """Median over `reps` runs, each bracketed by its own events (the
+        host link is shared with other jobs on the machine, and one slow
+        run should not move the figure)."""
         for _ in range(2):
             fn()
-        a = torch.cuda.Event(enable_timing=True)
-        b = torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for _ in range(reps):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(reps)]
+        for a, b in evs:
+            a.record(stream)
             fn()
-        b.record(stream)
+            b.record(stream)
         torch.cuda.synchronize()
-        return a.elapsed_time(b) / reps
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
 
     def restore_layers():
         for l in range(w.L):
@@ -1162,7 +1184,8 @@ def bench_ttft80(args, image=None):
         "schedule": "pipelined: every layer's host->device copy on a copy stream up front, "
                     "layer l's scatter + append + attention on the compute stream after "
                     "layer l's copy event; pipelined_side_restore: one staged "
-                    "restore_layers call per layer on a side stream",
+                    "restore_layers call per layer on a side stream; each figure the "
+                    "median of 5 runs, each run timed by its own events",
         "device_status_ok": ok, "ms": ms, "trace": trace,
         "restore_hidden_frac": hidden / restore_ms,
         "pipelined_over_bound": ms["pipelined"] / max(ms["stage_only"], ms["prefill_only"]),
