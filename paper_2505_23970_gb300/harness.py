@@ -328,6 +328,24 @@ class LayerStack:
             if trace is not None:
                 trace["computed"][l].record(main)
 
+    def capture(self, pipelined: bool = True, schedule: str = "copy-stream"):
+        """Record one run() into a CUDA graph (torch.cuda.CUDAGraph) after one
+        eager run on the capture's side stream; replay() then re-issues every
+        copy, kernel and event dependency of the whole layer stack with one
+        launch, so the host's per-call cost and jitter leave the step.  The
+        graph reuses this stack's buffers: its inputs are whatever they hold
+        at replay time."""
+        import torch
+        side = torch.cuda.Stream(device=self.device)
+        side.wait_stream(torch.cuda.current_stream(self.device))
+        with torch.cuda.stream(side):
+            self.run(pipelined=pipelined, schedule=schedule)
+        torch.cuda.current_stream(self.device).wait_stream(side)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            self.run(pipelined=pipelined, schedule=schedule)
+        return graph
+
     def prefill_only(self):
         """Append + attention of every layer (the compute half alone)."""
         import torch

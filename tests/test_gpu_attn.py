@@ -444,3 +444,36 @@ def test_pair_kernel_bad_block_table_entry_is_reported_not_faulted():
     db.attn()
     assert db.check() == gcb.GC_ERR_OUT_OF_RANGE
     db.close()
+
+
+@pytest.mark.parametrize("q8", [False, True])
+def test_layer_pipeline_captured_in_a_cuda_graph(q8):
+    """The copy-stream layer pipeline recorded into a CUDA graph and replayed
+    gives the eager run's pool and outputs bit for bit."""
+    import torch
+    from paper_2505_23970_gb300.harness import LayerStack
+    w = wl.custom("layers-graph", 2, 16, 2, 128, 16, [520, 47], [40, 129], seed=16)
+    w.L = 3
+    eager = LayerStack(w, keep_outputs=True)
+    if q8:
+        eager.restore_all(None)
+        eager.use_q8()
+    eager.run(pipelined=True)
+    torch.cuda.synchronize()
+    assert eager.check() == gcb.GC_OK
+    graphed = LayerStack(w, keep_outputs=True)
+    if q8:
+        graphed.restore_all(None)
+        graphed.use_q8()
+    g = graphed.capture(pipelined=True)
+    for o in graphed.outs:
+        o.fill_(float("nan"))
+    graphed.pool.planes().view(torch.int16).fill_(0x7FC0)
+    g.replay()
+    torch.cuda.synchronize()
+    assert graphed.check() == gcb.GC_OK
+    assert np.array_equal(eager.pool_bits(), graphed.pool_bits())
+    for a, b in zip(eager.outs, graphed.outs):
+        assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+    eager.close()
+    graphed.close()
