@@ -477,3 +477,31 @@ def test_layer_pipeline_captured_in_a_cuda_graph(q8):
         assert torch.equal(a.view(torch.int16), b.view(torch.int16))
     eager.close()
     graphed.close()
+
+
+# ------------------------------------------------------- the largest batch
+def _max_batch_workload(seed):
+    rng = np.random.default_rng(seed)
+    B = 8192
+    P = rng.integers(0, 40, size=B)
+    n = rng.integers(0, 4, size=B)
+    return wl.custom(f"batch-8192-{seed}", B, 4, 2, 128, 16, P, n, seed=seed)
+
+
+@pytest.mark.parametrize("kernel", ["one-sm", "pairs"])
+def test_largest_batch(kernel):
+    """8192 requests, the most one call takes (the unit table then fills
+    the shared memory both kernels have left), on the one-SM kernel and on SM
+    pairs; 8193 requests are refused before anything is launched."""
+    w = _max_batch_workload(41)
+    if kernel == "pairs":
+        on_pair_kernel(w)
+    full_parity(w)
+    import torch
+    dummy = torch.zeros(16, dtype=torch.int32, device="cuda")
+    pool = gcb.KVPool.create(1, 2, 128, 16, 4)
+    with pytest.raises(gcb.GcError) as e:
+        gcb.gc_prefix_prefill_attn(dummy, pool.handle, dummy, dummy, dummy, dummy, None, 0, dummy,
+                                   8193, 1, 4, 0.1, 16)
+    assert e.value.status == gcb.GC_ERR_UNSUPPORTED
+    pool.close()

@@ -241,3 +241,13 @@ def test_q8_every_page_from_the_image(d):
     ref = oracle.prefix_attn(w.q(), ref_pool, 0, w.block_table, w.prefix_lens, w.cu_new_lens,
                              w.scale)
     assert_attn_close(out.to(torch.float64).cpu().numpy(), ref, f"{w.name} [q8, all pages]")
+
+
+def test_q8_largest_batch():
+    """8192 requests through the 16-warp variant (its 8-bit state sits after
+    the unit table in shared memory)."""
+    rng = np.random.default_rng(43)
+    B = 8192
+    w = wl.custom("q8-batch-8192", B, 4, 2, 128, 16, rng.integers(0, 80, size=B),
+                  rng.integers(0, 4, size=B), seed=43)
+    full_q8_parity(w)
