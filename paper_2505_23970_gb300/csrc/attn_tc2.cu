@@ -68,7 +68,10 @@ constexpr int kRing = 4;              // slots of 16 KB in each of the K and V r
 constexpr int kSlotBytes = 16384;
 constexpr int kQBytes = kRows * kD * 2;  // 32 KB: two 64-column blocks of 128 rows
 constexpr int kSortMax = 512;
-constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
+// tensor memory: three S buffers of 128 columns (each half-row's P is written
+// over the first 32 of its own 64 S columns), O after them
+constexpr int kSBufs = 3;
+constexpr uint32_t kColS = 0, kColO = kSBufs * 128;
 constexpr uint32_t kIdescQK = idesc_bf16_f32(256, kKeys, false, false);
 constexpr uint32_t kIdescPV = idesc_bf16_f32(256, kD, false, true);
 // consumers of the work-item ring: in each CTA the V producer and the
@@ -91,16 +94,14 @@ struct Bars2 {
   uint64_t k_empty[kRing];    // the S product reading the slot done (softmax thread 0)
   uint64_t v_landed[kRing];   // the same for the V ring
   uint64_t v_full[kRing];
-  uint64_t v_empty[kRing];    // the PV product reading the slot done (softmax thread 0)
-  uint64_t s_full[2];         // S buffer computed (commit, both CTAs)
-  uint64_t s_free[2];         // even CTA: S buffer read by all softmax warps
-  uint64_t p_full[2];         // even CTA: P buffer written by all softmax warps
-  uint64_t pv_done[2];        // PV product from a P buffer done (commit, both CTAs)
+  uint64_t v_empty[kRing];    // the PV product reading the slot done (commit, both CTAs)
+  uint64_t s_full[kSBufs];    // S buffer computed (commit, both CTAs)
+  uint64_t p_full[kSBufs];    // even CTA: P written into the buffer by all softmax warps
+  uint64_t pv_done[kSBufs];   // PV product reading the buffer's P done (commit, both CTAs)
   uint64_t o_free;            // even CTA: O read by the epilogue
   uint64_t item_full[2];      // work-item ring, written by the even CTA's K producer
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: both issuers' last commits
-  uint32_t xseq[2][4];        // half-row softmax: exchanges published per warp
   int item_msg[2][8];         // a claimed item, decoded: it, b, tile, g, P, n, cu (it < 0: end)
   int v_keys[kRing];          // keys of the step in each V slot (< 128: rows past it zeroed)
   uint32_t tmem_base;
@@ -110,7 +111,7 @@ struct Bars2 {
 // Shared::cluster addresses of the barriers that live in the even CTA, and
 // of the peer's abort flag and item messages.
 struct Remote {
-  uint32_t q_full, k_full, v_full, s_free, p_full, o_free, item_empty, item_full, item_msg,
+  uint32_t q_full, k_full, v_full, p_full, o_free, item_empty, item_full, item_msg,
       abort_peer;
 };
 
@@ -445,17 +446,15 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
 
 // -------------------------------------------------------------- MMA issuers
 // Two threads of the even CTA, in different warps, issue the pair's MMAs:
-// one the S products, one the PV products.  They touch disjoint tensor
-// memory (S buffers / P buffers and O) and disjoint ring slots (K / V), so
-// they need no order between them, and a single thread issuing both (each
-// tcgen05.mma costs its issuing thread tens of cycles) could not keep the
-// tensor pipe busy.  Operand descriptors are built once per tile and
-// advanced by constant offsets.
+// one the S products, one the PV products.  Step t uses S buffer t mod 3:
+// S(t) writes it, the softmax reads it and writes P(t) over it, PV(t) reads
+// P(t) from it.  Operand descriptors are built once per tile and advanced by
+// constant offsets.
 //
-// S issuer: S(t) once K(t) is in and the softmax has read S(t-2) out of the
-// buffer (which it does first thing in step t-2), so S runs up to two steps
-// ahead of the softmax.  Frees the Q buffer by a commit after the item's last
-// S product (the softmax frees the ring slots).
+// S issuer: S(t) once K(t) is in and PV(t-3) is done (the buffer's last
+// reader), so S runs up to two steps ahead of the softmax and the softmax
+// never waits for a P buffer.  Frees the Q buffer by a commit after the
+// item's last S product (the softmax frees the K slots).
 __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Remote& rm,
                           uint32_t tmem, const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
@@ -474,10 +473,11 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
     const uint64_t dq = sdesc_sw128(q_smem + qb * kQBytes, 16, 1024);
     const uint32_t u_last = u + w.nt - 1;
     for (; ok && u <= u_last; ++u) {
-      const uint32_t sb = u & 1;
+      const uint32_t sb = u % kSBufs;
       const uint32_t slot = u % kRing;
       ok = mbar_wait(&bar.k_full[slot], (u / kRing) & 1, abortp);
-      if (ok && u >= 2) ok = mbar_wait(&bar.s_free[sb], ((u - 2) >> 1) & 1, abortp);
+      if (ok && u >= kSBufs)
+        ok = mbar_wait(&bar.pv_done[sb], ((u - kSBufs) / kSBufs) & 1, abortp);
       if (!ok) break;
       tc_fence_after();
       // K half: 8-key groups of 2 KB (the group's 8 rows of columns 0-63,
@@ -504,7 +504,8 @@ __device__ void s_issuer2(uint8_t* smem_q, uint8_t* smem_k, Bars2& bar, const Re
 
 // PV issuer: O += P(t) V(t) once the softmax has written P(t) and V(t) is
 // in; an item's first product (which overwrites O) also waits until the
-// previous item's epilogue has read O.
+// previous item's epilogue has read O.  Its commits tell both CTAs when the
+// S buffer and the V slot have been read.
 __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32_t tmem,
                            const Geom2& geo) {
   volatile int* abortp = &bar.abort_flag;
@@ -519,21 +520,24 @@ __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32
     if (it < 0) break;
     const uint32_t u_first = u, u_last = u + w.nt - 1;
     for (; ok && u <= u_last; ++u) {
-      const uint32_t pb = u & 1;
+      const uint32_t pb = u % kSBufs;
       const uint32_t slot = u % kRing;
-      ok = mbar_wait(&bar.p_full[pb], (u >> 1) & 1, abortp);
+      ok = mbar_wait(&bar.p_full[pb], (u / kSBufs) & 1, abortp);
       if (ok) ok = mbar_wait(&bar.v_full[slot], (u / kRing) & 1, abortp);
       const bool first = u == u_first;
       if (ok && first && k > 0) ok = mbar_wait(&bar.o_free, (k - 1) & 1, abortp);
       if (!ok) break;
       tc_fence_after();
       const uint64_t dv = sdesc_sw128(v_smem + slot * kSlotBytes, kSlotBytes, 1024);
-      const uint32_t a = tmem + kColP + pb * 64;
+      // P of keys [0, 64) at the buffer's column 0, of keys [64, 128) at column
+      // 64 (each half-row's own S columns); 16 keys = 8 packed columns
+      const uint32_t a = tmem + kColS + pb * 128;
 #pragma unroll
       for (int kk = 0; kk < kKeys / 16; ++kk)  // 16 keys = two 8-row groups of 1 KB
-        mma2_ts(tmem + kColO, a + kk * 8, dv + kk * (2048 >> 4), kIdescPV,
-                (!first || kk > 0) ? 1u : 0u);
+        mma2_ts(tmem + kColO, a + (kk >> 2) * 64 + (kk & 3) * 8, dv + kk * (2048 >> 4),
+                kIdescPV, (!first || kk > 0) ? 1u : 0u);
       mma2_commit_mc(&bar.pv_done[pb], 0x3);
+      mma2_commit_mc(&bar.v_empty[slot], 0x3);
     }
   }
   mma2_commit_mc(&bar.drain, 0x1);
@@ -547,8 +551,9 @@ __device__ void pv_issuer2(uint8_t* smem_v, Bars2& bar, const Remote& rm, uint32
 // w + 4 share the tensor-memory lanes of quadrant w & 3).  Each thread
 // exponentiates 64 scores per step, so a step's softmax takes about half the
 // time; the two halves of a row agree on its reference max through a
-// per-step exchange of their half-tile maxima in shared memory (a 64-thread
-// named barrier per quadrant), and add their partial sums at the end.
+// per-step exchange of their half-tile maxima in shared memory (one tagged
+// 16-bit word per row and half, polled by the partner thread), and add
+// their partial sums at the end.
 constexpr float kRescaleLog2 = 56.f;  // a term above 2^56 against the reference max
 
 // fp32 -> bf16 bits rounded toward +inf (finite and infinite inputs)
@@ -558,8 +563,19 @@ __device__ __forceinline__ uint16_t bf16_bits_ru(float x) {
   return r;
 }
 
-__device__ __forceinline__ float bf16_bits_to_f32(uint16_t b) {
-  return __uint_as_float(static_cast<uint32_t>(b) << 16);
+// bf16 bits -> 15-bit key, monotone in the value, rounded up: negative
+// values map to ~b, the others to b | 0x8000 (an order-preserving 16-bit
+// key), then half of it rounded up.  key15_to_f32 returns the value of the
+// key, at or above the input.
+__device__ __forceinline__ uint32_t bf16_key15_ru(uint16_t b) {
+  const uint32_t k = (b & 0x8000u) ? (~static_cast<uint32_t>(b) & 0xffffu) : (b | 0x8000u);
+  return min((k + 1) >> 1, 0x7fffu);
+}
+
+__device__ __forceinline__ float key15_to_f32(uint32_t k15) {
+  const uint32_t k = k15 << 1;
+  const uint32_t b = (k & 0x8000u) ? (k & 0x7fffu) : (~k & 0xffffu);
+  return __uint_as_float(b << 16);
 }
 
 
@@ -576,47 +592,44 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
   const int r = quad * 32 + lane;          // q row of this CTA's half = tensor-memory lane
   const uint32_t lane_addr = tmem + (static_cast<uint32_t>(quad * 32) << 16);
   uint32_t xn = 0;  // exchanges so far
-  volatile uint32_t* my_seq = &bar.xseq[hw][quad];
-  volatile uint32_t* other_seq = &bar.xseq[hw ^ 1][quad];
-  // The partner thread's value (same row, other half): each warp writes its
-  // 32 values, then its lane 0 publishes the exchange count; the warp spins
-  // (bounded) until the partner warp's count has caught up.  Values are
-  // double-buffered: a warp that runs ahead writes the other buffer, and
-  // cannot come back to this one before its partner has published the
-  // exchange after, which it does only once it has read this one.
-  auto exchange = [&](uint16_t v, bool& good) -> uint16_t {
-    const uint32_t xb = xn & 1;
-    xch[(xb * 2 + hw) * kRows + r] = v;
-    __syncwarp();
+  // The partner thread's 15-bit value (same row, other half).  Exchange n
+  // writes one 16-bit word, value << 1 | phase with phase = (n >> 1) & 1,
+  // into buffer n & 1 of this half, and polls (bounded) the partner's word
+  // in the same buffer until it carries that phase: one store, no fence (an
+  // aligned word cannot be seen half-written).  The word it replaces is
+  // exchange n - 2's, of the other phase.  The partner cannot overwrite a
+  // buffer before it is read: it writes exchange n + 2 only after reading
+  // exchange n + 1, which this thread writes only once its poll for
+  // exchange n has returned.  The words start with phase 1, which neither
+  // buffer's first exchange (n = 0, 1) carries.
+  auto exchange = [&](uint32_t v15, bool& good) -> uint32_t {
+    const uint32_t xb = xn & 1, phase = (xn >> 1) & 1;
+    volatile uint16_t* mine = xch + (xb * 2 + hw) * kRows + r;
+    volatile uint16_t* theirs = xch + (xb * 2 + (hw ^ 1)) * kRows + r;
+    *mine = static_cast<uint16_t>(v15 << 1 | phase);
     ++xn;
-    if (lane == 0) {
-      __threadfence_block();
-      *my_seq = xn;
-    }
+    uint32_t t = *theirs;
     bool ok_ = true;
-    const long long t0 = clock64();
-    while (*other_seq < xn) {
-      if (*abortp || clock64() - t0 > kWaitCycles) {
-        *abortp = 1;
-        ok_ = false;
-        break;
-      }
+    if ((t & 1u) != phase) {
+      const long long t0 = clock64();
+      do {
+        if (*abortp || clock64() - t0 > kWaitCycles) {
+          *abortp = 1;
+          ok_ = false;
+          break;
+        }
+        t = *theirs;
+      } while ((t & 1u) != phase);
     }
-    __threadfence_block();
     good = __all_sync(0xffffffffu, ok_);
-    return xch[(xb * 2 + (hw ^ 1)) * kRows + r];
+    return t >> 1;
   };
   uint32_t u = 0;  // global step counter
-  // One thread per CTA frees ring slots once the products that read them are
-  // known complete: K(u) when S(u) is, V(u) when PV(u) is (steps below
-  // v_released are freed).  This keeps the frees out of the tensor pipe's
-  // instruction stream, whose issue rate bounds the kernel.
+  // One thread per CTA frees K slot u once it has seen S(u) complete (V slots
+  // are freed by the PV issuer's commits).  When the softmax is at step u,
+  // PV(u - 3) is complete (S(u) was issued after it), so waits on
+  // pv_done for PV(u - 1) or PV(u - 2) cannot see a stale phase.
   const bool rel = warp == 4 && lane == 0;
-  uint32_t v_released = 0;
-  auto release_v_upto = [&](uint32_t v) {
-    if (rel)
-      for (; v_released <= v; ++v_released) mbar_arrive(&bar.v_empty[v_released % kRing]);
-  };
   bool ok = true;
   for (uint32_t k = 0; ok; ++k) {
     Item2 w;
@@ -631,10 +644,10 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     float m_run = -INFINITY, l = 0.f;
     const float sl2 = geo.scale_log2;
     for (int j = 0; j < w.nt; ++j, ++u) {
-      const uint32_t sb = u & 1;
+      const uint32_t sb = u % kSBufs;
       const uint32_t tS = lane_addr + kColS + sb * 128 + hw * 64;
-      const uint32_t tP = lane_addr + kColP + sb * 64 + hw * 32;
-      ok = wait_warp(&bar.s_full[sb], (u >> 1) & 1, abortp);
+      const uint32_t tP = tS;  // P over this half's scores, once they are in registers
+      ok = wait_warp(&bar.s_full[sb], (u / kSBufs) & 1, abortp);
       if (!ok) break;
       if (rel) mbar_arrive(&bar.k_empty[u % kRing]);
       tc_fence_after();
@@ -642,10 +655,6 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
       tmem_ld32(tS, sr[0]);
       tmem_ld32(tS + 32, sr[1]);
       tmem_wait_ld();
-      // S buffer free for S(u+2)
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive_remote(rm.s_free + 8 * sb);
       const int key0 = j * kKeys + hw * 64;
       if (key0 + 63 > kmax) {
 #pragma unroll
@@ -654,29 +663,30 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
           for (int e = 0; e < 32; ++e)
             if (key0 + c * 32 + e > kmax) sr[c][e] = __float_as_uint(-INFINITY);
       }
-      float mh0 = -INFINITY, mh1 = -INFINITY;
+      float mh[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};  // four short chains
 #pragma unroll
       for (int c = 0; c < 2; ++c)
 #pragma unroll
-        for (int e = 0; e < 32; e += 4) {
-          mh0 = fmax3(mh0, __uint_as_float(sr[c][e]), __uint_as_float(sr[c][e + 1]));
-          mh1 = fmax3(mh1, __uint_as_float(sr[c][e + 2]), __uint_as_float(sr[c][e + 3]));
-        }
-      // this half's max, rounded up to bf16 (16 bits to exchange); both
+        for (int e = 0; e < 32; e += 8)
+#pragma unroll
+          for (int x = 0; x < 4; ++x)
+            mh[x] = fmax3(mh[x], __uint_as_float(sr[c][e + 2 * x]),
+                          __uint_as_float(sr[c][e + 2 * x + 1]));
+      // this half's max, rounded up to bf16 and then to a 15-bit key; both
       // halves of the row then take the max of the same two rounded values,
       // a reference at or above the row's true tile max
-      const uint16_t mh = bf16_bits_ru(fmaxf(mh0, mh1));
-      const uint16_t mo = exchange(mh, ok);
+      const uint32_t mh_key =
+          bf16_key15_ru(bf16_bits_ru(fmaxf(fmaxf(mh[0], mh[1]), fmaxf(mh[2], mh[3]))));
+      const uint32_t mo = exchange(mh_key, ok);
       if (!ok) break;
-      const float mt = fmaxf(bf16_bits_to_f32(mh), bf16_bits_to_f32(mo)) * sl2;
+      const float mt = fmaxf(key15_to_f32(mh_key), key15_to_f32(mo)) * sl2;
       if (j == 0) {
         m_run = mt;  // first tile of the row: exact max (key 0 is always visible)
       } else if (__any_sync(0xffffffffu, mt - m_run > kRescaleLog2)) {
         // O must hold every earlier step before it is rescaled; both halves of
         // each row take the same decision from the same two maxima
-        ok = wait_warp(&bar.pv_done[(u - 1) & 1], ((u - 1) >> 1) & 1, abortp);
+        ok = wait_warp(&bar.pv_done[(u - 1) % kSBufs], ((u - 1) / kSBufs) & 1, abortp);
         if (!ok) break;
-        release_v_upto(u - 1);
         tc_fence_after();
         const float m_new = fmaxf(m_run, mt);
         const float alpha = m_new > m_run ? ex2_approx(m_run - m_new) : 1.f;
@@ -692,12 +702,6 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
         }
         l *= alpha;
         m_run = m_new;
-      }
-      // P buffer sb is free once PV(u-2) is done
-      if (u >= 2) {
-        ok = wait_warp(&bar.pv_done[sb], ((u - 2) >> 1) & 1, abortp);
-        if (!ok) break;
-        release_v_upto(u - 2);
       }
       {
         const uint64_t sc2 = f2_pack(sl2, sl2);
@@ -731,17 +735,18 @@ __device__ void softmax2h(uint32_t rank, Bars2& bar, const Remote& rm, uint32_t 
     }
     if (!ok) break;
     // ---- epilogue: O / l -> bf16 (this half's 64 columns), once the item's last PV is done
-    // the partner's partial sum, 16 bits at a time
+    // the partner's partial sum, 15 + 15 + 2 bits
     const uint32_t lb = __float_as_uint(l);
-    const uint32_t lo_hi = exchange(static_cast<uint16_t>(lb >> 16), ok);
+    const uint32_t l0 = exchange(lb >> 17, ok);
     if (!ok) break;
-    const uint32_t lo_lo = exchange(static_cast<uint16_t>(lb & 0xffffu), ok);
+    const uint32_t l1 = exchange((lb >> 2) & 0x7fffu, ok);
     if (!ok) break;
-    const float l_row = l + __uint_as_float((lo_hi << 16) | lo_lo);
+    const uint32_t l2 = exchange(lb & 3u, ok);
+    if (!ok) break;
+    const float l_row = l + __uint_as_float(l0 << 17 | l1 << 2 | l2);
     const uint32_t ul = u - 1;
-    ok = wait_warp(&bar.pv_done[ul & 1], (ul >> 1) & 1, abortp);
+    ok = wait_warp(&bar.pv_done[ul % kSBufs], (ul / kSBufs) & 1, abortp);
     if (!ok) break;
-    release_v_upto(ul);
     tc_fence_after();
     const int h = w.g * geo.G + r % geo.G;
     const float inv_l = 1.f / l_row;
@@ -790,7 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   Bars2& bar = *reinterpret_cast<Bars2*>(smem_v + kRing * kSlotBytes);
   int* item_start = reinterpret_cast<int*>(&bar + 1);  // [batch + 1]
   int16_t* order = reinterpret_cast<int16_t*>(item_start + geo.batch + 1);
-  // half-row softmax exchange area [2 buffers][2 halves][128 rows]
+  // half-row softmax exchange words [2 buffers][2 halves][128 rows]
   uint16_t* xch = reinterpret_cast<uint16_t*>(order + (geo.batch <= kSortMax ? kSortMax : 0));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
@@ -800,12 +805,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar.q_landed[i], 1);
       mbar_init(&bar.q_full[i], 2);
       mbar_init(&bar.q_empty[i], 1);
-      mbar_init(&bar.s_full[i], 1);
-      mbar_init(&bar.s_free[i], 2 * kSoftmaxWarps);
-      mbar_init(&bar.p_full[i], 2 * kSoftmaxWarps);
-      mbar_init(&bar.pv_done[i], 1);
       mbar_init(&bar.item_full[i], 1);
       mbar_init(&bar.item_empty[i], kItemConsumers);
+    }
+    for (int i = 0; i < kSBufs; ++i) {
+      mbar_init(&bar.s_full[i], 1);
+      mbar_init(&bar.p_full[i], 2 * kSoftmaxWarps);
+      mbar_init(&bar.pv_done[i], 1);
     }
     for (int s = 0; s < kRing; ++s) {
       mbar_init(&bar.k_landed[s], 1);
@@ -817,7 +823,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(&bar.o_free, 2 * kSoftmaxWarps);
     mbar_init(&bar.drain, 2);
-    for (int q = 0; q < 8; ++q) bar.xseq[q >> 2][q & 3] = 0;
     bar.abort_flag = 0;
     fence_barrier_init();
   }
@@ -830,6 +835,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc2(&bar.tmem_base, 512);
     tmem_relinquish2();
   }
+  // exchange words start with phase 1 (no exchange has been written)
+  for (int i = threadIdx.x; i < 2 * 2 * kRows; i += kThreads) xch[i] = 1;
   if (geo.batch <= kSortMax) {
     // rank requests by total length, longest first (ties by index)
     for (int b = threadIdx.x; b < geo.batch; b += kThreads) {
@@ -874,7 +881,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     rm.q_full = mapa(smem_addr(&bar.q_full[0]), lead);
     rm.k_full = mapa(smem_addr(&bar.k_full[0]), lead);
     rm.v_full = mapa(smem_addr(&bar.v_full[0]), lead);
-    rm.s_free = mapa(smem_addr(&bar.s_free[0]), lead);
     rm.p_full = mapa(smem_addr(&bar.p_full[0]), lead);
     rm.o_free = mapa(smem_addr(&bar.o_free), lead);
     rm.item_empty = mapa(smem_addr(&bar.item_empty[0]), lead);
