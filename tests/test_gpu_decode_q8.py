@@ -212,3 +212,30 @@ def test_q8_decode_every_page_from_the_image(d):
                              w.scale)
     assert_attn_close(db.out.to(torch.float64).cpu().numpy(), ref, f"{w.name} [q8 decode]")
     db.close()
+
+
+@pytest.mark.parametrize("G", [8, 2])
+def test_q8_decode_score_jump_rescales(G):
+    """Two pages late in a context whose K scales are 200x the rest: their
+    scores exceed the reference max taken from the first tile by far more than
+    the lazy-rescale threshold, so O and the sums are rescaled mid-request;
+    bit for bit the two-step path, within tolerance of the oracle on the same
+    image."""
+    import torch
+    w = wl.custom(f"q8dec-jump-G{G}", 2, 4 * G, 4, 128, 16, [2000, 700], [1, 1], seed=21 + G)
+    case = Q8Case(w)
+    for j in (100, 101):  # request 0's pages 100 and 101 (image blocks 100, 101)
+        hdr = case.img[j, 0, 0, :4 * w.Hkv].view(np.float32)
+        hdr *= 200.0
+    status, out, _ = run_decode_q8(case)
+    assert status == gcb.GC_OK
+    assert _bits_equal(out, run_restore_then_decode(case)), f"{w.name}: differs"
+    ref = oracle.prefix_attn(w.q(), case.oracle_pool(), 0, w.block_table, w.prefix_lens,
+                             w.cu_new_lens, w.scale)
+    assert_attn_close(out.to(torch.float64).cpu().numpy(), ref, f"{w.name} [q8 decode]")
+
+
+def test_q8_decode_one_long_request_beside_a_short_one():
+    """One request of 20000 keys (cut between several CTAs' shares, merged in
+    the kernel) next to a request of 3 keys."""
+    decode_q8_parity(wl.custom("q8dec-one-long", 2, 64, 8, 128, 16, [19999, 2], [1, 1], seed=23))
