@@ -270,8 +270,8 @@ def traffic_record(kernel: str, workload: str):
     the current kernel source."""
     import hashlib
     p = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.json")
-    src = os.path.join(ROOT, "paper_2505_23970_gb300", "csrc", "attn_tc.cu" if kernel.startswith(
-        "attn") else "kv_copy.cu")
+    src_file = {"attn_tc2": "attn_tc2.cu", "attn_tc": "attn_tc.cu"}.get(kernel, "kv_copy.cu")
+    src = os.path.join(ROOT, "paper_2505_23970_gb300", "csrc", src_file)
     if not os.path.exists(p):
         return None
     d = json.load(open(p))
@@ -512,8 +512,8 @@ def run_ours(args):
         "config": arm_config(w, world),
         "roofline": {"bound": "tensor", "achieved": attn_tflops, "peak": peak_t,
                      "unit": "TFLOP/s", "frac": attn_tflops / peak_t,
-                     "traffic": traffic_record("attn_tc", WORKLOAD),
-                     "kernel": "attn_tc_kernel<128, 0>", "peak_source": pk["source"] + " burst",
+                     "traffic": traffic_record("attn_tc2", WORKLOAD),
+                     "kernel": "attn_tc2_kernel", "peak_source": pk["source"] + " burst",
                      "frac_of_sustained": (attn_tflops / pk["bf16_tflops_sustained"]
                                            if pk.get("bf16_tflops_sustained") else None),
                      "flops_per_launch": flops, "ms_per_launch": attn_ms},
@@ -872,7 +872,7 @@ def bench_configs(args, pk):
         res[w.name] = {
             "batch": w.B, "new_tokens": w.T_new, "prefix_tokens": int(w.prefix_lens.sum()),
             "page_size": w.ps,
-            "attn_kernel": ("attn_tc2_kernel (CTA pairs)" if w.d == 128 and w.max_blocks * w.ps >= 65536
+            "attn_kernel": ("attn_tc2_kernel (CTA pairs)" if w.d == 128
                             else f"attn_tc_kernel<{w.d}>"),
             "steps": steps, "ms_per_step": ms, "tok_per_s": w.T_new / (ms / 1e3),
             "attn_ms": at_ms, "attn_tflops": at_tf, "attn_frac_burst": at_tf / peak_t,

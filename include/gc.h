@@ -337,11 +337,9 @@ GC_API gc_status gc_kv_append(gc_kv_pool* pool, const void* k_new, const void* v
  *   total_new_tokens  T_new = cu_new_lens[batch], passed from the host; it
  *               bounds every q / out row access.  A request whose rows would
  *               pass it is skipped and recorded as GC_ERR_OUT_OF_RANGE.
- *   Kernels (head_dim 128): a call whose block table can describe contexts
- *   of 65536 tokens or more (max_blocks_per_seq * page_size >= 65536) runs
- *   on pairs of SMs (tcgen05 cta_group::2, each K/V tile split between the
- *   two SMs); other calls run one work item per SM.  Both compute the same
- *   operation to the same tolerance.
+ *   Kernels: head_dim 128 runs on pairs of SMs (tcgen05 cta_group::2, each
+ *   K/V tile split between the two SMs); head_dim 64 runs one work item per
+ *   SM.  Both compute the same operation to the same tolerance.
  *   Size limit: the kernel numbers its work items (a kv head of a request
  *   and 256 of its q rows) with 32-bit ints, so T_new * (Hq/Hkv) + 256 and
  *   Hkv * (T_new * (Hq/Hkv) / 256 + batch) + 2 * (SM count) must both stay
@@ -390,11 +388,14 @@ GC_API gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool*
 
 /* Prefill over a context whose cached pages stay in the 8-bit cache tier
  * (Sec. 6.1: the 70B runs keep the KV in INT8; Sec. 3.2: an 8-bit tier
- * halves what storage holds and what a restore moves).  The result is
- * exactly that of gc_kv_restore_q8 of the 8-bit pages into the pool
- * followed by gc_prefix_prefill_attn, but the pages are never written to
- * the pool: the kernel dequantises each one (x' = bf16_rne(c * s), the
- * restore's rounding) into the tile it would have loaded.
+ * halves what storage holds and what a restore moves).  The operation is
+ * gc_kv_restore_q8 of the 8-bit pages into the pool followed by
+ * gc_prefix_prefill_attn, but the pages are never written to the pool: the
+ * kernel dequantises each one (x' = bf16_rne(c * s), the restore's
+ * rounding) into the tile it would have loaded.  At head_dim 64 the result
+ * is bit-identical to those two calls (both run on the one-SM kernel); at
+ * head_dim 128 gc_prefix_prefill_attn runs on SM pairs, whose sums run in
+ * another order, and the two agree within the attention tolerance.
  * Arguments as gc_prefix_prefill_attn, plus:
  *   q8_image   device memory, 16-byte aligned: the 8-bit image
  *              [n_image_blocks][L][2][gc_kv_q8_chunk_bytes], or with

@@ -1145,18 +1145,14 @@ gc_status launch(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
   return GC_OK;
 }
 
-// head_dim 128: contexts of up to kPairMinKeys tokens run on the single-SM
-// kernel above; calls whose block table can describe longer contexts run on
-// the CTA-pair kernel (attn_tc2.cu), which is faster when every work item
-// spans hundreds of K/V steps (measured on the 131072-token document layer)
-// and slower when items are short (its per-item start-up is longer).
-constexpr long long kPairMinKeys = 65536;
-
+// head_dim 128 prefill runs on the CTA-pair kernel (attn_tc2.cu): measured
+// faster than the single-SM kernel above on every layer shape (70B layer 1.50
+// against 1.95 ms, Llama-3-8B layer 0.173 against 0.205 ms, the conversation
+// mix and the long document alike).  The single-SM kernel serves head_dim
+// 64, pages read from the 8-bit image and decode at head_dim 64.
 gc_status launch_d128(const gc_kv_pool* pool, const AttnArgs& a, cudaStream_t stream,
                       int* work_counter) {
-  if (static_cast<long long>(a.max_blocks) * pool->cfg.page_size >= kPairMinKeys)
-    return launch_attn_tc2(pool, a, stream, work_counter);
-  return launch<128>(pool, a, stream, work_counter);
+  return launch_attn_tc2(pool, a, stream, work_counter);
 }
 
 }  // namespace

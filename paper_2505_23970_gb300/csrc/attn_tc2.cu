@@ -86,14 +86,13 @@ struct Geom2 {
 };
 
 struct Bars2 {
-  uint64_t q_landed[2];       // this CTA's Q half copied (tx)
-  uint64_t q_full[2];         // even CTA: both Q halves landed (2 forwards)
+  uint64_t q_full[2];         // even CTA: both Q halves landed (2 arrivals + both copies' bytes)
   uint64_t q_empty[2];        // the item's last S product done (commit, both CTAs)
-  uint64_t k_landed[kRing];   // this CTA's K slot copied (tx)
-  uint64_t k_full[kRing];     // even CTA: both K halves of the slot ready (2 forwards)
+  uint64_t k_landed[kRing];   // (unused: K copies always complete on k_full)
+  uint64_t k_full[kRing];     // even CTA: both K halves of the slot landed (2 arrivals + bytes)
   uint64_t k_empty[kRing];    // the S product reading the slot done (softmax thread 0)
-  uint64_t v_landed[kRing];   // the same for the V ring
-  uint64_t v_full[kRing];
+  uint64_t v_landed[kRing];   // this CTA's V half of an item's last, partial step (tx)
+  uint64_t v_full[kRing];     // even CTA: both V halves of the slot ready (2 arrivals + bytes)
   uint64_t v_empty[kRing];    // the PV product reading the slot done (commit, both CTAs)
   uint64_t s_full[kSBufs];    // S buffer computed (commit, both CTAs)
   uint64_t p_full[kSBufs];    // even CTA: P written into the buffer by all softmax warps
@@ -103,7 +102,6 @@ struct Bars2 {
   uint64_t item_empty[2];     // even CTA: item slot read by every consumer of both CTAs
   uint64_t drain;             // even CTA: both issuers' last commits
   int item_msg[2][8];         // a claimed item, decoded: it, b, tile, g, P, n, cu (it < 0: end)
-  int v_keys[kRing];          // keys of the step in each V slot (< 128: rows past it zeroed)
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -215,101 +213,39 @@ __device__ __forceinline__ void raise_abort(Bars2& bar, const Remote& rm) {
 // copies in parallel (a copy instruction costs its warp tens of cycles per
 // box, and 16-token pages need many boxes).
 //
-// Each producer also reports its own copies, in order, to the even CTA once
-// they have landed (a V slot whose step ends past the sequence gets its tail
-// rows zeroed first: their P is 0, but 0 * NaN is NaN).  It does so whenever
-// it would otherwise wait, so a slot can never wait on a report that the
-// producer, blocked on that slot, has not made.
+// Both CTAs' copies for a ring slot (or a Q buffer) complete on the even
+// CTA's full barrier: each producer arrives there once per use with the bytes
+// of its own copies (arrive.expect_tx) and issues them with pair completion,
+// so the phase ends once both halves have landed and no copy has to be
+// watched and reported (watching and reporting every landed copy made the V
+// producer the slowest stage of the pipeline).  The exception is a V step
+// that ends before 128 keys (an item's last): its rows past the end must be
+// zeroed once they have landed (their P is 0, but 0 * NaN is NaN), so that
+// copy completes on this CTA's own landed barrier, the producer waits for it,
+// zeroes the rows and then arrives on the full barrier.
 template <bool kIsK>
 struct Producer {
-  Bars2& bar;
-  const Remote& rm;
   uint8_t* ring;         // kRing slots of 16 KB
-  uint64_t* landed;      // this CTA's landed barriers of the ring
+  uint64_t* landed;      // this CTA's landed barriers of the ring (partial V steps)
   uint64_t* empty;
-  uint32_t full_remote;  // even CTA's full barriers of the ring
+  uint32_t full_cl;      // shared::cluster address of the even CTA's full barrier 0
   volatile int* abortp;
   int lane;
-  uint32_t issued = 0, fwd = 0;      // ring uses issued / reported
-  uint32_t q_issued = 0, q_fwd = 0;  // K producer: Q halves issued / reported
+  uint32_t issued = 0;   // ring uses issued
+  uint32_t lphase = 0;   // per slot: parity of the slot's next landed phase
 
-  // lane 0's probe of a barrier phase, for the whole warp
-  __device__ __forceinline__ bool probe(uint64_t* b, uint32_t parity) {
-    const bool t = lane == 0 ? mbar_test(b, parity) : false;
-    return __shfl_sync(0xffffffffu, t, 0);
+  // bounded wait of the whole warp (the lanes agree on the outcome)
+  __device__ __forceinline__ bool wait(uint64_t* b, uint32_t parity) {
+    return wait_warp(b, parity, abortp);
   }
 
-  // Report landed copies in order; with `block`, wait (bounded) for all of
-  // them.  Returns false if the wait gave up.
-  __device__ bool forward(bool block) {
-    const long long t0 = clock64();
-    while (true) {
-      bool progress = false;
-      if (kIsK && q_fwd < q_issued) {
-        const uint32_t qb = q_fwd & 1;
-        if (probe(&bar.q_landed[qb], (q_fwd >> 1) & 1)) {
-          if (lane == 0) mbar_arrive_remote(rm.q_full + 8 * qb);
-          ++q_fwd;
-          progress = true;
-        }
-      }
-      if (fwd < issued) {
-        const uint32_t slot = fwd % kRing;
-        if (probe(&landed[slot], (fwd / kRing) & 1)) {
-          bool zeroed = false;
-          if (!kIsK) {
-            const int nkeys = bar.v_keys[slot];
-            if (nkeys < kKeys) {
-              uint4* z = reinterpret_cast<uint4*>(ring + slot * kSlotBytes + nkeys * 128);
-              for (int e = lane; e < (kKeys - nkeys) * 8; e += 32) z[e] = make_uint4(0, 0, 0, 0);
-              fence_proxy_async_smem();
-              zeroed = true;
-            }
-          }
-          __syncwarp();
-          // zeroed rows are generic-proxy writes the other SM's tensor core
-          // reads: publish them at cluster scope; a plain landed copy needs none
-          if (lane == 0) {
-            if (zeroed) mbar_arrive_cluster(full_remote + 8 * slot);
-            else mbar_arrive_remote(full_remote + 8 * slot);
-          }
-          ++fwd;
-          progress = true;
-        }
-      }
-      const bool done = fwd == issued && (!kIsK || q_fwd == q_issued);
-      if (done || (!block && !progress)) return true;
-      if (*abortp) return false;
-      if (clock64() - t0 > kWaitCycles) {
-        *abortp = 1;
-        return false;
-      }
-    }
-  }
-
-  // Wait (bounded) for a barrier phase, reporting landed copies meanwhile.
-  __device__ bool wait(uint64_t* b, uint32_t parity) {
-    const long long t0 = clock64();
-    while (!probe(b, parity)) {
-      if (!forward(false)) return false;
-      if (*abortp) return false;
-      if (clock64() - t0 > kWaitCycles) {
-        *abortp = 1;
-        return false;
-      }
-    }
-    return true;
-  }
-
-  // Copies in flight when the kernel gives up land before the CTA exits
-  // (bounded, ignores the abort flag).
+  // Copies still in flight when the kernel gives up land before the CTA exits:
+  // their completion goes to the even CTA's barriers, so wait out a time far
+  // above a copy's latency (about 60 us).
   __device__ void drain() {
-    if (lane != 0) return;
-    int no_abort = 0;
-    for (uint32_t q = q_fwd; kIsK && q < q_issued; ++q)
-      mbar_wait(&bar.q_landed[q & 1], (q >> 1) & 1, &no_abort);
-    for (uint32_t x = fwd; x < issued; ++x)
-      mbar_wait(&landed[x % kRing], (x / kRing) & 1, &no_abort);
+    const long long t0 = clock64();
+    while (clock64() - t0 < (1ll << 17)) {
+    }
   }
 };
 
@@ -323,7 +259,7 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
                           const int32_t* __restrict__ cu_new_lens, int32_t* status,
                           int* work_counter) {
   const int lane = threadIdx.x & 31;
-  Producer<kIsK> pr{bar, rm, smem_ring, kIsK ? bar.k_landed : bar.v_landed,
+  Producer<kIsK> pr{smem_ring, kIsK ? bar.k_landed : bar.v_landed,
                     kIsK ? bar.k_empty : bar.v_empty, kIsK ? rm.k_full : rm.v_full,
                     &bar.abort_flag, lane};
   bool ok = true;
@@ -383,13 +319,14 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
       ok = pr.wait(&bar.q_empty[qb], ((k >> 1) & 1) ^ 1);
       if (!ok) break;
       if (lane == 0) {
-        mbar_arrive_expect_tx(&bar.q_landed[qb], kQBytes);
+        const uint32_t qf = rm.q_full + 8 * qb;
+        mbar_arrive_expect_tx_remote(qf, kQBytes);
 #pragma unroll
         for (int h = 0; h < 2; ++h)
-          tma_load_3d(smem_q + qb * kQBytes + h * (kRows * 128), map_q, &bar.q_landed[qb],
-                      h * 64, w.g * geo.G, w.cu + w.tok0);
+          tma_load_3d_pair(smem_q + qb * kQBytes + h * (kRows * 128), map_q, qf, h * 64,
+                           w.g * geo.G, w.cu + w.tok0);
       }
-      ++pr.q_issued;
+      __syncwarp();
     }
     // K/V steps.  Lane i holds the block-table entry of page i of a step
     // (-2: no such page before the end of the sequence); the next step's
@@ -422,25 +359,40 @@ __device__ void producer2(uint32_t rank, uint8_t* smem_q, uint8_t* smem_ring, Ba
       const uint32_t x = pr.issued, slot = x % kRing;
       ok = pr.wait(&pr.empty[slot], ((x / kRing) & 1) ^ 1);
       if (!ok) break;
-      if (lane == 0) {
-        if (!kIsK) bar.v_keys[slot] = min(kKeys, w.T - key0);
-        mbar_arrive_expect_tx(&pr.landed[slot], static_cast<uint32_t>(good) * box_bytes);
-      }
-      __syncwarp();
+      const uint32_t full = pr.full_cl + 8 * slot;
+      const uint32_t bytes = static_cast<uint32_t>(good) * box_bytes;
       uint8_t* dst = smem_ring + slot * kSlotBytes + lane * box_bytes;
-      if (row >= 0) {
-        if (kIsK)
-          tma_load_4d(dst, map_kv, &pr.landed[slot], 0, 0, 0, row >> 3);
-        else
-          tma_load_2d(dst, map_kv, &pr.landed[slot], static_cast<int>(rank) * 64, row);
+      const int nkeys = min(kKeys, w.T - key0);
+      if (kIsK || nkeys == kKeys) {
+        if (lane == 0) mbar_arrive_expect_tx_remote(full, bytes);
+        __syncwarp();
+        if (row >= 0) {
+          if (kIsK)
+            tma_load_4d_pair(dst, map_kv, full, 0, 0, 0, row >> 3);
+          else
+            tma_load_2d_pair(dst, map_kv, full, static_cast<int>(rank) * 64, row);
+        }
+      } else {
+        // an item's last V step: land here, zero the rows past the end, report
+        const uint32_t par = (pr.lphase >> slot) & 1u;
+        pr.lphase ^= 1u << slot;
+        if (lane == 0) mbar_arrive_expect_tx(&pr.landed[slot], bytes);
+        __syncwarp();
+        if (row >= 0) tma_load_2d(dst, map_kv, &pr.landed[slot], static_cast<int>(rank) * 64, row);
+        ok = pr.wait(&pr.landed[slot], par);
+        if (!ok) break;
+        uint4* z = reinterpret_cast<uint4*>(smem_ring + slot * kSlotBytes + nkeys * 128);
+        for (int e = lane; e < (kKeys - nkeys) * 8; e += 32) z[e] = make_uint4(0, 0, 0, 0);
+        fence_proxy_async_smem();
+        __syncwarp();
+        // the zeroed rows are generic-proxy writes the other SM's tensor core
+        // reads: publish them at cluster scope
+        if (lane == 0) mbar_arrive_cluster(full);
       }
       ++pr.issued;
-      pr.forward(false);
       pages = pages_next;
     }
   }
-  // report every copy issued (the issuers wait for them), or drain on failure
-  if (ok) ok = pr.forward(true);
   if (!ok) pr.drain();
 }
 
@@ -802,7 +754,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&bar.q_landed[i], 1);
       mbar_init(&bar.q_full[i], 2);
       mbar_init(&bar.q_empty[i], 1);
       mbar_init(&bar.item_full[i], 1);

@@ -351,9 +351,9 @@ def test_work_item_bound_refused_before_launch():
 
 
 # ------------------------------------------------------- the CTA-pair kernel
-# head_dim 128 prefill runs on the CTA-pair kernel when the block table can
-# describe contexts of 65536 tokens or more (the long-document configs do);
-# widening a block table with unused (-1) columns routes any workload there.
+# head_dim 128 prefill runs on the CTA-pair kernel; these cases also widen
+# the block table with unused (-1) columns to a 65536-token capacity, as a
+# long-context server's tables are.
 PAIR_KEYS = 65536
 
 
@@ -480,22 +480,21 @@ def test_layer_pipeline_captured_in_a_cuda_graph(q8):
 
 
 # ------------------------------------------------------- the largest batch
-def _max_batch_workload(seed):
+def _max_batch_workload(seed, d=128):
     rng = np.random.default_rng(seed)
     B = 8192
     P = rng.integers(0, 40, size=B)
     n = rng.integers(0, 4, size=B)
-    return wl.custom(f"batch-8192-{seed}", B, 4, 2, 128, 16, P, n, seed=seed)
+    return wl.custom(f"batch-8192-{seed}-d{d}", B, 4, 2, d, 16, P, n, seed=seed)
 
 
 @pytest.mark.parametrize("kernel", ["one-sm", "pairs"])
 def test_largest_batch(kernel):
     """8192 requests, the most one call takes (the unit table then fills
-    the shared memory both kernels have left), on the one-SM kernel and on SM
-    pairs; 8193 requests are refused before anything is launched."""
-    w = _max_batch_workload(41)
-    if kernel == "pairs":
-        on_pair_kernel(w)
+    the shared memory both kernels have left), on the one-SM kernel (head_dim
+    64) and on SM pairs (head_dim 128); 8193 requests are refused before
+    anything is launched."""
+    w = _max_batch_workload(41, d=64 if kernel == "one-sm" else 128)
     full_parity(w)
     import torch
     dummy = torch.zeros(16, dtype=torch.int32, device="cuda")

@@ -4,9 +4,12 @@ The operation is defined as the 8-bit restore (Sec. 6.1 keeps the 70B KV in
 INT8) followed by prefix-reuse attention (Sec. 2.2), so the oracle is
 oracle.kv_restore_q8 of every cached page, oracle.kv_append and
 oracle.prefix_attn.  The GPU path never writes the 8-bit pages into the
-pool; it is checked bit for bit against the library's own two-step path
-(gc_kv_restore_q8 of every page, then gc_prefix_prefill_attn on the same
-one-SM kernel) and within the attention tolerance against the oracle."""
+pool; it runs on the single-SM kernel's 8-bit variant and is checked against
+the library's own two-step path (gc_kv_restore_q8 of every page, then
+gc_prefix_prefill_attn): bit for bit at head_dim 64, where that path runs on
+the same single-SM kernel, and within the attention tolerance at head_dim
+128, where it runs on SM pairs; and within the attention tolerance against
+the oracle."""
 import numpy as np
 import pytest
 
@@ -83,25 +86,38 @@ def _bits_equal(a, b):
     return torch.equal(a.view(torch.int16), b.view(torch.int16))
 
 
+def same_as_two_step(w, out, two_step, what, rows=None):
+    """Bit for bit at head_dim 64 (both on the single-SM kernel); within the
+    attention tolerance at 128 (the two-step path runs on SM pairs)."""
+    import torch
+    if w.d == 64:
+        assert _bits_equal(out, two_step), f"{what}: differs from restore + attn"
+        return
+    a = out.to(torch.float64).cpu().numpy()
+    b = two_step.to(torch.float64).cpu().numpy()
+    if rows is not None:
+        a, b = gather_rows(a, w, rows), gather_rows(b, w, rows)
+    assert_attn_close(a, b, f"{what} vs restore + attn")
+
+
 def full_q8_parity(w, **kw):
     case = Q8Case(w, **kw)
     status, out, _ = run_q8(case)
     assert status == gcb.GC_OK
-    assert _bits_equal(out, run_restore_then_attn(case)), f"{w.name}: differs from restore + attn"
+    same_as_two_step(w, out, run_restore_then_attn(case), w.name)
     import torch
     ref = oracle.prefix_attn(w.q(), case.oracle_pool(), 0, w.block_table, w.prefix_lens,
                              w.cu_new_lens, w.scale)
     return assert_attn_close(out.to(torch.float64).cpu().numpy(), ref, f"{w.name} [q8]")
 
 
-def sampled_q8_parity(w, n_random=512, bit_exact=True):
+def sampled_q8_parity(w, n_random=512):
     import torch
     case = Q8Case(w)
     status, out, _ = run_q8(case)
     assert status == gcb.GC_OK
-    if bit_exact:
-        assert _bits_equal(out, run_restore_then_attn(case)), f"{w.name}: differs"
     rows = sample_rows(w, n_random)
+    same_as_two_step(w, out, run_restore_then_attn(case), w.name, rows)
     ref = oracle.prefix_attn_rows(w.q(), case.oracle_pool(), 0, w.block_table, w.prefix_lens,
                                   w.cu_new_lens, w.scale, rows)
     got = gather_rows(out.to(torch.float64).cpu().numpy(), w, rows)
@@ -114,8 +130,8 @@ def sampled_q8_parity(w, n_random=512, bit_exact=True):
 def test_q8_shapes_ragged(G, d, ps):
     """Head groupings, both head sizes and every page size, with prefixes
     that end inside a page, a request without prefix and one without new
-    tokens: bit-exact against restore + attention, within tolerance of the
-    oracle."""
+    tokens: against restore + attention (bit for bit at head_dim 64) and
+    within tolerance of the oracle."""
     Hkv = 2
     w = wl.custom(f"q8-G{G}-d{d}-ps{ps}", 5, G * Hkv, Hkv, d, ps, [300, 0, 1000, 17, 640],
                   [70, 45, 0, 260, 129], seed=G * 7 + d + ps)
@@ -145,9 +161,8 @@ def test_q8_conversation_mix_sampled():
 
 
 def test_q8_long_document_sampled():
-    """131072 cached tokens in 64-token pages.  The all-pool path runs this
-    block table on SM pairs, so only the oracle comparison applies."""
-    sampled_q8_parity(wl.long_document(B=1), n_random=128, bit_exact=False)
+    """131072 cached tokens in 64-token pages."""
+    sampled_q8_parity(wl.long_document(B=1), n_random=128)
 
 
 @pytest.mark.parametrize("layer_major", [False, True])
@@ -159,7 +174,7 @@ def test_q8_layer_of_a_multilayer_image(layer_major):
     case = Q8Case(w)
     status, out, _ = run_q8(case, layer=1, layer_major=layer_major)
     assert status == gcb.GC_OK
-    assert _bits_equal(out, run_restore_then_attn(case, layer=1))
+    same_as_two_step(w, out, run_restore_then_attn(case, layer=1), "layer 1")
     import torch
     ref = oracle.prefix_attn(w.q(), case.oracle_pool(), 1, w.block_table, w.prefix_lens,
                              w.cu_new_lens, w.scale)
@@ -217,7 +232,8 @@ def test_q8_host_checks():
 def test_q8_every_page_from_the_image(d):
     """Sequences that end inside an image page: V rows past the end are
     zeroed by the converters (the pool holds NaN everywhere), keys past the
-    end are masked; bit-exact against restore + attention."""
+    end are masked; against restore + attention (bit for bit at head_dim 64)
+    and the oracle."""
     import torch
     w = wl.custom(f"q8-allimg-d{d}", 4, 16, 2, d, 16, [300, 0, 77, 640], [70, 45, 3, 129],
                   seed=17 + d)
@@ -236,7 +252,7 @@ def test_q8_every_page_from_the_image(d):
                          None, gcb.GC_RESTORE_SRC_DEVICE)
     db.attn()
     assert db.check() == gcb.GC_OK
-    assert _bits_equal(out, db.out)
+    same_as_two_step(w, out, db.out, w.name)
     db.close()
     ref = oracle.prefix_attn(w.q(), ref_pool, 0, w.block_table, w.prefix_lens, w.cu_new_lens,
                              w.scale)
