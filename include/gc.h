@@ -416,7 +416,10 @@ GC_API gc_status gc_prefix_prefill_attn_noalloc(const void* q, const gc_kv_pool*
  * producer loads each image page's codes into the K/V ring (TMA) and a
  * fourth warpgroup dequantises them there, while the TMA unit loads the
  * pool pages.  Shared memory limits batch to 8192 as for
- * gc_prefix_prefill_attn.
+ * gc_prefix_prefill_attn.  Every work item dequantises its own copy of the
+ * pages it reads, so with many new tokens per cached page the two-step path
+ * (gc_kv_restore_q8, then gc_prefix_prefill_attn) is faster; this call
+ * keeps no bf16 copy of the cached pages in the pool.
  * Errors: as gc_prefix_prefill_attn; GC_ERR_INVALID_ARG also for unknown
  * flags, a NULL q8_table (or q8_image with n_image_blocks > 0), a
  * misaligned q8_image. */
